@@ -1,0 +1,322 @@
+"""Pins of the CPU oracle against facts the paper and the mathematics fix.
+
+None of these tests re-types an oracle formula: each checks the oracle
+against a hand-derived closed form, a brute-force enumeration, a library
+routine (scipy / torch softmax and attention), or an invariant stated in the
+paper (Sec. 3.5 single-image limit, App. B.1 Lemma 1, App. B.2 normalisation).
+"""
+
+import itertools
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import conduit_oracle as O
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "worked_example.json")
+
+
+def _worked_inputs():
+    ex = json.load(open(GOLDEN))
+    inp = ex["inputs"]
+    w = np.array(inp["weights_w"], dtype=np.float64)
+    L, Hq, Hkv, nq, N = inp["num_layers"], inp["num_q_heads"], inp["num_kv_heads"], inp["n_q"], len(w)
+    q = np.zeros((L, Hq, nq, 1))
+    q[0, :, :, 0] = np.array(inp["queries"]["layer0"])
+    q[1, :, :, 0] = np.array(inp["queries"]["layer1"])
+    k = np.zeros((L, Hkv, N, 1))
+    k[:, 0, :, 0] = np.log(w)
+    v = np.zeros((L, Hkv, N, 1))
+    v[0, 0, :, 0] = inp["values"]["layer0"]
+    v[1, 0, :, 0] = inp["values"]["layer1"]
+    return ex, q, k, v, inp["img_off"]
+
+
+# ---------------------------------------------------------------- closed form
+def test_worked_example_scores():
+    ex, q, k, v, img_off = _worked_inputs()
+    e = ex["expected"]
+    sc = O.score_request(q, k, v, img_off)
+    np.testing.assert_allclose(sc["a"], e["a"], rtol=0, atol=1e-14)
+    np.testing.assert_allclose(sc["vn"], e["vn"], rtol=0, atol=1e-14)
+    np.testing.assert_allclose(sc["s"], e["s"], rtol=0, atol=1e-14)
+    np.testing.assert_allclose(sc["A"], e["A"], rtol=0, atol=1e-14)
+    np.testing.assert_allclose(sc["g"], e["g"], rtol=0, atol=1e-14)
+    c = O.image_coefficients(sc["g"], 1.0)
+    np.testing.assert_allclose(c, e["c_lambda1"], rtol=0, atol=1e-14)
+    np.testing.assert_allclose(O.composite_score(sc["s"], c, img_off), e["s_hat_lambda1"], rtol=0, atol=1e-14)
+
+
+@pytest.mark.parametrize("lam,key", [(1.0, "topk_lambda1"), (0.0, "topk_lambda0")])
+def test_worked_example_selection(lam, key):
+    ex, q, k, v, img_off = _worked_inputs()
+    for kk, want in ex["expected"][key].items():
+        out = O.refresh_mask(q, k, v, img_off, lam=lam, k_budget=int(kk))
+        assert out["idx"].tolist() == want
+        assert out["mask"].tolist() == [1 if t in want else 0 for t in range(4)]
+
+
+# ------------------------------------------------------------------- budget
+def test_budget_eq2():
+    assert O.budget(0.0, 1000) == 0
+    assert O.budget(1.0, 1000) == 1000
+    assert O.budget(0.10, 256) == 25          # floor(25.6)
+    assert O.budget(0.10, 1024) == 102
+    assert O.budget(0.10, 8192) == 819
+    assert O.budget(0.05, 41472) == 2073
+    assert O.budget(0.20, 41472) == 8294
+    assert O.budget(0.3, 10) == 3             # decimal ratio lands on the integer
+    assert O.budget(0.7, 10) == 7
+    with pytest.raises(ValueError):
+        O.budget(-0.1, 10)
+    with pytest.raises(ValueError):
+        O.budget(1.5, 10)
+
+
+# -------------------------------------------------- Lemma 1 brute force
+def _brute_force_topk(s_hat, k):
+    """argmin over |T| = k of sum_{t not in T} s_hat_t^2 (App. B.1, Lemma 1);
+    among minimisers the lexicographically smallest index tuple."""
+    n = len(s_hat)
+    best, best_val = None, None
+    for T in itertools.combinations(range(n), k):
+        rest = [t for t in range(n) if t not in T]
+        val = sum(s_hat[t] * s_hat[t] for t in rest)
+        if best_val is None or val < best_val:
+            best, best_val = T, val
+    return list(best)
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_topk_is_lemma1_minimiser_with_ties(seed):
+    rng = np.random.default_rng(seed)
+    n = 10
+    # small integers: exact squares and sums in fp64, many ties
+    s_hat = rng.integers(0, 5, size=n).astype(np.float64)
+    for k in range(n + 1):
+        assert O.topk_select(s_hat, k).tolist() == _brute_force_topk(s_hat.tolist(), k)
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_topk_is_lemma1_minimiser_distinct(seed):
+    rng = np.random.default_rng(100 + seed)
+    n = 11
+    s_hat = rng.random(n)
+    for k in (0, 1, 3, 5, 10, 11):
+        assert O.topk_select(s_hat, k).tolist() == _brute_force_topk(s_hat.tolist(), k)
+
+
+def test_topk_matches_library_sort():
+    rng = np.random.default_rng(7)
+    s_hat = rng.random(500)
+    k = 123
+    want = np.sort(np.argsort(-s_hat, kind="stable")[:k])
+    assert O.topk_select(s_hat, k).tolist() == want.tolist()
+    t = torch.topk(torch.from_numpy(s_hat), k).indices.sort().values
+    assert O.topk_select(s_hat, k).tolist() == t.tolist()
+
+
+# ------------------------------------------------- library softmax / GQA map
+def _rand_request(seed, L=2, Hq=6, Hkv=2, nq=5, N=37, d=8, spans=(0, 10, 25, 37)):
+    rng = np.random.default_rng(seed)
+    q = rng.standard_normal((L, Hq, nq, d))
+    k = rng.standard_normal((L, Hkv, N, d)) * 1.5
+    v = rng.standard_normal((L, Hkv, N, d)) * rng.lognormal(0, 0.5, size=(1, 1, N, 1))
+    return q, k, v, list(spans)
+
+
+def test_head_query_mean_matches_torch_softmax_with_gqa():
+    q, k, v, _ = _rand_request(1)
+    L, Hq, nq, d = q.shape
+    Hkv = k.shape[1]
+    for l in range(L):
+        kk = torch.from_numpy(k[l]).repeat_interleave(Hq // Hkv, dim=0)      # head h -> kv h // G
+        logits = torch.matmul(torch.from_numpy(q[l]), kk.transpose(-1, -2)) / math.sqrt(d)
+        alpha = torch.softmax(logits, dim=-1)                                  # over visual keys
+        want = alpha.mean(dim=(0, 1)).numpy()
+        np.testing.assert_allclose(O.head_query_mean_attention(q[l], k[l]), want, rtol=1e-12, atol=1e-15)
+
+
+def test_surrogate_special_case_eq5():
+    """L = 1, H = 1, |Q| = 1: s_t = alpha_t ||V_t|| (Eq. 5), via scipy softmax and numpy norm."""
+    scipy_special = pytest.importorskip("scipy.special")
+    rng = np.random.default_rng(3)
+    N, d = 50, 16
+    q = rng.standard_normal((1, 1, 1, d))
+    k = rng.standard_normal((1, 1, N, d)) * 2
+    v = rng.standard_normal((1, 1, N, d))
+    alpha = scipy_special.softmax(q[0, 0, 0] @ k[0, 0].T / math.sqrt(d))
+    want = alpha * np.linalg.norm(v[0, 0], axis=1)
+    sc = O.score_request(q, k, v, [0, N])
+    np.testing.assert_allclose(sc["s"], want, rtol=1e-12, atol=0)
+
+
+def test_value_norm_is_over_concatenated_heads():
+    # heads carry 3 and 4 along one axis: the concatenated norm is 5
+    v = np.zeros((2, 3, 4))
+    v[0, :, 1] = 3.0
+    v[1, :, 2] = -4.0
+    np.testing.assert_array_equal(O.value_norms(v), [5.0, 5.0, 5.0])
+    rng = np.random.default_rng(4)
+    v = rng.standard_normal((4, 9, 8))
+    want = np.linalg.norm(np.concatenate([v[g] for g in range(4)], axis=1), axis=1)
+    np.testing.assert_allclose(O.value_norms(v), want, rtol=1e-14)
+
+
+# ----------------------------------------------------- paper invariants
+def test_softmax_identities():
+    q, k, v, spans = _rand_request(5)
+    sc = O.score_request(q, k, v, spans)
+    np.testing.assert_allclose(sc["a"].sum(axis=1), 1.0, rtol=0, atol=1e-13)   # each a^(l) sums to 1
+    np.testing.assert_allclose(sc["A"].sum(), q.shape[0], atol=1e-13)           # sum_t A_t = |L|
+    n_j = np.diff(spans)
+    np.testing.assert_allclose((n_j * sc["g"]).sum(), 1.0, atol=1e-13)          # sum_j n_j g_j = 1
+
+
+def test_key_shift_invariance():
+    q, k, v, spans = _rand_request(6)
+    b = np.random.default_rng(60).standard_normal((q.shape[0], k.shape[1], 1, k.shape[3]))
+    a1 = O.score_request(q, k, v, spans)
+    a2 = O.score_request(q, k + b, v, spans)
+    np.testing.assert_allclose(a2["a"], a1["a"], rtol=1e-10, atol=1e-15)
+    np.testing.assert_allclose(a2["s"], a1["s"], rtol=1e-10, atol=1e-15)
+
+
+def test_value_scale_equivariance():
+    q, k, v, spans = _rand_request(7)
+    r1 = O.refresh_mask(q, k, v, spans, k_budget=9)
+    r2 = O.refresh_mask(q, k, 3.5 * v, spans, k_budget=9)
+    np.testing.assert_allclose(r2["s"], 3.5 * r1["s"], rtol=1e-13)
+    assert r2["idx"].tolist() == r1["idx"].tolist()
+
+
+def test_zero_value_norm_gives_zero_score():
+    q, k, v, spans = _rand_request(8)
+    v[:, :, [3, 11, 30], :] = 0.0
+    sc = O.score_request(q, k, v, spans)
+    assert sc["s"][3] == 0.0 and sc["s"][11] == 0.0 and sc["s"][30] == 0.0
+    assert (sc["s"][[0, 1, 2]] > 0).all()
+
+
+def test_uniform_norm_reproduces_raw_attention_ranking():
+    """Drop-||V|| ablation (Table 5): a uniform norm ranks by attention alone."""
+    q, k, v, _ = _rand_request(9)
+    N = k.shape[2]
+    rng = np.random.default_rng(90)
+    z = rng.standard_normal(v.shape)
+    zc = np.transpose(z, (0, 2, 1, 3)).reshape(z.shape[0], N, -1)
+    zc = zc / np.linalg.norm(zc, axis=-1, keepdims=True) * 2.0
+    v_uni = np.transpose(zc.reshape(z.shape[0], N, z.shape[1], z.shape[3]), (0, 2, 1, 3))
+    for kk in (1, 5, 20):
+        sel = O.refresh_mask(q, k, v_uni, [0, N], k_budget=kk)["idx"]
+        by_attention = O.topk_select(O.score_request(q, k, v_uni, [0, N])["A"], kk)
+        assert sel.tolist() == by_attention.tolist()
+
+
+def test_single_image_limit():
+    """K = 1: c_1 = 1 for every lambda and selection is intra-image top-k of s (Sec. 3.5)."""
+    q, k, v, _ = _rand_request(10)
+    N = k.shape[2]
+    for lam in (0.0, 0.25, 0.5, 1.0):
+        assert O.image_coefficients(np.array([0.0123]), lam).tolist() == [1.0]
+        out = O.refresh_mask(q, k, v, [0, N], lam=lam, k_budget=7)
+        want = np.sort(np.argsort(-out["s"], kind="stable")[:7])
+        assert out["idx"].tolist() == want.tolist()
+
+
+def test_lambda_zero_is_plain_global_topk():
+    q, k, v, spans = _rand_request(11)
+    out = O.refresh_mask(q, k, v, spans, lam=0.0, k_budget=8)
+    assert np.all(out["c"] == 1.0)
+    want = np.sort(np.argsort(-out["s"], kind="stable")[:8])
+    assert out["idx"].tolist() == want.tolist()
+
+
+def test_mean_coefficient_is_one():
+    rng = np.random.default_rng(12)
+    for _ in range(20):
+        g = rng.random(rng.integers(2, 40)) * 1e-3
+        for lam in (0.0, 0.3, 1.0):
+            assert abs(O.image_coefficients(g, lam).mean() - 1.0) < 1e-12
+
+
+def test_relevant_image_is_amplified():
+    """lambda = 1 raises tokens of an above-average image (Sec. 3.4)."""
+    g = np.array([0.1, 0.3, 0.2])
+    c = O.image_coefficients(g, 1.0)
+    assert c[1] > 1.0 > c[0] and abs(c[2] - 1.0) < 1e-15
+
+
+def test_budget_zero_and_full():
+    q, k, v, spans = _rand_request(13)
+    N = k.shape[2]
+    out0 = O.refresh_mask(q, k, v, spans, r=0.0)
+    assert out0["k"] == 0 and out0["idx"].size == 0 and out0["mask"].sum() == 0
+    out1 = O.refresh_mask(q, k, v, spans, r=1.0)
+    assert out1["idx"].tolist() == list(range(N)) and out1["mask"].sum() == N
+
+
+def test_scored_layer_subset():
+    q, k, v, spans = _rand_request(14, L=3)
+    one = O.score_request(q, k, v, spans, layers=[1])
+    alone = O.score_request(q[1:2], k[1:2], v[1:2], spans)
+    np.testing.assert_allclose(one["s"], alone["s"], rtol=1e-15)
+    np.testing.assert_allclose(one["g"], alone["g"], rtol=1e-15)
+
+
+# --------------------------------------------------------- refresh step
+def test_gather_scatter_roundtrip():
+    rng = np.random.default_rng(15)
+    cache = rng.standard_normal((2, 3, 20, 4))
+    idx = [1, 5, 19]
+    rows = rng.standard_normal((2, 3, 3, 4))
+    patched = O.kv_scatter(cache, idx, rows)
+    np.testing.assert_array_equal(O.kv_gather(patched, idx), rows)
+    keep = [t for t in range(20) if t not in idx]
+    np.testing.assert_array_equal(patched[:, :, keep], cache[:, :, keep])
+    np.testing.assert_array_equal(O.kv_gather(cache, idx)[:, 1, 2], cache[:, 2, 5])
+
+
+def test_refresh_attention_full_budget_is_causal_sdpa():
+    """k = N with no patch is ordinary causal self-attention: torch SDPA with GQA."""
+    rng = np.random.default_rng(16)
+    L, Hq, Hkv, N, d = 2, 4, 2, 13, 8
+    k = rng.standard_normal((L, Hkv, N, d))
+    v = rng.standard_normal((L, Hkv, N, d))
+    q_rows = rng.standard_normal((L, N, Hq, d))
+    out = O.refresh_attention(q_rows, k, v, list(range(N)))
+    for l in range(L):
+        qt = torch.from_numpy(q_rows[l]).transpose(0, 1)                      # [Hq, N, d]
+        kt = torch.from_numpy(k[l]).repeat_interleave(Hq // Hkv, dim=0)
+        vt = torch.from_numpy(v[l]).repeat_interleave(Hq // Hkv, dim=0)
+        want = torch.nn.functional.scaled_dot_product_attention(qt, kt, vt, is_causal=True)
+        np.testing.assert_allclose(out[l], want.transpose(0, 1).numpy(), rtol=1e-12, atol=1e-13)
+
+
+def test_refresh_attention_sparse_rows_match_sdpa_rows():
+    rng = np.random.default_rng(17)
+    L, Hq, Hkv, N, d = 1, 4, 1, 30, 16
+    k = rng.standard_normal((L, Hkv, N, d))
+    v = rng.standard_normal((L, Hkv, N, d))
+    idx = [2, 9, 10, 29]
+    q_all = rng.standard_normal((L, N, Hq, d))
+    out = O.refresh_attention(q_all[:, idx], k, v, idx)
+    qt = torch.from_numpy(q_all[0]).transpose(0, 1)
+    kt = torch.from_numpy(k[0]).repeat_interleave(Hq, dim=0)
+    vt = torch.from_numpy(v[0]).repeat_interleave(Hq, dim=0)
+    full = torch.nn.functional.scaled_dot_product_attention(qt, kt, vt, is_causal=True).transpose(0, 1).numpy()
+    np.testing.assert_allclose(out[0], full[idx], rtol=1e-12, atol=1e-13)
+
+
+def test_refresh_attention_first_position_returns_its_value():
+    rng = np.random.default_rng(18)
+    k = rng.standard_normal((1, 2, 6, 4))
+    v = rng.standard_normal((1, 2, 6, 4))
+    q = rng.standard_normal((1, 1, 4, 4)) * 10
+    out = O.refresh_attention(q, k, v, [0])
+    for h in range(4):
+        np.testing.assert_array_equal(out[0, 0, h], v[0, h // 2, 0])
