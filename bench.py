@@ -1,0 +1,488 @@
+"""Benchmark of Conduit's hot path on GB300: one step = scoring pass, selection,
+gather, scatter and refresh attention over one batch of a synthetic workload.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl conduit|reference]
+                  [--config single|multi|longdoc|batched|tiny]
+
+Prints one JSON line. ``value`` is cached visual tokens passed through the
+whole step per second (device time, inputs resident in HBM, L2 flushed
+between steps); ``e2e`` is the same through the public step with the cache,
+queries and fresh rows copied from pinned host memory each step and the
+selection and refresh output copied back. Under torchrun every rank runs its
+own replica on its own GPU (the path has no exchange step); the step time is
+the maximum over ranks.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+_CORES = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else (os.cpu_count() or 1)
+for _v in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
+    os.environ.setdefault(_v, str(_CORES))
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+METRIC = "cached visual tokens scored+selected/sec and refresh-pass µs; % of HBM roofline"
+UNIT = "tokens/s"
+DESCR = {
+    "tiny": "tiny single-image: 1 layer, 1 image x 256 visual tokens, 16 query-prefix tokens, 4/2 heads, head_dim 64, fp32, budget 10%",
+    "single": "single high-res image: 28 layers, 28/4 heads, head_dim 128, bf16 cache [28,4,1024,128], 32 query-prefix tokens, budget 10%",
+    "multi": "multi-image: 8 images x 1024 tokens, 28 layers, 28/4 heads, head_dim 128, bf16, 64 query-prefix tokens, budget 10%",
+    "longdoc": "long document: 32 pages x 1296 tokens, 36 layers, 32/8 heads, head_dim 128, bf16, 48 query-prefix tokens, budget 10%",
+    "batched": "batched serving: 16 requests x 4 images x 2048 tokens, 28 layers, 28/4 heads, head_dim 128, bf16 paged (16-token pages), 32-128 query tokens, budgets 5/10/20%",
+}
+L2_FLUSH_BYTES = 256 << 20
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), float(p["bf16_tflops"]), float(p.get("bf16_tflops_sustained", p["bf16_tflops"])), "measured"
+    except Exception:
+        return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+# fp32 CUDA-core peak: 152 SMs x 128 FMA lanes x 2 FLOP x 2.07 GHz (max SM clock)
+ALU_FP32_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
+
+
+# ------------------------------------------------------------------ clocks
+class ClockSampler:
+    """nvidia-smi samples every 200 ms while the timed region runs."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index, self.proc, self.lines = index, None, []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self._t = threading.Thread(target=self._read, daemon=True)
+            self._t.start()
+        except Exception:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ------------------------------------------------------------ distributed
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def reduce_max(value: float, world: int) -> float:
+    """Maximum of a float over ranks (identity on one rank)."""
+    if world == 1:
+        return value
+    import torch.distributed as dist
+    dev = torch.device("cuda", torch.cuda.current_device()) if dist.get_backend() == "nccl" else torch.device("cpu")
+    t = torch.tensor([value], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world: int):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+# ------------------------------------------------------------ work models
+def work_model(pipe) -> dict:
+    """Algorithmic bytes / FLOPs of one step, per C-ABI call."""
+    kv, b = pipe.kv, pipe.batch
+    esz = pipe.kv.k.element_size()
+    L = kv.num_layers if pipe.layers is None else len(pipe.layers)
+    Lall, Hq, Hkv, d = kv.num_layers, kv.num_q_heads, kv.num_kv_heads, kv.head_dim
+    tok, qo = b.tok_off.tolist(), b.q_off.tolist()
+    R, K = b.num_requests, b.num_images
+    n_tot = tok[-1]
+    score_bytes = 2 * L * Hkv * n_tot * d * esz + L * Hq * qo[-1] * d * esz + 8 * n_tot + 4 * K
+    score_flops = sum(2 * L * Hq * (qo[r + 1] - qo[r]) * (tok[r + 1] - tok[r]) * d for r in range(R))
+    k_sel = pipe.n_sel
+    sel_bytes = 4 * n_tot + 4 * K + 4 * n_tot + n_tot + 4 * k_sel + 4 * K
+    copy_bytes = 2 * 2 * Lall * k_sel * Hkv * d * esz
+    idx = pipe.idx[:k_sel].cpu().tolist()
+    off = pipe.idx_off.tolist()
+    ref_flops, ref_bytes = 0, 2 * 2 * Lall * k_sel * Hq * d * esz
+    for r in range(R):
+        ps = idx[off[r]:off[r + 1]]
+        ref_flops += sum(4 * Hq * d * (p + 1) for p in ps) * Lall
+        if ps:
+            ref_bytes += 2 * Lall * Hkv * (max(ps) + 1) * d * esz
+    return {
+        "score": {"bytes": score_bytes, "flops": score_flops},
+        "select": {"bytes": sel_bytes, "flops": 0},
+        "gather": {"bytes": copy_bytes, "flops": 0},
+        "scatter": {"bytes": copy_bytes, "flops": 0},
+        "refresh": {"bytes": ref_bytes, "flops": ref_flops},
+    }
+
+
+CALL_KERNELS = {  # kernels behind each C-ABI call in this build, and their bound
+    "score": (["value_sumsq_kernel", "rowstats_kernel", "colsum_kernel", "finalize_tokens_kernel",
+               "image_means_kernel"], "alu"),
+    "select": (["select_kernel"], "hbm"),
+    "gather": (["kv_copy_kernel"], "hbm"),
+    "scatter": (["kv_copy_kernel"], "hbm"),
+    "refresh": (["refresh_simt_kernel"], "alu"),
+}
+KERNEL_SOURCES = {"score": "score_simt.cu", "select": "select.cu", "gather": "kvcopy.cu",
+                  "scatter": "kvcopy.cu", "refresh": "refresh_simt.cu"}
+
+
+def _src_hash(call: str) -> str:
+    p = os.path.join(ROOT, "paper_2609_05821_gb300", "csrc", KERNEL_SOURCES[call])
+    with open(p, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:12]
+
+
+def _traffic(call: str, workload: str):
+    """DRAM bytes per launch from a committed ncu summary, if its source hash still matches."""
+    p = os.path.join(ROOT, "profiles", "traffic.txt")
+    if not os.path.exists(p):
+        return None
+    for line in open(p):
+        f = line.split()
+        if len(f) >= 4 and not line.startswith("#") and f[0] == call and f[1] == workload:
+            return float(f[2]) if f[3] == _src_hash(call) else None
+    return None
+
+
+# -------------------------------------------------------------- our arm
+def build_pipeline(cfg: str, device):
+    from paper_2609_05821_gb300 import pipeline, synth
+    w = synth.workload(cfg)
+    inputs = synth.make_inputs(w, device=device)
+    return pipeline.from_inputs(inputs), w
+
+
+def time_steps(fn, steps: int, flush=None):
+    """Per-step device time (ms) with CUDA events on the current stream."""
+    stream = torch.cuda.current_stream()
+    times = []
+    for _ in range(steps):
+        if flush is not None:
+            flush()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        fn()
+        b.record(stream)
+        b.synchronize()
+        times.append(a.elapsed_time(b))
+    return times
+
+
+def run_conduit(args):
+    world, rank, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", init_method="env://")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    from paper_2609_05821_gb300 import conduit as C
+
+    pipe, w = build_pipeline(args.config, dev)
+    n_tok = pipe.batch.n_tot
+    flush_buf = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    flush = lambda: flush_buf.zero_()
+
+    # warm-up (eager), then one graph of the whole step
+    for _ in range(args.warmup):
+        pipe.step()
+    torch.cuda.synchronize()
+    launches0 = C.conduit_launch_count()
+    pipe.step()
+    torch.cuda.synchronize()
+    launches_per_step = C.conduit_launch_count() - launches0
+    if not args.no_graph:
+        pipe.capture()
+        for _ in range(max(1, args.warmup)):
+            pipe.step()
+    torch.cuda.synchronize()
+
+    # timed region: K whole steps
+    hbm, tc, tc_sus, peak_src = _peaks()
+    barrier(world)
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        t0 = time.perf_counter()
+        step_ms = time_steps(pipe.step, args.steps, flush)
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - t0
+    barrier(world)
+    mean_ms = sum(step_ms) / len(step_ms)
+    max_ms = reduce_max(mean_ms, world)
+
+    # per-call breakdown over K eager steps (events on the launching stream)
+    graph, pipe.graph = pipe.graph, None
+    calls = {"score": [], "select": [], "gather": [], "scatter": [], "refresh": []}
+    from paper_2609_05821_gb300 import conduit as CC
+    stream = torch.cuda.current_stream()
+    for _ in range(args.steps):
+        flush()
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(6)]
+        ev[0].record(stream)
+        CC.conduit_score(pipe.kv, pipe.batch, pipe.q, pipe.layers, pipe.s, pipe.attn_sum, pipe.g,
+                         pipe.ws_score, pipe.status)
+        ev[1].record(stream)
+        CC.conduit_select_topk(pipe.batch, pipe.s, pipe.g, pipe.lam, pipe.idx_off, pipe.idx_off_dev,
+                               pipe.idx, pipe.mask, pipe.s_hat, pipe.coeff, pipe.ws_sel, pipe.status)
+        ev[2].record(stream)
+        CC.conduit_kv_gather(pipe.kv, pipe.batch, pipe.idx, pipe.idx_off, pipe.idx_off_dev,
+                             pipe.k_old, pipe.v_old)
+        ev[3].record(stream)
+        CC.conduit_kv_scatter(pipe.kv, pipe.batch, pipe.idx, pipe.idx_off, pipe.idx_off_dev,
+                              pipe.k_rows, pipe.v_rows)
+        ev[4].record(stream)
+        CC.conduit_refresh_attn(pipe.kv, pipe.batch, pipe.idx, pipe.idx_off, pipe.idx_off_dev,
+                                pipe.q_rows, pipe.out, pipe.ws_ref, pipe.status)
+        ev[5].record(stream)
+        ev[5].synchronize()
+        for i, name in enumerate(calls):
+            calls[name].append(ev[i].elapsed_time(ev[i + 1]))
+    pipe.graph = graph
+    call_ms = {k: sum(v) / len(v) for k, v in calls.items()}
+    status = C.conduit_read_status(pipe.status)
+
+    # roofline of the dominant call
+    model = work_model(pipe)
+    dom = max(call_ms, key=call_ms.get)
+    kernels, bound = CALL_KERNELS[dom]
+    sec = call_ms[dom] / 1e3
+    if bound == "hbm":
+        achieved, peak, unit = model[dom]["bytes"] / sec / 1e9, hbm, "GB/s"
+        peak_note = f"HBM copy, {peak_src}"
+    elif bound == "tensor":
+        achieved, peak, unit = model[dom]["flops"] / sec / 1e12, tc, "TFLOP/s"
+        peak_note = f"bf16 dense burst, {peak_src}"
+    else:
+        achieved, peak, unit = model[dom]["flops"] / sec / 1e12, ALU_FP32_TFLOPS, "TFLOP/s"
+        peak_note = "fp32 FMA: 152 SMs x 128 lanes x 2 FLOP x 2.07 GHz"
+    traffic = _traffic(dom, args.config)
+    roofline = {"bound": bound, "achieved": round(achieved, 3), "peak": round(peak, 1), "unit": unit,
+                "frac": round(achieved / peak, 4), "traffic": traffic, "kernel": dom,
+                "kernels": kernels, "peak_source": peak_note,
+                "hbm_frac": round(model[dom]["bytes"] / sec / 1e9 / hbm, 4)}
+    breakdown = {}
+    for name, ms in call_ms.items():
+        s_ = ms / 1e3
+        breakdown[name] = {"us": round(ms * 1e3, 2),
+                           "GB_per_s": round(model[name]["bytes"] / s_ / 1e9, 1),
+                           "hbm_frac": round(model[name]["bytes"] / s_ / 1e9 / hbm, 4)}
+        if model[name]["flops"]:
+            breakdown[name]["TFLOP_per_s"] = round(model[name]["flops"] / s_ / 1e12, 2)
+
+    # end to end through the public step with host buffers
+    host = pipe.host_buffers()
+    for _ in range(2):
+        pipe.step_from_host(host)
+    torch.cuda.synchronize()
+    e2e_ms = time_steps(lambda: pipe.step_from_host(host), max(3, min(args.steps, 10)))
+    e2e_mean = reduce_max(sum(e2e_ms) / len(e2e_ms), world)
+
+    out = {
+        "metric": METRIC, "value": round(world * n_tok / (max_ms / 1e3), 1), "unit": UNIT,
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(max_ms, 5), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16" if pipe.kv.k.dtype == torch.bfloat16 else "f32",
+        "data": "synthetic (seeded; shapes and value laws of the paper's workloads)",
+        "config": {"workload": DESCR[args.config], "name": args.config, "tokens_per_step": n_tok,
+                   "budget_total": pipe.n_sel, "layers": pipe.kv.num_layers,
+                   "l2": f"flushed between timed steps ({L2_FLUSH_BYTES >> 20} MB write)",
+                   "cuda_graph": not args.no_graph, "parallelism": f"replicas x{world}"},
+        "score_select_tokens_per_s": round(n_tok / ((call_ms["score"] + call_ms["select"]) / 1e3), 1),
+        "refresh_pass_us": round((call_ms["gather"] + call_ms["scatter"] + call_ms["refresh"]) * 1e3, 2),
+        "breakdown": breakdown,
+        "roofline": roofline,
+        "e2e": {"value": round(world * n_tok / (e2e_mean / 1e3), 1), "unit": UNIT,
+                "h2d_bytes_per_step": pipe.h2d_bytes(), "d2h_bytes_per_step": pipe.d2h_bytes()},
+        "gpu_launches": launches_per_step * args.steps,
+        "clocks": clk.summary(),
+        "status": status,
+        "wall_s_timed": round(wall, 3),
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        out["cpu_baseline"] = cpu_baseline(args.config, args.cpu_seconds)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+
+
+# ------------------------------------------------------- CPU oracle arm
+def oracle_step_sample(cfg: str, budget_seconds: float, seed_inputs=None):
+    """Time the CPU oracle on a bounded sample of one step of the workload.
+
+    Scoring runs layer by layer over all of request 0's tokens until about
+    60 % of the budget is spent; selection runs once on the sample's scores;
+    refresh attention runs for a few selected rows of the sampled layers.
+    Returns (estimated seconds per full step, description).
+    """
+    from oracle import conduit_oracle as O
+    from paper_2609_05821_gb300 import synth
+    w = synth.workload(cfg)
+    inputs = seed_inputs or synth.make_inputs(w, device="cpu")
+    tok, qo = inputs["tok_off"].tolist(), inputs["q_off"].tolist()
+    R, L = len(tok) - 1, w.num_layers
+    t0, t1, q0, q1 = tok[0], tok[1], qo[0], qo[1]
+    spans = [x - t0 for x in inputs["img_off"].tolist()[: inputs["req_img_off"].tolist()[1] + 1]]
+    ql = lambda l: inputs["q"][l, :, q0:q1].double().numpy()
+    kl = lambda l: inputs["k"][l, :, t0:t1].double().numpy()
+    vl = lambda l: inputs["v"][l, :, t0:t1].double().numpy()
+    a, vn, layer_t = [], [], []
+    start = time.perf_counter()
+    for l in range(L):
+        ts = time.perf_counter()
+        a.append(O.head_query_mean_attention(ql(l), kl(l)))
+        vn.append(O.value_norms(vl(l)))
+        layer_t.append(time.perf_counter() - ts)
+        if time.perf_counter() - start > 0.6 * budget_seconds:
+            break
+    ts = time.perf_counter()
+    a_, vn_ = np.stack(a), np.stack(vn)
+    s = O.throughput_score(a_, vn_)
+    g = O.image_mean_attention(a_, spans)
+    c = O.image_coefficients(g, 1.0)
+    kk = O.budget(inputs["ratios"][0], t1 - t0)
+    idx = O.topk_select(O.composite_score(s, c, spans), kk)
+    t_sel = time.perf_counter() - ts
+    rows = idx[: max(1, min(len(idx), 8))]
+    fr = synth.make_fresh_rows(w, len(rows), device="cpu")
+    ts = time.perf_counter()
+    n_ref_layers = min(len(layer_t), 2)
+    for l in range(n_ref_layers):
+        kp = O.kv_scatter(kl(l)[None], rows, fr["k_rows"][l:l + 1].double().numpy())
+        vp = O.kv_scatter(vl(l)[None], rows, fr["v_rows"][l:l + 1].double().numpy())
+        O.refresh_attention(fr["q_rows"][l:l + 1].double().numpy(), kp, vp, rows)
+    t_ref = time.perf_counter() - ts
+    n_sel_total = sum(O.budget(r, tok[i + 1] - tok[i]) for i, r in enumerate(inputs["ratios"]))
+    per_layer = sum(layer_t) / len(layer_t)
+    est = (per_layer * L * R + t_sel * R +
+           t_ref / (n_ref_layers * len(rows)) * L * n_sel_total)
+    desc = (f"request 0: scoring of {len(layer_t)}/{L} layers over all {t1 - t0} tokens, one "
+            f"selection, refresh of {len(rows)} rows x {n_ref_layers} layers; extrapolated to "
+            f"{R} request(s) x {L} layers x {n_sel_total} refreshed rows")
+    return est, desc, time.perf_counter() - start
+
+
+def cpu_baseline(cfg: str, seconds: float) -> dict:
+    n_tok = _workload_tokens(cfg)
+    est, desc, spent = oracle_step_sample(cfg, seconds)
+    return {"value": round(n_tok / est, 2), "unit": UNIT, "cores": _CORES, "kind": "oracle",
+            "sample": desc, "sample_seconds": round(spent, 1),
+            "threads_note": f"numpy BLAS threads = {_CORES}; elementwise numpy is single-threaded"}
+
+
+def _workload_tokens(cfg: str) -> int:
+    from paper_2609_05821_gb300 import synth
+    w = synth.workload(cfg)
+    return w.num_requests * w.tokens_per_request
+
+
+def run_reference(args):
+    world, rank, _ = dist_env()
+    if rank != 0:
+        return
+    from paper_2609_05821_gb300 import synth
+    w = synth.workload(args.config)
+    inputs = synth.make_inputs(w, device="cpu")
+    n_tok = _workload_tokens(args.config)
+    per_step = max(2.0, min(20.0, 150.0 / max(1, args.steps + args.warmup)))
+    for _ in range(args.warmup):
+        oracle_step_sample(args.config, per_step, inputs)
+    ests, desc = [], ""
+    for _ in range(args.steps):
+        est, desc, _ = oracle_step_sample(args.config, per_step, inputs)
+        ests.append(est)
+    est = statistics.median(ests)
+    value = round(world * n_tok / est, 2)
+    out = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(est * 1e3, 3),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded; shapes and value laws of the paper's workloads)",
+        "config": {"workload": DESCR[args.config], "name": args.config, "tokens_per_step": n_tok},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": _CORES, "kind": "oracle",
+                         "sample": desc},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(out), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="conduit", choices=["conduit", "reference"])
+    ap.add_argument("--config", default="single", choices=sorted(DESCR))
+    ap.add_argument("--no-graph", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    args = ap.parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_conduit(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,228 @@
+/*
+ * conduit.h - C ABI of the GB300 library for Conduit's query-conditioned
+ * scoring pass and budgeted selective refresh (Conduit, Sec. 3 and
+ * Algorithm 1).
+ *
+ * Conventions shared by every entry point:
+ *  - Every call returns a conduit_status. No exception crosses the ABI.
+ *  - Arguments are checked on the host before anything is enqueued; a call
+ *    that returns CONDUIT_ERR_INVALID_ARG, _UNSUPPORTED or _WORKSPACE has
+ *    launched nothing and touched no device memory.
+ *  - Pointers marked "device" are caller-owned device memory; pointers
+ *    marked "host" are caller-owned host memory read during the call only.
+ *    The library never allocates device memory: scratch space comes from a
+ *    caller workspace whose size the matching *_workspace_size call returns.
+ *  - All device work is enqueued on the caller's stream (a cudaStream_t
+ *    passed as void*; NULL means the legacy default stream) and is
+ *    asynchronous. No call synchronises, except conduit_read_status.
+ *  - Conditions found on the device (a non-finite score, a bounded wait that
+ *    ran out) are OR-ed into a caller-provided device int32 status word as
+ *    CONDUIT_FLAG_* bits; conduit_read_status turns the word into a status.
+ *  - conduit_last_error_string() describes the last failure of the calling
+ *    thread.
+ *
+ * Token positions are request-local indices 0 .. N_r-1 of the request's
+ * visual tokens. Image spans are contiguous, non-empty and tile each
+ * request's tokens (Sec. 3.1, Eq. 1).
+ */
+#ifndef CONDUIT_H
+#define CONDUIT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define CONDUIT_VERSION 100 /* 1.0.0 */
+#define CONDUIT_MAX_LAYERS 512
+
+typedef int32_t conduit_status;
+enum {
+  CONDUIT_OK = 0,
+  CONDUIT_ERR_INVALID_ARG = 1, /* a pointer, size, span or budget is wrong */
+  CONDUIT_ERR_UNSUPPORTED = 2, /* valid, but a shape or dtype this build lacks */
+  CONDUIT_ERR_CUDA = 3,        /* a CUDA runtime call failed */
+  CONDUIT_ERR_NONFINITE = 4,   /* device found a NaN / Inf score (status word) */
+  CONDUIT_ERR_TIMEOUT = 5,     /* a bounded device wait ran out (status word) */
+  CONDUIT_ERR_WORKSPACE = 6    /* workspace pointer missing, misaligned or short */
+};
+
+/* Bits of the device status word. */
+enum { CONDUIT_FLAG_NONFINITE = 1, CONDUIT_FLAG_TIMEOUT = 2 };
+
+/* Element type of K, V, queries, fresh rows and refresh outputs. */
+enum { CONDUIT_F32 = 0, CONDUIT_BF16 = 1 };
+
+/*
+ * The reused visual KV cache (Sec. 3.1; paged storage as in the serving
+ * engine of Sec. 4.3).
+ *  contiguous (page_size == 0): k, v are [L][Hkv][N_tot][d]; request r's
+ *    tokens are rows tok_off[r] .. tok_off[r+1]-1.
+ *  paged (page_size > 0): k, v are pools [L][P][Hkv][page_size][d];
+ *    request r's token t lives in physical page
+ *    page_table[r * max_pages_per_req + t / page_size] at row t % page_size.
+ * k and v are 16-byte aligned device pointers of dtype `dtype`.
+ */
+typedef struct conduit_kv {
+  int32_t num_layers;        /* L */
+  int32_t num_q_heads;       /* Hq */
+  int32_t num_kv_heads;      /* Hkv, Hq % Hkv == 0 (grouped-query attention) */
+  int32_t head_dim;          /* d, a multiple of 8 in [8, 256] */
+  int32_t dtype;             /* CONDUIT_F32 or CONDUIT_BF16 */
+  int32_t page_size;         /* 0 = contiguous, else rows per page */
+  int32_t num_pages;         /* P (paged only) */
+  int32_t max_pages_per_req; /* row length of page_table (paged only) */
+  void* k;                   /* device */
+  void* v;                   /* device */
+  const int32_t* page_table; /* device [R][max_pages_per_req] (paged only) */
+} conduit_kv;
+
+/*
+ * A batch of requests, each with its visual-token span, its image spans
+ * (Eq. 1: V_j, n_j, pi(t)) and its scoring query span Q (App. A.2: the text
+ * block after the last image). Every offset array exists twice, on the host
+ * (for checks and launch sizing) and on the device (for the kernels), with
+ * equal contents.
+ *  tok_off    [R+1]  request r owns global token rows tok_off[r] .. tok_off[r+1]-1
+ *  img_off    [K+1]  image j owns global token rows img_off[j] .. img_off[j+1]-1
+ *  req_img_off[R+1]  request r owns images req_img_off[r] .. req_img_off[r+1]-1
+ *  q_off      [R+1]  request r owns query rows q_off[r] .. q_off[r+1]-1
+ */
+typedef struct conduit_batch {
+  int32_t num_requests; /* R >= 1 */
+  int32_t num_images;   /* K (total over requests) >= R */
+  const int32_t* tok_off;         /* host */
+  const int32_t* img_off;         /* host */
+  const int32_t* req_img_off;     /* host */
+  const int32_t* q_off;           /* host */
+  const int32_t* tok_off_dev;     /* device */
+  const int32_t* img_off_dev;     /* device */
+  const int32_t* req_img_off_dev; /* device */
+  const int32_t* q_off_dev;       /* device */
+} conduit_batch;
+
+/* Library version, CONDUIT_VERSION of the build. */
+int32_t conduit_version(void);
+
+/* Text of the calling thread's last error ("" if none). Never NULL. */
+const char* conduit_last_error_string(void);
+
+/*
+ * Refresh budget k = floor(r * N_vis), Eq. 2 and Algorithm 1 (first step).
+ * A guard of 1e-9 makes decimal ratios land on integers (0.3 * 10 -> 3).
+ * Returns -1 if r is outside [0, 1] or NaN, or n_vis is negative.
+ */
+int32_t conduit_budget(double r, int64_t n_vis);
+
+/*
+ * Query-conditioned scoring pass (Sec. 3.3, Eqs. 6-8; Algorithm 1 scoring
+ * loops). For every request, scored layer l and token t:
+ *   alpha_{q,t,l,h} = softmax over the request's N_r visual keys of
+ *                     <q_{l,h,q}, k_{l,h/G,t}> / sqrt(d)            (fp32)
+ *   a_t^(l)  = sum_q sum_h alpha / (|Q| Hq)                          Eq. 6
+ *   v_t^(l)  = || concat_g V_{l,g,t} ||_2                            Sec. 3.3
+ *   s[t]     = (1/|L|) sum_l a_t^(l) v_t^(l)                         Eq. 7
+ *   attn_sum[t] = sum_l a_t^(l)
+ *   g[j]     = (1/(|L| n_j)) sum_l sum_{t in V_j} a_t^(l)            Eq. 8
+ *  q         device [L][Hq][Q_tot][d], dtype of kv (post-RoPE queries)
+ *  layers    host [n_layers] strictly increasing scored layer ids, or NULL
+ *            for all L layers (App. A.2 default); n_layers <= CONDUIT_MAX_LAYERS
+ *  s, attn_sum  device fp32 [N_tot] (attn_sum may be NULL)
+ *  g         device fp32 [K]
+ *  workspace device, 256-byte aligned, conduit_score_workspace_size bytes
+ *  status    device int32 status word or NULL (NONFINITE if a score is NaN/Inf)
+ * Results are deterministic: the same inputs give bitwise-equal outputs.
+ */
+conduit_status conduit_score_workspace_size(const conduit_kv* kv, const conduit_batch* batch,
+                                            int32_t n_layers, size_t* bytes);
+conduit_status conduit_score(const conduit_kv* kv, const conduit_batch* batch, const void* q,
+                             const int32_t* layers, int32_t n_layers, float* s, float* attn_sum,
+                             float* g, void* workspace, size_t workspace_bytes, int32_t* status,
+                             void* stream);
+
+/*
+ * Image-level amplification and one global top-k per request (Sec. 3.4-3.5,
+ * Eqs. 9-11; Algorithm 1 last loops).
+ *   c_j    = (1 - lambda) + lambda g_j / g_bar, g_bar = mean of the request's g_j;
+ *            exactly 1 when the request has one image (Sec. 3.5) or g_bar == 0
+ *   s_hat_t = s_t c_{pi(t)}                                          Eq. 10
+ *   T_r    = TopK_t(s_hat, k_r), ties to the lowest index            Eq. 11
+ *  s, g       device fp32 [N_tot], [K] (outputs of conduit_score)
+ *  lambda     in [0, 1]
+ *  idx_off    host [R+1], idx_off_dev device [R+1]: prefix sums of the
+ *             budgets, k_r = idx_off[r+1] - idx_off[r], 0 <= k_r <= N_r
+ *  idx        device int32 [idx_off[R]]: request r's selected request-local
+ *             token indices at idx[idx_off[r] ..], ascending
+ *  mask       device uint8 [N_tot] refresh mask (1 = recompute) or NULL
+ *  s_hat      device fp32 [N_tot] or NULL;  coeff device fp32 [K] c_j or NULL
+ *  status     NONFINITE if an s_hat is NaN / Inf
+ */
+conduit_status conduit_select_workspace_size(const conduit_batch* batch, size_t* bytes);
+conduit_status conduit_select_topk(const conduit_batch* batch, const float* s, const float* g,
+                                   float lambda, const int32_t* idx_off, const int32_t* idx_off_dev,
+                                   int32_t* idx, uint8_t* mask, float* s_hat, float* coeff,
+                                   void* workspace, size_t workspace_bytes, int32_t* status,
+                                   void* stream);
+
+/*
+ * Gather of the selected rows of every layer (selective recompute, Sec. 3.1
+ * and 3.5): k_rows[l][i][g][:] = K[l][g][idx_i][:] (same for V), where i runs
+ * over all requests' selections in idx order.
+ *  k_rows, v_rows  device [L][idx_off[R]][Hkv][d], dtype of kv
+ */
+conduit_status conduit_kv_gather(const conduit_kv* kv, const conduit_batch* batch,
+                                 const int32_t* idx, const int32_t* idx_off,
+                                 const int32_t* idx_off_dev, void* k_rows, void* v_rows,
+                                 void* stream);
+
+/*
+ * Scatter of recomputed K/V rows into the cache, all layers in one launch
+ * (Sec. 3.5: selected entries are recomputed, the rest are reused):
+ * K[l][g][idx_i][:] = k_rows[l][i][g][:] (same for V). In place in kv->k, kv->v.
+ *  k_rows, v_rows  device [L][idx_off[R]][Hkv][d], dtype of kv
+ */
+conduit_status conduit_kv_scatter(const conduit_kv* kv, const conduit_batch* batch,
+                                  const int32_t* idx, const int32_t* idx_off,
+                                  const int32_t* idx_off_dev, const void* k_rows,
+                                  const void* v_rows, void* stream);
+
+/*
+ * Causal attention of the refreshed rows over the patched cache (Sec. 3.1
+ * and 4.3, selective recompute): for every layer l, selected row i at
+ * position p_i = idx_i and query head h,
+ *   out[l][i][h] = sum_{j <= p_i} softmax_j(<q_rows[l][i][h], K'[l][h/G][j]> / sqrt(d)) V'[l][h/G][j]
+ * where K', V' are the cache after conduit_kv_scatter (call it first).
+ * Softmax and accumulation in fp32; out is written in the cache dtype.
+ *  q_rows, out  device [L][idx_off[R]][Hq][d], dtype of kv
+ *  idx must be ascending within each request (conduit_select_topk's order).
+ */
+conduit_status conduit_refresh_workspace_size(const conduit_kv* kv, const conduit_batch* batch,
+                                              const int32_t* idx_off, size_t* bytes);
+conduit_status conduit_refresh_attn(const conduit_kv* kv, const conduit_batch* batch,
+                                    const int32_t* idx, const int32_t* idx_off,
+                                    const int32_t* idx_off_dev, const void* q_rows, void* out,
+                                    void* workspace, size_t workspace_bytes, int32_t* status,
+                                    void* stream);
+
+/*
+ * Number of kernels this library has enqueued in this process (launched, or
+ * recorded into a stream capture) since it was loaded. Diagnostic only.
+ */
+int64_t conduit_launch_count(void);
+
+/* Zero the device status word (enqueued on stream). */
+conduit_status conduit_clear_status(int32_t* status, void* stream);
+
+/*
+ * Synchronise `stream`, copy the status word to *word (host) and return
+ * CONDUIT_OK, CONDUIT_ERR_NONFINITE or CONDUIT_ERR_TIMEOUT (timeout wins).
+ */
+conduit_status conduit_read_status(const int32_t* status, void* stream, int32_t* word);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CONDUIT_H */

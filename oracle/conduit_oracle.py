@@ -202,16 +202,15 @@ def score_request(q: np.ndarray, k: np.ndarray, v: np.ndarray,
                   img_off: Sequence[int], layers: Optional[Sequence[int]] = None) -> dict:
     """The query-conditioned scoring pass for one request (Algorithm 1, scoring loop).
 
-    q: [L, Hq, n_q, d]; k, v: [L, Hkv, N, d]; layers: the scored layer set
-    (default all layers, App. A.2). Returns a, vn ([|L|, N]), s, A ([N]) and g ([K]).
+    q: [L, Hq, n_q, d]; k, v: [L, Hkv, N, d] (anything whose [l] gives one
+    layer's array); layers: the scored layer set (default all layers, App. A.2).
+    Returns a, vn ([|L|, N]), s, A ([N]) and g ([K]).
     """
-    q = np.asarray(q, dtype=np.float64)
-    k = np.asarray(k, dtype=np.float64)
-    v = np.asarray(v, dtype=np.float64)
+    f64 = lambda x: np.asarray(x, dtype=np.float64)
     if layers is None:
-        layers = list(range(k.shape[0]))
-    a = np.stack([head_query_mean_attention(q[l], k[l]) for l in layers])
-    vn = np.stack([value_norms(v[l]) for l in layers])
+        layers = list(range(len(k)))
+    a = np.stack([head_query_mean_attention(f64(q[l]), f64(k[l])) for l in layers])
+    vn = np.stack([value_norms(f64(v[l])) for l in layers])
     s = throughput_score(a, vn)
     attn_sum = a.sum(axis=0)
     g = image_mean_attention(a, img_off)
@@ -227,7 +226,7 @@ def refresh_mask(q: np.ndarray, k: np.ndarray, v: np.ndarray, img_off: Sequence[
     Either r (Eq. 2) or an explicit k_budget is given. k == 0 returns the
     all-zero mask without running the scoring pass, as Algorithm 1 does.
     """
-    n = k.shape[2]
+    n = np.asarray(k[0]).shape[1]
     kk = budget(r, n) if k_budget is None else int(k_budget)
     if kk == 0:
         return {"k": 0, "idx": np.zeros(0, dtype=np.int64), "mask": np.zeros(n, dtype=np.uint8)}

@@ -1,0 +1,377 @@
+// C ABI: host-side argument checks, workspace sizing and launch sequencing.
+// Every check runs before anything is enqueued; nothing here allocates.
+#include <atomic>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <string>
+
+#include "internal.cuh"
+
+using namespace conduit;
+
+namespace {
+
+std::atomic<int64_t> g_launches{0};
+
+thread_local std::string g_last_error;
+
+conduit_status fail(conduit_status code, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return code;
+}
+
+conduit_status cuda_fail(cudaError_t err, const char* what) {
+  return fail(CONDUIT_ERR_CUDA, "%s: %s", what, cudaGetErrorString(err));
+}
+
+constexpr size_t kAlign = 256;
+size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+conduit_status check_batch(const conduit_batch* b) {
+  if (!b) return fail(CONDUIT_ERR_INVALID_ARG, "batch is NULL");
+  if (b->num_requests < 1) return fail(CONDUIT_ERR_INVALID_ARG, "num_requests must be >= 1");
+  if (b->num_images < b->num_requests)
+    return fail(CONDUIT_ERR_INVALID_ARG, "num_images must be >= num_requests");
+  if (!b->tok_off || !b->img_off || !b->req_img_off || !b->q_off)
+    return fail(CONDUIT_ERR_INVALID_ARG, "a host offset array is NULL");
+  if (!b->tok_off_dev || !b->img_off_dev || !b->req_img_off_dev || !b->q_off_dev)
+    return fail(CONDUIT_ERR_INVALID_ARG, "a device offset array is NULL");
+  const int R = b->num_requests, K = b->num_images;
+  if (b->tok_off[0] != 0 || b->q_off[0] != 0 || b->req_img_off[0] != 0)
+    return fail(CONDUIT_ERR_INVALID_ARG, "tok_off, q_off and req_img_off must start at 0");
+  if (b->req_img_off[R] != K)
+    return fail(CONDUIT_ERR_INVALID_ARG, "req_img_off[R] must equal num_images");
+  for (int r = 0; r < R; ++r) {
+    if (b->tok_off[r + 1] <= b->tok_off[r])
+      return fail(CONDUIT_ERR_INVALID_ARG, "request %d has no visual tokens", r);
+    if (b->q_off[r + 1] < b->q_off[r])
+      return fail(CONDUIT_ERR_INVALID_ARG, "q_off must be non-decreasing (request %d)", r);
+    const int j0 = b->req_img_off[r], j1 = b->req_img_off[r + 1];
+    if (j1 <= j0) return fail(CONDUIT_ERR_INVALID_ARG, "request %d has no images", r);
+    if (j1 - j0 > kMaxImagesPerRequest)
+      return fail(CONDUIT_ERR_UNSUPPORTED, "request %d has more than %d images", r,
+                  kMaxImagesPerRequest);
+    if (b->img_off[j0] != b->tok_off[r] || b->img_off[j1] != b->tok_off[r + 1])
+      return fail(CONDUIT_ERR_INVALID_ARG, "images of request %d do not tile its tokens", r);
+    for (int j = j0; j < j1; ++j)
+      if (b->img_off[j + 1] <= b->img_off[j])
+        return fail(CONDUIT_ERR_INVALID_ARG, "image %d is empty or out of order", j);
+  }
+  return CONDUIT_OK;
+}
+
+conduit_status check_kv(const conduit_kv* kv, const conduit_batch* b) {
+  if (!kv) return fail(CONDUIT_ERR_INVALID_ARG, "kv is NULL");
+  if (kv->num_layers < 1 || kv->num_q_heads < 1 || kv->num_kv_heads < 1)
+    return fail(CONDUIT_ERR_INVALID_ARG, "layer and head counts must be >= 1");
+  if (kv->num_q_heads % kv->num_kv_heads)
+    return fail(CONDUIT_ERR_INVALID_ARG, "num_q_heads must be a multiple of num_kv_heads");
+  if (kv->head_dim < 8 || kv->head_dim > 256 || kv->head_dim % 8)
+    return fail(CONDUIT_ERR_UNSUPPORTED, "head_dim must be a multiple of 8 in [8, 256]");
+  if (kv->dtype != CONDUIT_F32 && kv->dtype != CONDUIT_BF16)
+    return fail(CONDUIT_ERR_INVALID_ARG, "dtype must be CONDUIT_F32 or CONDUIT_BF16");
+  if (!kv->k || !kv->v) return fail(CONDUIT_ERR_INVALID_ARG, "kv->k or kv->v is NULL");
+  if (!aligned16(kv->k) || !aligned16(kv->v))
+    return fail(CONDUIT_ERR_INVALID_ARG, "kv->k and kv->v must be 16-byte aligned");
+  if ((kv->num_q_heads / kv->num_kv_heads) * kv->head_dim > 4096)
+    return fail(CONDUIT_ERR_UNSUPPORTED, "(Hq/Hkv) * head_dim must be <= 4096");
+  if (kv->page_size < 0) return fail(CONDUIT_ERR_INVALID_ARG, "page_size must be >= 0");
+  if (kv->page_size > 0) {
+    if (!kv->page_table || kv->num_pages < 1 || kv->max_pages_per_req < 1)
+      return fail(CONDUIT_ERR_INVALID_ARG, "paged cache needs page_table, num_pages, max_pages_per_req");
+    for (int r = 0; r < b->num_requests; ++r) {
+      const int64_t n = b->tok_off[r + 1] - b->tok_off[r];
+      if (n > int64_t(kv->max_pages_per_req) * kv->page_size)
+        return fail(CONDUIT_ERR_INVALID_ARG, "request %d has more tokens than its page-table row holds", r);
+    }
+  }
+  return CONDUIT_OK;
+}
+
+KvDev make_kv(const conduit_kv* kv, const conduit_batch* b) {
+  KvDev d{};
+  d.k = kv->k;
+  d.v = kv->v;
+  d.L = kv->num_layers;
+  d.Hq = kv->num_q_heads;
+  d.Hkv = kv->num_kv_heads;
+  d.d = kv->head_dim;
+  d.G = kv->num_q_heads / kv->num_kv_heads;
+  d.dtype = kv->dtype;
+  d.page_size = kv->page_size;
+  d.num_pages = kv->num_pages;
+  d.max_pages = kv->max_pages_per_req;
+  d.page_table = kv->page_table;
+  d.n_tot = b->tok_off[b->num_requests];
+  return d;
+}
+
+BatchDev make_batch(const conduit_batch* b) {
+  return BatchDev{b->num_requests, b->num_images, b->tok_off_dev, b->img_off_dev,
+                  b->req_img_off_dev, b->q_off_dev};
+}
+
+conduit_status make_layers(const conduit_kv* kv, const int32_t* layers, int32_t n_layers,
+                           LayerList* out) {
+  if (!layers) {
+    if (n_layers != 0 && n_layers != kv->num_layers)
+      return fail(CONDUIT_ERR_INVALID_ARG, "layers == NULL needs n_layers == 0 or num_layers");
+    if (kv->num_layers > CONDUIT_MAX_LAYERS)
+      return fail(CONDUIT_ERR_UNSUPPORTED, "more than %d layers", CONDUIT_MAX_LAYERS);
+    out->n = kv->num_layers;
+    for (int i = 0; i < kv->num_layers; ++i) out->ids[i] = i;
+    return CONDUIT_OK;
+  }
+  if (n_layers < 1 || n_layers > CONDUIT_MAX_LAYERS)
+    return fail(CONDUIT_ERR_INVALID_ARG, "n_layers must be in [1, %d]", CONDUIT_MAX_LAYERS);
+  for (int i = 0; i < n_layers; ++i) {
+    if (layers[i] < 0 || layers[i] >= kv->num_layers)
+      return fail(CONDUIT_ERR_INVALID_ARG, "layer id %d out of range", layers[i]);
+    if (i && layers[i] <= layers[i - 1])
+      return fail(CONDUIT_ERR_INVALID_ARG, "layer ids must be strictly increasing");
+    out->ids[i] = layers[i];
+  }
+  out->n = n_layers;
+  return CONDUIT_OK;
+}
+
+struct ScoreLayout {
+  size_t stats, pa, ss, attn, total;
+};
+
+ScoreLayout score_layout(const conduit_kv* kv, const conduit_batch* b, int n_layers) {
+  const size_t n_tot = size_t(b->tok_off[b->num_requests]);
+  const size_t q_tot = size_t(b->q_off[b->num_requests]);
+  ScoreLayout s{};
+  size_t off = 0;
+  s.stats = off;
+  off += align_up(size_t(n_layers) * kv->num_q_heads * q_tot * sizeof(float2));
+  s.pa = off;
+  off += align_up(size_t(n_layers) * kv->num_kv_heads * n_tot * sizeof(float));
+  s.ss = off;
+  off += align_up(size_t(n_layers) * n_tot * sizeof(float));
+  s.attn = off;
+  off += align_up(n_tot * sizeof(float));
+  s.total = off;
+  return s;
+}
+
+conduit_status check_workspace(void* ws, size_t have, size_t need) {
+  if (need == 0) return CONDUIT_OK;
+  if (!ws) return fail(CONDUIT_ERR_WORKSPACE, "workspace is NULL but %zu bytes are needed", need);
+  if (reinterpret_cast<uintptr_t>(ws) % kAlign)
+    return fail(CONDUIT_ERR_WORKSPACE, "workspace must be 256-byte aligned");
+  if (have < need)
+    return fail(CONDUIT_ERR_WORKSPACE, "workspace has %zu bytes, %zu needed", have, need);
+  return CONDUIT_OK;
+}
+
+conduit_status check_selection(const conduit_batch* b, const int32_t* idx_off,
+                               const int32_t* idx_off_dev, bool need_idx, const int32_t* idx) {
+  if (!idx_off || !idx_off_dev)
+    return fail(CONDUIT_ERR_INVALID_ARG, "idx_off (host) and idx_off_dev (device) are required");
+  if (idx_off[0] != 0) return fail(CONDUIT_ERR_INVALID_ARG, "idx_off[0] must be 0");
+  for (int r = 0; r < b->num_requests; ++r) {
+    const int kr = idx_off[r + 1] - idx_off[r];
+    if (kr < 0 || kr > b->tok_off[r + 1] - b->tok_off[r])
+      return fail(CONDUIT_ERR_INVALID_ARG, "budget of request %d is outside [0, N_r]", r);
+  }
+  if (need_idx && idx_off[b->num_requests] > 0 && !idx)
+    return fail(CONDUIT_ERR_INVALID_ARG, "idx is NULL");
+  return CONDUIT_OK;
+}
+
+int max_budget(const conduit_batch* b, const int32_t* idx_off) {
+  int m = 0;
+  for (int r = 0; r < b->num_requests; ++r) m = std::max(m, idx_off[r + 1] - idx_off[r]);
+  return m;
+}
+
+}  // namespace
+
+namespace conduit {
+void count_launches(int n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
+}  // namespace conduit
+
+extern "C" {
+
+int32_t conduit_version(void) { return CONDUIT_VERSION; }
+
+int64_t conduit_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
+
+const char* conduit_last_error_string(void) { return g_last_error.c_str(); }
+
+int32_t conduit_budget(double r, int64_t n_vis) {
+  if (!(r >= 0.0 && r <= 1.0) || n_vis < 0) return -1;
+  const double k = std::floor(r * double(n_vis) + 1e-9);
+  return int32_t(std::min<double>(k, double(n_vis)));
+}
+
+conduit_status conduit_score_workspace_size(const conduit_kv* kv, const conduit_batch* batch,
+                                            int32_t n_layers, size_t* bytes) {
+  conduit_status st;
+  if (!bytes) return fail(CONDUIT_ERR_INVALID_ARG, "bytes is NULL");
+  if ((st = check_batch(batch)) || (st = check_kv(kv, batch))) return st;
+  const int nl = n_layers > 0 ? n_layers : kv->num_layers;
+  *bytes = score_layout(kv, batch, nl).total;
+  return CONDUIT_OK;
+}
+
+conduit_status conduit_score(const conduit_kv* kv, const conduit_batch* batch, const void* q,
+                             const int32_t* layers, int32_t n_layers, float* s, float* attn_sum,
+                             float* g, void* workspace, size_t workspace_bytes, int32_t* status,
+                             void* stream) {
+  conduit_status st;
+  if ((st = check_batch(batch)) || (st = check_kv(kv, batch))) return st;
+  if (!q || !s || !g) return fail(CONDUIT_ERR_INVALID_ARG, "q, s and g are required");
+  if (!aligned16(q)) return fail(CONDUIT_ERR_INVALID_ARG, "q must be 16-byte aligned");
+  for (int r = 0; r < batch->num_requests; ++r)
+    if (batch->q_off[r + 1] == batch->q_off[r])
+      return fail(CONDUIT_ERR_INVALID_ARG, "request %d has an empty scoring span", r);
+  static thread_local LayerList ll;
+  if ((st = make_layers(kv, layers, n_layers, &ll))) return st;
+  const ScoreLayout lay = score_layout(kv, batch, ll.n);
+  if ((st = check_workspace(workspace, workspace_bytes, lay.total))) return st;
+
+  const KvDev kd = make_kv(kv, batch);
+  const BatchDev bd = make_batch(batch);
+  const int R = batch->num_requests;
+  int max_tok = 0, max_rows = 0;
+  for (int r = 0; r < R; ++r) {
+    max_tok = std::max(max_tok, batch->tok_off[r + 1] - batch->tok_off[r]);
+    max_rows = std::max(max_rows, kd.G * (batch->q_off[r + 1] - batch->q_off[r]));
+  }
+  char* ws = static_cast<char*>(workspace);
+  float2* stats = reinterpret_cast<float2*>(ws + lay.stats);
+  float* pa = reinterpret_cast<float*>(ws + lay.pa);
+  float* ss = reinterpret_cast<float*>(ws + lay.ss);
+  float* attn = attn_sum ? attn_sum : reinterpret_cast<float*>(ws + lay.attn);
+  cudaStream_t cs = static_cast<cudaStream_t>(stream);
+  cudaError_t err;
+  if ((err = launch_value_sumsq(kd, bd, ll, max_tok, ss, cs))) return cuda_fail(err, "value_sumsq");
+  if ((err = launch_score_simt(kd, bd, q, batch->q_off[R], ll, max_rows, max_tok, stats, pa, cs)))
+    return cuda_fail(err, "score");
+  if ((err = launch_finalize(pa, ss, bd, ll.n, kd.Hkv, kd.Hq, kd.n_tot, s, attn, g, status, cs)))
+    return cuda_fail(err, "finalize");
+  return CONDUIT_OK;
+}
+
+conduit_status conduit_select_workspace_size(const conduit_batch* batch, size_t* bytes) {
+  conduit_status st;
+  if (!bytes) return fail(CONDUIT_ERR_INVALID_ARG, "bytes is NULL");
+  if ((st = check_batch(batch))) return st;
+  *bytes = align_up(size_t(batch->tok_off[batch->num_requests]) * sizeof(uint32_t));
+  return CONDUIT_OK;
+}
+
+conduit_status conduit_select_topk(const conduit_batch* batch, const float* s, const float* g,
+                                   float lambda, const int32_t* idx_off,
+                                   const int32_t* idx_off_dev, int32_t* idx, uint8_t* mask,
+                                   float* s_hat, float* coeff, void* workspace,
+                                   size_t workspace_bytes, int32_t* status, void* stream) {
+  conduit_status st;
+  if ((st = check_batch(batch))) return st;
+  if (!s || !g) return fail(CONDUIT_ERR_INVALID_ARG, "s and g are required");
+  if (!(lambda >= 0.f && lambda <= 1.f))
+    return fail(CONDUIT_ERR_INVALID_ARG, "lambda must lie in [0, 1]");
+  if ((st = check_selection(batch, idx_off, idx_off_dev, true, idx))) return st;
+  size_t need = 0;
+  conduit_select_workspace_size(batch, &need);
+  if ((st = check_workspace(workspace, workspace_bytes, need))) return st;
+  cudaError_t err = launch_select(make_batch(batch), s, g, lambda, idx_off_dev, idx, mask, s_hat,
+                                  coeff, static_cast<uint32_t*>(workspace), status,
+                                  static_cast<cudaStream_t>(stream));
+  if (err) return cuda_fail(err, "select");
+  return CONDUIT_OK;
+}
+
+static conduit_status kv_copy(const conduit_kv* kv, const conduit_batch* batch,
+                              const int32_t* idx, const int32_t* idx_off,
+                              const int32_t* idx_off_dev, const void* k_rows,
+                              const void* v_rows, bool scatter, void* stream) {
+  conduit_status st;
+  if ((st = check_batch(batch)) || (st = check_kv(kv, batch))) return st;
+  if ((st = check_selection(batch, idx_off, idx_off_dev, true, idx))) return st;
+  const int n_sel = idx_off[batch->num_requests];
+  if (n_sel > 0 && (!k_rows || !v_rows))
+    return fail(CONDUIT_ERR_INVALID_ARG, "k_rows and v_rows are required");
+  if (n_sel > 0 && (!aligned16(k_rows) || !aligned16(v_rows)))
+    return fail(CONDUIT_ERR_INVALID_ARG, "k_rows and v_rows must be 16-byte aligned");
+  cudaError_t err = launch_kv_copy(make_kv(kv, batch), make_batch(batch), idx, idx_off_dev, n_sel,
+                                   max_budget(batch, idx_off), scatter, const_cast<void*>(k_rows),
+                                   const_cast<void*>(v_rows), static_cast<cudaStream_t>(stream));
+  if (err) return cuda_fail(err, scatter ? "kv_scatter" : "kv_gather");
+  return CONDUIT_OK;
+}
+
+conduit_status conduit_kv_gather(const conduit_kv* kv, const conduit_batch* batch,
+                                 const int32_t* idx, const int32_t* idx_off,
+                                 const int32_t* idx_off_dev, void* k_rows, void* v_rows,
+                                 void* stream) {
+  return kv_copy(kv, batch, idx, idx_off, idx_off_dev, k_rows, v_rows, false, stream);
+}
+
+conduit_status conduit_kv_scatter(const conduit_kv* kv, const conduit_batch* batch,
+                                  const int32_t* idx, const int32_t* idx_off,
+                                  const int32_t* idx_off_dev, const void* k_rows,
+                                  const void* v_rows, void* stream) {
+  return kv_copy(kv, batch, idx, idx_off, idx_off_dev, k_rows, v_rows, true, stream);
+}
+
+conduit_status conduit_refresh_workspace_size(const conduit_kv* kv, const conduit_batch* batch,
+                                              const int32_t* idx_off, size_t* bytes) {
+  conduit_status st;
+  if (!bytes) return fail(CONDUIT_ERR_INVALID_ARG, "bytes is NULL");
+  if ((st = check_batch(batch)) || (st = check_kv(kv, batch))) return st;
+  (void)idx_off;
+  *bytes = 0;
+  return CONDUIT_OK;
+}
+
+conduit_status conduit_refresh_attn(const conduit_kv* kv, const conduit_batch* batch,
+                                    const int32_t* idx, const int32_t* idx_off,
+                                    const int32_t* idx_off_dev, const void* q_rows, void* out,
+                                    void* workspace, size_t workspace_bytes, int32_t* status,
+                                    void* stream) {
+  conduit_status st;
+  if ((st = check_batch(batch)) || (st = check_kv(kv, batch))) return st;
+  if ((st = check_selection(batch, idx_off, idx_off_dev, true, idx))) return st;
+  const int n_sel = idx_off[batch->num_requests];
+  if (n_sel == 0) return CONDUIT_OK;
+  if (!q_rows || !out) return fail(CONDUIT_ERR_INVALID_ARG, "q_rows and out are required");
+  (void)workspace;
+  (void)workspace_bytes;
+  (void)status;
+  cudaError_t err = launch_refresh_simt(make_kv(kv, batch), make_batch(batch), idx, idx_off_dev,
+                                        n_sel, q_rows, out, static_cast<cudaStream_t>(stream));
+  if (err) return cuda_fail(err, "refresh_attn");
+  return CONDUIT_OK;
+}
+
+conduit_status conduit_clear_status(int32_t* status, void* stream) {
+  if (!status) return fail(CONDUIT_ERR_INVALID_ARG, "status is NULL");
+  cudaError_t err = cudaMemsetAsync(status, 0, sizeof(int32_t), static_cast<cudaStream_t>(stream));
+  if (err) return cuda_fail(err, "clear_status");
+  return CONDUIT_OK;
+}
+
+conduit_status conduit_read_status(const int32_t* status, void* stream, int32_t* word) {
+  if (!status || !word) return fail(CONDUIT_ERR_INVALID_ARG, "status and word are required");
+  cudaError_t err = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+  if (err) return cuda_fail(err, "read_status (synchronize)");
+  err = cudaMemcpy(word, status, sizeof(int32_t), cudaMemcpyDeviceToHost);
+  if (err) return cuda_fail(err, "read_status (copy)");
+  if (*word & CONDUIT_FLAG_TIMEOUT) return CONDUIT_ERR_TIMEOUT;
+  if (*word & CONDUIT_FLAG_NONFINITE) return CONDUIT_ERR_NONFINITE;
+  return CONDUIT_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,172 @@
+// Image-level amplification and exact global top-k (Conduit Eqs. 9-11).
+//
+// One CTA per request:
+//   c_j = (1 - lambda) + lambda g_j / g_bar  (c = 1 for one image or g_bar = 0)
+//   s_hat_t = s_t c_{pi(t)}
+//   radix select over the float bit patterns (s_hat >= 0, so unsigned order
+//   equals value order; -0 is canonicalised to +0) finds the k-th largest
+//   key exactly; every key above it is taken, and keys equal to it are taken
+//   in ascending token order until k are chosen (ties to the lowest index).
+//   Selected indices are written in ascending order together with the mask.
+#include "internal.cuh"
+
+namespace conduit {
+namespace {
+
+constexpr int kSelThreads = 1024;
+
+// Block-wide exclusive scan of one int per thread; returns the prefix and
+// stores the block total in *total.
+__device__ __forceinline__ int block_exclusive_scan(int v, int* warp_s, int* total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  int x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) warp_s[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    int w = lane < (kSelThreads >> 5) ? warp_s[lane] : 0;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, w, o);
+      if (lane >= o) w += y;
+    }
+    if (lane < (kSelThreads >> 5)) warp_s[lane] = w;  // inclusive warp prefixes
+  }
+  __syncthreads();
+  const int before = (warp > 0 ? warp_s[warp - 1] : 0) + x - v;
+  if (total) *total = warp_s[(kSelThreads >> 5) - 1];
+  __syncthreads();
+  return before;
+}
+
+__global__ void __launch_bounds__(kSelThreads) select_kernel(BatchDev b, const float* s,
+                                                             const float* g, float lambda,
+                                                             const int32_t* idx_off, int32_t* idx,
+                                                             uint8_t* mask, float* s_hat,
+                                                             float* coeff, uint32_t* keys,
+                                                             int32_t* status) {
+  __shared__ float c_s[kMaxImagesPerRequest];
+  __shared__ int img_s[kMaxImagesPerRequest + 1];
+  __shared__ unsigned hist[256];
+  __shared__ int warp_s[32];
+  __shared__ uint32_t prefix_s;
+  __shared__ int remaining_s;
+  __shared__ float gbar_s;
+
+  const int r = blockIdx.x;
+  const int t0 = b.tok_off[r], N = b.tok_off[r + 1] - t0;
+  const int j0 = b.req_img_off[r], K = b.req_img_off[r + 1] - j0;
+  const int k = idx_off[r + 1] - idx_off[r];
+  int32_t* out = idx + idx_off[r];
+
+  // c_j (Eq. 9): g_bar in a fixed order by one thread.
+  for (int j = threadIdx.x; j <= K; j += blockDim.x) img_s[j] = b.img_off[j0 + j] - t0;
+  if (threadIdx.x == 0) {
+    float sum = 0.f;
+    for (int j = 0; j < K; ++j) sum += g[j0 + j];
+    gbar_s = sum / float(K);
+  }
+  __syncthreads();
+  const float gbar = gbar_s;
+  for (int j = threadIdx.x; j < K; j += blockDim.x) {
+    const float c = (K == 1 || gbar == 0.f) ? 1.f : (1.f - lambda) + lambda * (g[j0 + j] / gbar);
+    c_s[j] = c;
+    if (coeff) coeff[j0 + j] = c;
+  }
+  __syncthreads();
+
+  // s_hat (Eq. 10) and its sortable key.
+  bool bad = false;
+  for (int t = threadIdx.x; t < N; t += blockDim.x) {
+    int lo = 0, hi = K - 1;  // image of token t
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (img_s[mid] <= t) lo = mid; else hi = mid - 1;
+    }
+    float sh = s[t0 + t] * c_s[lo];
+    if (!isfinite(sh) || sh < 0.f) bad = true;
+    if (sh == 0.f) sh = 0.f;  // -0 -> +0
+    if (s_hat) s_hat[t0 + t] = sh;
+    keys[t0 + t] = __float_as_uint(sh);
+  }
+  if (bad) flag_status(status, CONDUIT_FLAG_NONFINITE);
+  __syncthreads();
+
+  if (k == 0) {
+    if (mask)
+      for (int t = threadIdx.x; t < N; t += blockDim.x) mask[t0 + t] = 0;
+    return;
+  }
+
+  // Radix select of the k-th largest key: four 8-bit digits, MSB first.
+  if (threadIdx.x == 0) {
+    prefix_s = 0u;
+    remaining_s = k;
+  }
+  uint32_t pmask = 0u;
+  for (int shift = 24; shift >= 0; shift -= 8) {
+    for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0u;
+    __syncthreads();
+    const uint32_t prefix = prefix_s;
+    for (int t = threadIdx.x; t < N; t += blockDim.x) {
+      const uint32_t key = keys[t0 + t];
+      if ((key & pmask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      int rem = remaining_s, digit = 255;
+      for (; digit > 0; --digit) {
+        const int c = int(hist[digit]);
+        if (c >= rem) break;
+        rem -= c;
+      }
+      remaining_s = rem;
+      prefix_s = prefix | (uint32_t(digit) << shift);
+    }
+    pmask |= 255u << shift;
+    __syncthreads();
+  }
+  const uint32_t kth = prefix_s;
+  const int need = remaining_s;  // keys equal to kth still to take, >= 1
+
+  // Contiguous token ranges per thread keep the output in ascending order.
+  const int per = (N + kSelThreads - 1) / kSelThreads;
+  const int lo = min(N, int(threadIdx.x) * per), hi = min(N, lo + per);
+  int gt = 0, eq = 0;
+  for (int t = lo; t < hi; ++t) {
+    const uint32_t key = keys[t0 + t];
+    gt += key > kth;
+    eq += key == kth;
+  }
+  const int eq_base = block_exclusive_scan(eq, warp_s, nullptr);
+  const int take_eq = max(0, min(eq, need - eq_base));
+  const int pos0 = block_exclusive_scan(gt + take_eq, warp_s, nullptr);
+  int pos = pos0, seen_eq = 0;
+  for (int t = lo; t < hi; ++t) {
+    const uint32_t key = keys[t0 + t];
+    bool sel = key > kth;
+    if (key == kth) {
+      sel = seen_eq < take_eq;
+      ++seen_eq;
+    }
+    if (sel) out[pos++] = t;
+    if (mask) mask[t0 + t] = sel ? 1 : 0;
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_select(const BatchDev& b, const float* s, const float* g, float lambda,
+                          const int32_t* idx_off_dev, int32_t* idx, uint8_t* mask, float* s_hat,
+                          float* coeff, uint32_t* keys, int32_t* status, cudaStream_t stream) {
+  select_kernel<<<b.R, kSelThreads, 0, stream>>>(b, s, g, lambda, idx_off_dev, idx, mask, s_hat,
+                                                 coeff, keys, status);
+  count_launches(1);
+  return cudaGetLastError();
+}
+
+}  // namespace conduit

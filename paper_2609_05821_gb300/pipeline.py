@@ -1,0 +1,158 @@
+"""One pass of Conduit's hot path over a batch: the user-facing step.
+
+``RefreshPipeline.step()`` enqueues, on one CUDA stream and through the C ABI:
+  1. conduit_score        scoring pass over the reused visual cache (Eqs. 6-8)
+  2. conduit_select_topk  amplification + one global top-k per request (Eqs. 9-11)
+  3. conduit_kv_gather    stale K/V rows of the selected tokens
+  4. conduit_kv_scatter   fresh K/V rows written into the cache
+  5. conduit_refresh_attn causal attention of the refreshed rows over the patched cache
+All buffers are allocated once at construction, so a step allocates nothing
+and can be captured in a CUDA graph (``capture()``). ``step_from_host()`` is
+the end-to-end form: it copies the step's inputs from pinned host memory,
+runs the step, and copies the selection and the refresh output back.
+"""
+
+from __future__ import annotations
+
+from typing import Optional, Sequence
+
+import torch
+
+from . import conduit as C
+
+
+class RefreshPipeline:
+    def __init__(self, k: torch.Tensor, v: torch.Tensor, q: torch.Tensor, num_q_heads: int,
+                 tok_off, img_off, req_img_off, q_off, ratios: Sequence[float],
+                 fresh: dict, lam: float = 1.0, layers: Optional[Sequence[int]] = None,
+                 page_size: int = 0, page_table: Optional[torch.Tensor] = None,
+                 budgets: Optional[Sequence[int]] = None):
+        dev = k.device
+        self.device = dev
+        self.kv = C.KvCache(k, v, num_q_heads, page_size, page_table)
+        self.batch = C.Batch(tok_off, img_off, req_img_off, q_off, device=dev)
+        self.q = q
+        self.lam = float(lam)
+        self.layers = None if layers is None else list(layers)
+        tok = self.batch.tok_off.tolist()
+        n_r = [tok[r + 1] - tok[r] for r in range(self.batch.num_requests)]
+        if budgets is None:
+            budgets = [C.conduit_budget(r, n) for r, n in zip(ratios, n_r)]
+        self.budgets = [int(x) for x in budgets]
+        self.idx_off, self.idx_off_dev = C.idx_offsets(self.budgets, dev)
+        self.n_sel = int(self.idx_off[-1])
+        n_tot, K = self.batch.n_tot, self.batch.num_images
+        f32 = dict(dtype=torch.float32, device=dev)
+        self.s = torch.empty(n_tot, **f32)
+        self.attn_sum = torch.empty(n_tot, **f32)
+        self.g = torch.empty(K, **f32)
+        self.s_hat = torch.empty(n_tot, **f32)
+        self.coeff = torch.empty(K, **f32)
+        self.mask = torch.empty(n_tot, dtype=torch.uint8, device=dev)
+        self.idx = torch.empty(max(self.n_sel, 1), dtype=torch.int32, device=dev)
+        self.status = torch.zeros(1, dtype=torch.int32, device=dev)
+        nl = 0 if self.layers is None else len(self.layers)
+        self.ws_score = torch.empty(max(C.conduit_score_workspace_size(self.kv, self.batch, nl), 1),
+                                    dtype=torch.uint8, device=dev)
+        self.ws_sel = torch.empty(max(C.conduit_select_workspace_size(self.batch), 1),
+                                  dtype=torch.uint8, device=dev)
+        need = C.conduit_refresh_workspace_size(self.kv, self.batch, self.idx_off)
+        self.ws_ref = torch.empty(need, dtype=torch.uint8, device=dev) if need else None
+        L, Hkv, Hq, d = self.kv.num_layers, self.kv.num_kv_heads, num_q_heads, self.kv.head_dim
+        self.q_rows = fresh["q_rows"]
+        self.k_rows = fresh["k_rows"]
+        self.v_rows = fresh["v_rows"]
+        assert self.q_rows.shape == (L, self.n_sel, Hq, d)
+        self.k_old = torch.empty((L, self.n_sel, Hkv, d), dtype=k.dtype, device=dev)
+        self.v_old = torch.empty_like(self.k_old)
+        self.out = torch.empty_like(self.q_rows)
+        self.graph = None
+
+    # ----------------------------------------------------------------- steps
+    def score_select(self, stream=None):
+        C.conduit_score(self.kv, self.batch, self.q, self.layers, self.s, self.attn_sum, self.g,
+                        self.ws_score, self.status, stream)
+        C.conduit_select_topk(self.batch, self.s, self.g, self.lam, self.idx_off, self.idx_off_dev,
+                              self.idx, self.mask, self.s_hat, self.coeff, self.ws_sel,
+                              self.status, stream)
+
+    def refresh(self, stream=None):
+        C.conduit_kv_gather(self.kv, self.batch, self.idx, self.idx_off, self.idx_off_dev,
+                            self.k_old, self.v_old, stream)
+        C.conduit_kv_scatter(self.kv, self.batch, self.idx, self.idx_off, self.idx_off_dev,
+                             self.k_rows, self.v_rows, stream)
+        C.conduit_refresh_attn(self.kv, self.batch, self.idx, self.idx_off, self.idx_off_dev,
+                               self.q_rows, self.out, self.ws_ref, self.status, stream)
+
+    def step(self, stream=None):
+        """One pass of the whole hot path (launches only; asynchronous)."""
+        if self.graph is not None:
+            self.graph.replay()
+            return
+        self.score_select(stream)
+        self.refresh(stream)
+
+    def capture(self):
+        """Capture one step in a CUDA graph; later step() calls replay it."""
+        s = torch.cuda.Stream(device=self.device)
+        s.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(s):
+            self.score_select(s)
+            self.refresh(s)
+        torch.cuda.current_stream().wait_stream(s)
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            self.score_select()
+            self.refresh()
+        self.graph = g
+
+    # ------------------------------------------------------------- end to end
+    def host_buffers(self) -> dict:
+        """Pinned host copies of everything a step consumes and returns."""
+        pin = lambda t: torch.empty(t.shape, dtype=t.dtype, pin_memory=True).copy_(t)
+        return {
+            "k": pin(self.kv.k), "v": pin(self.kv.v), "q": pin(self.q),
+            "q_rows": pin(self.q_rows), "k_rows": pin(self.k_rows), "v_rows": pin(self.v_rows),
+            "idx": torch.empty(self.idx.shape, dtype=torch.int32, pin_memory=True),
+            "out": torch.empty(self.out.shape, dtype=self.out.dtype, pin_memory=True),
+        }
+
+    def step_from_host(self, host: dict):
+        """H2D copy of the cache, queries and fresh rows; the step; D2H of idx and out."""
+        for name, dst in (("k", self.kv.k), ("v", self.kv.v), ("q", self.q),
+                          ("q_rows", self.q_rows), ("k_rows", self.k_rows), ("v_rows", self.v_rows)):
+            dst.copy_(host[name], non_blocking=True)
+        self.step()
+        host["idx"].copy_(self.idx, non_blocking=True)
+        host["out"].copy_(self.out, non_blocking=True)
+
+    def h2d_bytes(self) -> int:
+        ts = (self.kv.k, self.kv.v, self.q, self.q_rows, self.k_rows, self.v_rows)
+        return sum(t.numel() * t.element_size() for t in ts)
+
+    def d2h_bytes(self) -> int:
+        return self.idx.numel() * 4 + self.out.numel() * self.out.element_size()
+
+
+def from_inputs(inputs: dict, lam: float = 1.0, paged: Optional[bool] = None,
+                layers=None, budgets=None, fresh: Optional[dict] = None) -> RefreshPipeline:
+    """A pipeline over a batch drawn by ``synth.make_inputs``."""
+    from . import synth
+    w = inputs["workload"]
+    dev = inputs["k"].device
+    tok = inputs["tok_off"].tolist()
+    n_r = [tok[r + 1] - tok[r] for r in range(len(tok) - 1)]
+    if budgets is None:
+        budgets = [C.conduit_budget(r, n) for r, n in zip(inputs["ratios"], n_r)]
+    if fresh is None:
+        fresh = synth.make_fresh_rows(w, sum(budgets), device=dev)
+    paged = bool(w.page_size) if paged is None else paged
+    k, v, table, ps = inputs["k"], inputs["v"], None, 0
+    if paged:
+        ps = w.page_size or 16
+        k, table = synth.to_paged(inputs["k"], tok, ps, w.seed)
+        v, _ = synth.to_paged(inputs["v"], tok, ps, w.seed)
+    return RefreshPipeline(k, v, inputs["q"], w.num_q_heads, inputs["tok_off"], inputs["img_off"],
+                           inputs["req_img_off"], inputs["q_off"], inputs["ratios"], fresh, lam=lam,
+                           layers=layers, page_size=ps, page_table=table, budgets=budgets)

@@ -1,0 +1,166 @@
+"""The C ABI on the host: exported symbols and argument checks (no GPU needed).
+
+Every call here fails its host-side checks, which run before anything is
+enqueued, so none of them touches a device.
+"""
+
+import ctypes
+import os
+import re
+import subprocess
+
+import pytest
+import torch
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "conduit.h")
+
+
+@pytest.fixture(scope="module")
+def C():
+    from paper_2609_05821_gb300 import _build
+    _build.build()
+    from paper_2609_05821_gb300 import conduit
+    return conduit
+
+
+def _declared():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(conduit_[a-z_]+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = _declared()
+    for want in ("conduit_score", "conduit_select_topk", "conduit_refresh_attn", "conduit_kv_scatter",
+                 "conduit_kv_gather", "conduit_budget", "conduit_score_workspace_size",
+                 "conduit_read_status"):
+        assert want in names
+
+
+def test_library_exports_every_declared_symbol(C):
+    lib = ctypes.CDLL(C.LIB_PATH)
+    missing = [n for n in _declared() if not hasattr(lib, n)]
+    assert missing == []
+    nm = subprocess.run(["nm", "-D", "--defined-only", C.LIB_PATH], capture_output=True, text=True)
+    exported = set(re.findall(r"\bT (conduit_[a-z_]+)\b", nm.stdout))
+    assert set(_declared()) <= exported
+
+
+def test_version_and_budget(C):
+    assert C.conduit_version() == 100
+    assert C.conduit_budget(0.10, 256) == 25
+    assert C.conduit_budget(0.10, 1024) == 102
+    assert C.conduit_budget(0.05, 41472) == 2073
+    assert C.conduit_budget(0.20, 41472) == 8294
+    assert C.conduit_budget(0.3, 10) == 3
+    assert C.conduit_budget(0.0, 999) == 0
+    assert C.conduit_budget(1.0, 999) == 999
+    assert C.conduit_budget(-0.01, 10) == -1
+    assert C.conduit_budget(1.01, 10) == -1
+    assert C.conduit_budget(float("nan"), 10) == -1
+    assert C.conduit_budget(0.5, -1) == -1
+
+
+def test_budget_matches_oracle(C):
+    from oracle import conduit_oracle as O
+    for r in (0.0, 0.01, 0.05, 0.1, 0.125, 0.2, 0.3, 0.7, 0.99, 1.0):
+        for n in (1, 7, 10, 256, 1000, 1024, 8192, 41472):
+            assert C.conduit_budget(r, n) == O.budget(r, n)
+
+
+def _batch(C, tok=(0, 64, 128), img=(0, 32, 64, 128), rio=(0, 2, 3), qo=(0, 4, 8)):
+    return C.Batch(list(tok), list(img), list(rio), list(qo), device="cpu")
+
+
+def _kv(C, L=2, Hq=4, Hkv=2, d=64, n=128, dtype=torch.bfloat16, **kw):
+    k = torch.zeros((L, Hkv, n, d), dtype=dtype)
+    return C.KvCache(k, torch.zeros_like(k), Hq, **kw)
+
+
+def _expect(C, code, fn, *args, match=None):
+    with pytest.raises(C.ConduitError) as ei:
+        fn(*args)
+    assert ei.value.code == code, str(ei.value)
+    if match:
+        assert re.search(match, str(ei.value)), str(ei.value)
+
+
+def test_score_rejects_bad_arguments(C):
+    kv, b = _kv(C), _batch(C)
+    q = torch.zeros((2, 4, 8, 64), dtype=torch.bfloat16)
+    ws = torch.zeros(1, dtype=torch.uint8)
+    # workspace too small / missing
+    _expect(C, C.ERR_WORKSPACE, C.conduit_score, kv, b, q, None, None, None, None, ws)
+    # unsorted images
+    bad = _batch(C, img=(0, 70, 64, 128))
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_score, kv, bad, q, match="empty or out of order")
+    # images that do not tile the request
+    bad = _batch(C, img=(0, 32, 60, 128))
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_score, kv, bad, q, match="tile")
+    # empty request
+    bad = _batch(C, tok=(0, 0, 128), img=(0, 0, 64, 128))
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_score, kv, bad, q)
+    # empty scoring span
+    bad = _batch(C, qo=(0, 0, 8))
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_score, kv, bad, q, match="scoring span")
+    # layer ids
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_score, kv, b, q, [1, 0], match="increasing")
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_score, kv, b, q, [5], match="out of range")
+    # head mismatch
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_score, _kv(C, Hq=5), b, q, match="multiple")
+    # head_dim
+    _expect(C, C.ERR_UNSUPPORTED, C.conduit_score, _kv(C, d=12), b, q, match="head_dim")
+    # null query
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_score, kv, b, None)
+
+
+def test_select_rejects_bad_budgets_and_lambda(C):
+    b = _batch(C)
+    s = torch.zeros(128)
+    g = torch.zeros(3)
+    off, off_d = C.idx_offsets([10, 65], "cpu")          # 65 > 64 tokens of request 1
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_select_topk, b, s, g, 1.0, off, off_d, match="budget")
+    off, off_d = C.idx_offsets([10, 5], "cpu")
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_select_topk, b, s, g, 1.5, off, off_d, match="lambda")
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_select_topk, b, s, g, float("nan"), off, off_d)
+    ws = torch.zeros(8, dtype=torch.uint8)
+    _expect(C, C.ERR_WORKSPACE, C.conduit_select_topk, b, s, g, 1.0, off, off_d, None, None, None,
+            None, ws)
+
+
+def test_kv_copy_and_refresh_reject_bad_arguments(C):
+    kv, b = _kv(C), _batch(C)
+    off, off_d = C.idx_offsets([3, 4], "cpu")
+    idx = torch.zeros(7, dtype=torch.int32)
+    rows = torch.zeros((2, 7, 2, 64), dtype=torch.bfloat16)
+    bad_off = torch.tensor([1, 3, 7], dtype=torch.int32)
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_kv_scatter, kv, b, idx, bad_off, off_d, rows, rows)
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_kv_gather, kv, b, idx, off, None, rows, rows)
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_refresh_attn, kv, b, None, off, off_d, rows)
+    paged = torch.zeros((2, 8, 2, 16, 64), dtype=torch.bfloat16)
+    table = torch.zeros((2, 3), dtype=torch.int32)      # 3 pages x 16 < 64 tokens
+    kvp = C.KvCache(paged, torch.zeros_like(paged), 4, 16, table)
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_kv_scatter, kvp, b, idx, off, off_d, rows, rows,
+            match="page-table")
+
+
+def test_kv_cache_python_checks(C):
+    k = torch.zeros((1, 2, 8, 64), dtype=torch.float16)
+    _expect(C, C.ERR_UNSUPPORTED, C.KvCache, k, k.clone(), 2)
+    k = torch.zeros((1, 2, 8, 64))
+    _expect(C, C.ERR_INVALID_ARG, C.KvCache, k, torch.zeros((1, 2, 8, 32)), 2)
+
+
+def test_last_error_is_thread_local(C):
+    import threading
+    kv, b = _kv(C), _batch(C)
+    q = torch.zeros((2, 4, 8, 64), dtype=torch.bfloat16)
+    with pytest.raises(C.ConduitError):
+        C.conduit_score(kv, b, q, [9])
+    main_msg = C._lib.conduit_last_error_string().decode()
+    seen = []
+    t = threading.Thread(target=lambda: seen.append(C._lib.conduit_last_error_string().decode()))
+    t.start()
+    t.join()
+    assert seen == [""] and "out of range" in main_msg
