@@ -80,6 +80,9 @@ class ClockSampler:
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self._t = threading.Thread(target=self._read, daemon=True)
             self._t.start()
+            t_end = time.time() + 5.0  # the timed region starts once sampling runs
+            while not self.lines and time.time() < t_end and self.proc.poll() is None:
+                time.sleep(0.02)
         except Exception:
             self.proc = None
         return self
@@ -90,6 +93,9 @@ class ClockSampler:
 
     def __exit__(self, *a):
         if self.proc is not None:
+            n0, t_end = len(self.lines), time.time() + 1.0  # one sample after the region
+            while len(self.lines) == n0 and time.time() < t_end:
+                time.sleep(0.02)
             self.proc.terminate()
             try:
                 self.proc.wait(timeout=5)
@@ -424,10 +430,18 @@ def oracle_step_sample(cfg: str, budget_seconds: float, seed_inputs=None):
 
 
 def cpu_baseline(cfg: str, seconds: float) -> dict:
+    """The oracle, as it stands, on the host cores: repeated bounded samples for ~`seconds`."""
+    from paper_2609_05821_gb300 import synth
     n_tok = _workload_tokens(cfg)
-    est, desc, spent = oracle_step_sample(cfg, seconds)
+    inputs = synth.make_inputs(synth.workload(cfg), device="cpu")
+    ests, spent, desc = [], 0.0, ""
+    while spent < seconds:
+        est, desc, dt = oracle_step_sample(cfg, seconds, inputs)
+        ests.append(est)
+        spent += dt
+    est = statistics.median(ests)
     return {"value": round(n_tok / est, 2), "unit": UNIT, "cores": _CORES, "kind": "oracle",
-            "sample": desc, "sample_seconds": round(spent, 1),
+            "sample": f"{len(ests)} repetition(s) of: {desc}", "sample_seconds": round(spent, 1),
             "threads_note": f"numpy BLAS threads = {_CORES}; elementwise numpy is single-threaded"}
 
 

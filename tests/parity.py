@@ -7,7 +7,9 @@ Tolerances (written here once, used by every parity test):
   selection        |T_gpu| = k and T_gpu, T_ref agree outside the band of
                    tokens whose oracle s_hat lies within rtol of the k-th value
   gather/scatter   bitwise (they copy the given rows)
-  refresh output   <= 2e-2 absolute for bf16, 1e-5 relative (+1e-6 abs) for fp32
+  refresh output   bf16: <= 2e-2 absolute + 2^-8 relative (the output is stored in
+                   bf16, whose half-ulp is 2^-8 of the value); fp32: 1e-5
+                   relative + 1e-6 absolute
 """
 
 from __future__ import annotations
