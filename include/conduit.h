@@ -167,6 +167,32 @@ conduit_status conduit_select_topk(const conduit_batch* batch, const float* s, c
                                    void* stream);
 
 /*
+ * conduit_select_topk without a caller workspace. The paper has no
+ * counterpart: this is a convenience of this library for callers that cannot
+ * hand it device scratch memory, for instance a serving engine that has
+ * given all free device memory to its paged KV pool and keeps no allocator
+ * handle on this path, or plain C code with no device allocator at all.
+ * Arguments and results are those of conduit_select_topk, minus workspace.
+ *  - Scratch comes from one static device array of the library, sized for
+ *    CONDUIT_NOALLOC_MAX_TOKENS tokens (4 MiB), which every GPU that loads
+ *    the library keeps until the process exits. A batch with more tokens
+ *    (tok_off[R]) is rejected with CONDUIT_ERR_UNSUPPORTED.
+ *  - The first call on a device looks up the array's device address with
+ *    that device current; make that first call before any stream capture.
+ *  - The call allocates nothing: no cudaMalloc, cudaFree or other
+ *    allocating routine.
+ *  - All calls share the array and it keeps the last call's contents. Each
+ *    call rewrites the part it reads, but calls whose work overlaps on the
+ *    GPU (other streams, other host threads) race on it: order them.
+ */
+#define CONDUIT_NOALLOC_MAX_TOKENS (1 << 20)
+conduit_status conduit_select_topk_noalloc(const conduit_batch* batch, const float* s,
+                                           const float* g, float lambda, const int32_t* idx_off,
+                                           const int32_t* idx_off_dev, int32_t* idx,
+                                           uint8_t* mask, float* s_hat, float* coeff,
+                                           int32_t* status, void* stream);
+
+/*
  * Gather of the selected rows of every layer (selective recompute, Sec. 3.1
  * and 3.5): k_rows[l][i][g][:] = K[l][g][idx_i][:] (same for V), where i runs
  * over all requests' selections in idx order.

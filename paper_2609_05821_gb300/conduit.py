@@ -69,6 +69,7 @@ def _load():
         "conduit_score": (st, [P, P, P, P, I32, P, P, P, P, SZ, P, P]),
         "conduit_select_workspace_size": (st, [P, ctypes.POINTER(SZ)]),
         "conduit_select_topk": (st, [P, P, P, ctypes.c_float, P, P, P, P, P, P, P, SZ, P, P]),
+        "conduit_select_topk_noalloc": (st, [P, P, P, ctypes.c_float, P, P, P, P, P, P, P, P]),
         "conduit_kv_gather": (st, [P, P, P, P, P, P, P, P]),
         "conduit_kv_scatter": (st, [P, P, P, P, P, P, P, P]),
         "conduit_refresh_workspace_size": (st, [P, P, P, ctypes.POINTER(SZ)]),
@@ -256,6 +257,24 @@ def conduit_select_topk(batch: Batch, s: torch.Tensor, g: torch.Tensor, lam: flo
                                     _ptr(coeff), _ptr(ws), ws.numel(), _ptr(status),
                                     _stream_ptr(stream)))
     return idx[:n_sel], mask, s_hat, coeff
+
+
+NOALLOC_MAX_TOKENS = 1 << 20
+
+
+def conduit_select_topk_noalloc(batch: Batch, s: torch.Tensor, g: torch.Tensor, lam: float,
+                                idx_off: torch.Tensor, idx_off_dev: torch.Tensor, idx: torch.Tensor,
+                                mask=None, s_hat=None, coeff=None, status=None, stream=None):
+    """conduit_select_topk with the library's static scratch instead of a workspace.
+
+    For callers that cannot give the library device scratch memory. Outputs
+    must be preallocated by the caller; nothing here or in the C call allocates.
+    """
+    _check(_lib.conduit_select_topk_noalloc(batch.ref(), _ptr(s), _ptr(g), float(lam),
+                                            _ptr(idx_off), _ptr(idx_off_dev), _ptr(idx),
+                                            _ptr(mask), _ptr(s_hat), _ptr(coeff), _ptr(status),
+                                            _stream_ptr(stream)))
+    return idx, mask, s_hat, coeff
 
 
 def conduit_kv_gather(kv: KvCache, batch: Batch, idx, idx_off, idx_off_dev, k_rows=None,

@@ -293,6 +293,28 @@ conduit_status conduit_select_topk(const conduit_batch* batch, const float* s, c
   return CONDUIT_OK;
 }
 
+conduit_status conduit_select_topk_noalloc(const conduit_batch* batch, const float* s,
+                                           const float* g, float lambda, const int32_t* idx_off,
+                                           const int32_t* idx_off_dev, int32_t* idx,
+                                           uint8_t* mask, float* s_hat, float* coeff,
+                                           int32_t* status, void* stream) {
+  conduit_status st;
+  if ((st = check_batch(batch))) return st;
+  if (!s || !g) return fail(CONDUIT_ERR_INVALID_ARG, "s and g are required");
+  if (!(lambda >= 0.f && lambda <= 1.f))
+    return fail(CONDUIT_ERR_INVALID_ARG, "lambda must lie in [0, 1]");
+  if ((st = check_selection(batch, idx_off, idx_off_dev, true, idx))) return st;
+  const int64_t n_tot = batch->tok_off[batch->num_requests];
+  if (n_tot > select_noalloc_max_tokens() || n_tot > CONDUIT_NOALLOC_MAX_TOKENS)
+    return fail(CONDUIT_ERR_UNSUPPORTED,
+                "batch has %lld tokens; the static scratch of conduit_select_topk_noalloc holds %d",
+                static_cast<long long>(n_tot), CONDUIT_NOALLOC_MAX_TOKENS);
+  cudaError_t err = launch_select_noalloc(make_batch(batch), s, g, lambda, idx_off_dev, idx, mask,
+                                          s_hat, coeff, status, static_cast<cudaStream_t>(stream));
+  if (err) return cuda_fail(err, "select_noalloc");
+  return CONDUIT_OK;
+}
+
 static conduit_status kv_copy(const conduit_kv* kv, const conduit_batch* batch,
                               const int32_t* idx, const int32_t* idx_off,
                               const int32_t* idx_off_dev, const void* k_rows,

@@ -88,6 +88,12 @@ cudaError_t launch_finalize(const float* pa, const float* ss, const BatchDev& b,
 cudaError_t launch_select(const BatchDev& b, const float* s, const float* g, float lambda,
                           const int32_t* idx_off_dev, int32_t* idx, uint8_t* mask, float* s_hat,
                           float* coeff, uint32_t* keys, int32_t* status, cudaStream_t stream);
+// Same selection with the keys in the library's static device array.
+int64_t select_noalloc_max_tokens();
+cudaError_t launch_select_noalloc(const BatchDev& b, const float* s, const float* g, float lambda,
+                                  const int32_t* idx_off_dev, int32_t* idx, uint8_t* mask,
+                                  float* s_hat, float* coeff, int32_t* status,
+                                  cudaStream_t stream);
 cudaError_t launch_kv_copy(const KvDev& kv, const BatchDev& b, const int32_t* idx,
                            const int32_t* idx_off_dev, int32_t n_sel, int max_sel, bool scatter,
                            void* k_rows, void* v_rows, cudaStream_t stream);

@@ -8,6 +8,8 @@
 //   key exactly; every key above it is taken, and keys equal to it are taken
 //   in ascending token order until k are chosen (ties to the lowest index).
 //   Selected indices are written in ascending order together with the mask.
+#include <mutex>
+
 #include "internal.cuh"
 
 namespace conduit {
@@ -158,7 +160,45 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(BatchDev b, const f
   }
 }
 
+// Scratch of conduit_select_topk_noalloc: the sortable keys of up to
+// kNoAllocMaxTokens tokens (4 MiB), resident on every device that loads the
+// library until the process exits. Each call overwrites the keys of its own
+// tokens before reading them, so nothing needs clearing between calls.
+constexpr int64_t kNoAllocMaxTokens = int64_t(1) << 20;
+static __device__ __align__(256) uint32_t g_noalloc_keys[kNoAllocMaxTokens];
+
+constexpr int kMaxDevices = 64;
+uint32_t* g_noalloc_ptr[kMaxDevices] = {};
+std::mutex g_noalloc_mu;
+
 }  // namespace
+
+int64_t select_noalloc_max_tokens() { return kNoAllocMaxTokens; }
+
+cudaError_t launch_select_noalloc(const BatchDev& b, const float* s, const float* g, float lambda,
+                                  const int32_t* idx_off_dev, int32_t* idx, uint8_t* mask,
+                                  float* s_hat, float* coeff, int32_t* status,
+                                  cudaStream_t stream) {
+  int dev = 0;
+  cudaError_t err = cudaGetDevice(&dev);
+  if (err) return err;
+  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+  uint32_t* keys = nullptr;
+  {
+    // Set-up once per device, with that device current: the host-side name of
+    // the array is not a device address, so ask the runtime for the address.
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    if (!g_noalloc_ptr[dev]) {
+      void* p = nullptr;
+      err = cudaGetSymbolAddress(&p, g_noalloc_keys);
+      if (err) return err;
+      g_noalloc_ptr[dev] = static_cast<uint32_t*>(p);
+    }
+    keys = g_noalloc_ptr[dev];
+  }
+  return launch_select(b, s, g, lambda, idx_off_dev, idx, mask, s_hat, coeff, keys, status,
+                       stream);
+}
 
 cudaError_t launch_select(const BatchDev& b, const float* s, const float* g, float lambda,
                           const int32_t* idx_off_dev, int32_t* idx, uint8_t* mask, float* s_hat,
