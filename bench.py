@@ -180,33 +180,42 @@ def work_model(pipe) -> dict:
     }
 
 
-CALL_KERNELS = {  # kernels behind each C-ABI call in this build, and their bound
-    "score": (["value_sumsq_kernel", "rowstats_kernel", "colsum_kernel", "finalize_tokens_kernel",
-               "image_means_kernel"], "alu"),
-    "select": (["select_kernel"], "hbm"),
-    "gather": (["kv_copy_kernel"], "hbm"),
-    "scatter": (["kv_copy_kernel"], "hbm"),
-    "refresh": (["refresh_simt_kernel"], "alu"),
-}
-KERNEL_SOURCES = {"score": "score_simt.cu", "select": "select.cu", "gather": "kvcopy.cu",
-                  "scatter": "kvcopy.cu", "refresh": "refresh_simt.cu"}
+def call_kernels(pipe) -> dict:
+    """Kernels behind each C-ABI call for this cache, their binding unit and source file.
+
+    bf16 caches with head_dim 128 take the tensor-core kernels; other shapes
+    the CUDA-core ones (the library makes the same choice).
+    """
+    tc = pipe.kv.k.dtype == torch.bfloat16 and pipe.kv.head_dim == 128
+    tail = ["finalize_tokens_kernel", "image_means_kernel"]
+    if tc:
+        score = (["value_sumsq_kernel", "rowstats_tc_kernel", "colsum_tc_kernel"] + tail, "hbm", "score_tc.cu")
+        refresh = (["refresh_tc_kernel"], "tensor", "refresh_tc.cu")
+    else:
+        score = (["value_sumsq_kernel", "rowstats_kernel", "colsum_kernel"] + tail, "alu", "score_simt.cu")
+        refresh = (["refresh_simt_kernel"], "alu", "refresh_simt.cu")
+    return {"score": score, "select": (["select_kernel"], "hbm", "select.cu"),
+            "gather": (["kv_copy_kernel"], "hbm", "kvcopy.cu"),
+            "scatter": (["kv_copy_kernel"], "hbm", "kvcopy.cu"), "refresh": refresh}
 
 
-def _src_hash(call: str) -> str:
-    p = os.path.join(ROOT, "paper_2609_05821_gb300", "csrc", KERNEL_SOURCES[call])
-    with open(p, "rb") as f:
+def _src_hash(src: str) -> str:
+    with open(os.path.join(ROOT, "paper_2609_05821_gb300", "csrc", src), "rb") as f:
         return hashlib.sha256(f.read()).hexdigest()[:12]
 
 
-def _traffic(call: str, workload: str):
-    """DRAM bytes per launch from a committed ncu summary, if its source hash still matches."""
+def _traffic(call: str, workload: str, src: str):
+    """DRAM bytes per launch from a committed ncu summary, if the kernel source is unchanged.
+
+    profiles/traffic.txt lines: <call> <workload> <bytes per launch> <sha256[:12] of the source>.
+    """
     p = os.path.join(ROOT, "profiles", "traffic.txt")
     if not os.path.exists(p):
         return None
     for line in open(p):
         f = line.split()
         if len(f) >= 4 and not line.startswith("#") and f[0] == call and f[1] == workload:
-            return float(f[2]) if f[3] == _src_hash(call) else None
+            return float(f[2]) if f[3] == _src_hash(src) else None
     return None
 
 
@@ -310,7 +319,7 @@ def run_conduit(args):
     # roofline of the dominant call
     model = work_model(pipe)
     dom = max(call_ms, key=call_ms.get)
-    kernels, bound = CALL_KERNELS[dom]
+    kernels, bound, src = call_kernels(pipe)[dom]
     sec = call_ms[dom] / 1e3
     if bound == "hbm":
         achieved, peak, unit = model[dom]["bytes"] / sec / 1e9, hbm, "GB/s"
@@ -321,7 +330,7 @@ def run_conduit(args):
     else:
         achieved, peak, unit = model[dom]["flops"] / sec / 1e12, ALU_FP32_TFLOPS, "TFLOP/s"
         peak_note = "fp32 FMA: 152 SMs x 128 lanes x 2 FLOP x 2.07 GHz"
-    traffic = _traffic(dom, args.config)
+    traffic = _traffic(dom, args.config, src)
     roofline = {"bound": bound, "achieved": round(achieved, 3), "peak": round(peak, 1), "unit": unit,
                 "frac": round(achieved / peak, 4), "traffic": traffic, "kernel": dom,
                 "kernels": kernels, "peak_source": peak_note,

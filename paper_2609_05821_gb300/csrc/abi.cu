@@ -144,16 +144,28 @@ conduit_status make_layers(const conduit_kv* kv, const int32_t* layers, int32_t 
 }
 
 struct ScoreLayout {
+  bool tc;     // tensor-core kernels (bf16, head_dim 128) or the CUDA-core ones
+  int chunk;   // tokens per tensor-core work unit
+  int max_tok;
   size_t stats, pa, ss, attn, total;
 };
 
 ScoreLayout score_layout(const conduit_kv* kv, const conduit_batch* b, int n_layers) {
-  const size_t n_tot = size_t(b->tok_off[b->num_requests]);
-  const size_t q_tot = size_t(b->q_off[b->num_requests]);
+  const int R = b->num_requests;
+  const size_t n_tot = size_t(b->tok_off[R]);
+  const size_t q_tot = size_t(b->q_off[R]);
   ScoreLayout s{};
+  s.tc = score_tc_supported(make_kv(kv, b));
+  for (int r = 0; r < R; ++r) s.max_tok = std::max(s.max_tok, b->tok_off[r + 1] - b->tok_off[r]);
+  const int64_t total_rows = int64_t(n_layers) * kv->num_q_heads * int64_t(q_tot);
   size_t off = 0;
   s.stats = off;
-  off += align_up(size_t(n_layers) * kv->num_q_heads * q_tot * sizeof(float2));
+  if (s.tc) {  // partial (max, sum) per row and token chunk
+    s.chunk = score_tc_chunk(R, b->tok_off, n_layers, kv->num_kv_heads);
+    off += align_up(score_tc_part_bytes(s.chunk, s.max_tok, total_rows));
+  } else {     // final (max, sum) per row
+    off += align_up(size_t(total_rows) * sizeof(float2));
+  }
   s.pa = off;
   off += align_up(size_t(n_layers) * kv->num_kv_heads * n_tot * sizeof(float));
   s.ss = off;
@@ -257,8 +269,11 @@ conduit_status conduit_score(const conduit_kv* kv, const conduit_batch* batch, c
   cudaStream_t cs = static_cast<cudaStream_t>(stream);
   cudaError_t err;
   if ((err = launch_value_sumsq(kd, bd, ll, max_tok, ss, cs))) return cuda_fail(err, "value_sumsq");
-  if ((err = launch_score_simt(kd, bd, q, batch->q_off[R], ll, max_rows, max_tok, stats, pa, cs)))
-    return cuda_fail(err, "score");
+  if (lay.tc)
+    err = launch_score_tc(kd, bd, q, batch->q_off[R], ll, max_tok, lay.chunk, stats, pa, status, cs);
+  else
+    err = launch_score_simt(kd, bd, q, batch->q_off[R], ll, max_rows, max_tok, stats, pa, cs);
+  if (err) return cuda_fail(err, "score");
   if ((err = launch_finalize(pa, ss, bd, ll.n, kd.Hkv, kd.Hq, kd.n_tot, s, attn, g, status, cs)))
     return cuda_fail(err, "finalize");
   return CONDUIT_OK;
@@ -372,8 +387,13 @@ conduit_status conduit_refresh_attn(const conduit_kv* kv, const conduit_batch* b
   (void)workspace;
   (void)workspace_bytes;
   (void)status;
-  cudaError_t err = launch_refresh_simt(make_kv(kv, batch), make_batch(batch), idx, idx_off_dev,
-                                        n_sel, q_rows, out, static_cast<cudaStream_t>(stream));
+  const KvDev kd = make_kv(kv, batch);
+  cudaError_t err =
+      refresh_tc_supported(kd)
+          ? launch_refresh_tc(kd, make_batch(batch), idx, idx_off_dev, idx_off, n_sel, q_rows, out,
+                              status, static_cast<cudaStream_t>(stream))
+          : launch_refresh_simt(kd, make_batch(batch), idx, idx_off_dev, n_sel, q_rows, out,
+                                static_cast<cudaStream_t>(stream));
   if (err) return cuda_fail(err, "refresh_attn");
   return CONDUIT_OK;
 }

@@ -82,6 +82,13 @@ cudaError_t launch_value_sumsq(const KvDev& kv, const BatchDev& b, const LayerLi
 cudaError_t launch_score_simt(const KvDev& kv, const BatchDev& b, const void* q, int32_t q_tot,
                               const LayerList& layers, int max_rows, int max_tokens,
                               float2* stats, float* pa, cudaStream_t stream);
+// Tensor-core scoring (bf16, head_dim 128): rows statistics then column sums.
+bool score_tc_supported(const KvDev& kv);
+int score_tc_chunk(int R, const int32_t* tok_off_host, int n_layers, int Hkv);
+size_t score_tc_part_bytes(int chunk, int max_tokens, int64_t total_rows);
+cudaError_t launch_score_tc(const KvDev& kv, const BatchDev& b, const void* q, int32_t q_tot,
+                            const LayerList& layers, int max_tokens, int chunk, float2* part,
+                            float* pa, int32_t* status, cudaStream_t stream);
 cudaError_t launch_finalize(const float* pa, const float* ss, const BatchDev& b, int n_layers,
                             int Hkv, int Hq, int64_t n_tot, float* s, float* attn_sum,
                             float* g, int32_t* status, cudaStream_t stream);
@@ -97,6 +104,10 @@ cudaError_t launch_select_noalloc(const BatchDev& b, const float* s, const float
 cudaError_t launch_kv_copy(const KvDev& kv, const BatchDev& b, const int32_t* idx,
                            const int32_t* idx_off_dev, int32_t n_sel, int max_sel, bool scatter,
                            void* k_rows, void* v_rows, cudaStream_t stream);
+bool refresh_tc_supported(const KvDev& kv);
+cudaError_t launch_refresh_tc(const KvDev& kv, const BatchDev& b, const int32_t* idx,
+                              const int32_t* idx_off_dev, const int32_t* idx_off_host, int32_t n_sel,
+                              const void* q_rows, void* out, int32_t* status, cudaStream_t stream);
 cudaError_t launch_refresh_simt(const KvDev& kv, const BatchDev& b, const int32_t* idx,
                                 const int32_t* idx_off_dev, int32_t n_sel, const void* q_rows,
                                 void* out, cudaStream_t stream);

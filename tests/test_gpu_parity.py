@@ -295,6 +295,30 @@ def test_index_driven_refresh_with_oracle_indices(C, P):
     _patched_equals_scatter(C, pipe, inputs)
 
 
+def test_refresh_late_max_jump_in_some_heads(C, P):
+    """Rows whose running max jumps far (> 2^8) at a late key tile while other
+    rows of the same warp do not: the lazy O rescale must stay correct."""
+    inputs = _small_multi(num_layers=1, tokens_per_image=128)   # N = 512, G = 7
+    d = inputs["k"].shape[-1]
+    u = torch.nn.functional.normalize(torch.randn(d, device="cuda"), dim=0)
+    k = inputs["k"].clone()
+    k[0, :, 400, :] = (45.0 * u).to(k.dtype)                    # planted key, not refreshed
+    base = {**inputs, "k": k, "v": inputs["v"].clone()}
+    sel = list(range(401, 481))
+    pipe = P.from_inputs(base, budgets=[len(sel)])
+    q_rows = pipe.q_rows.clone()
+    q_rows[:, :, 0::2, :] = (8.0 * u).to(q_rows.dtype)          # even heads aim at the planted key
+    pipe.q_rows.copy_(q_rows)
+    pipe.idx[:len(sel)] = torch.tensor(sel, dtype=torch.int32, device="cuda")
+    pipe.refresh()
+    torch.cuda.synchronize()
+    assert C.conduit_read_status(pipe.status) == C.OK
+    kp = O.kv_scatter(k[:, :, :512].double().cpu().numpy(), sel, pipe.k_rows.double().cpu().numpy())
+    vp = O.kv_scatter(inputs["v"][:, :, :512].double().cpu().numpy(), sel, pipe.v_rows.double().cpu().numpy())
+    want = O.refresh_attention(pipe.q_rows.double().cpu().numpy(), kp, vp, sel)
+    np.testing.assert_allclose(pipe.out.double().cpu().numpy(), want, rtol=2.0 ** -8, atol=2e-2)
+
+
 def test_nonfinite_input_sets_status_word(C, P):
     inputs = _small_multi()
     inputs["v"][0, 0, 7, 3] = float("nan")
