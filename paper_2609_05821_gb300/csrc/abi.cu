@@ -144,9 +144,9 @@ conduit_status make_layers(const conduit_kv* kv, const int32_t* layers, int32_t 
 }
 
 struct ScoreLayout {
-  bool tc;     // tensor-core kernels (bf16, head_dim 128) or the CUDA-core ones
-  int chunk;   // tokens per tensor-core work unit
-  int max_tok;
+  bool tc;     // tensor-core kernel (bf16, head_dim 128) or the CUDA-core ones
+  int rg_max;  // row groups per slab (column-sum partials per KV head)
+  int group_rows;
   size_t stats, pa, ss, attn, total;
 };
 
@@ -156,18 +156,19 @@ ScoreLayout score_layout(const conduit_kv* kv, const conduit_batch* b, int n_lay
   const size_t q_tot = size_t(b->q_off[R]);
   ScoreLayout s{};
   s.tc = score_tc_supported(make_kv(kv, b));
-  for (int r = 0; r < R; ++r) s.max_tok = std::max(s.max_tok, b->tok_off[r + 1] - b->tok_off[r]);
+  s.rg_max = 1;
+  if (s.tc) {
+    s.group_rows = kScoreGroupRows;
+    const int G = kv->num_q_heads / kv->num_kv_heads;
+    for (int r = 0; r < R; ++r)
+      s.rg_max = std::max(s.rg_max, score_tc_groups(G * (b->q_off[r + 1] - b->q_off[r])));
+  }
   const int64_t total_rows = int64_t(n_layers) * kv->num_q_heads * int64_t(q_tot);
   size_t off = 0;
   s.stats = off;
-  if (s.tc) {  // partial (max, sum) per row and token chunk
-    s.chunk = score_tc_chunk(R, b->tok_off, n_layers, kv->num_kv_heads);
-    off += align_up(score_tc_part_bytes(s.chunk, s.max_tok, total_rows));
-  } else {     // final (max, sum) per row
-    off += align_up(size_t(total_rows) * sizeof(float2));
-  }
+  if (!s.tc) off += align_up(size_t(total_rows) * sizeof(float2));  // (max, sum) per row
   s.pa = off;
-  off += align_up(size_t(n_layers) * kv->num_kv_heads * n_tot * sizeof(float));
+  off += align_up(size_t(n_layers) * kv->num_kv_heads * s.rg_max * n_tot * sizeof(float));
   s.ss = off;
   off += align_up(size_t(n_layers) * n_tot * sizeof(float));
   s.attn = off;
@@ -270,11 +271,12 @@ conduit_status conduit_score(const conduit_kv* kv, const conduit_batch* batch, c
   cudaError_t err;
   if ((err = launch_value_sumsq(kd, bd, ll, max_tok, ss, cs))) return cuda_fail(err, "value_sumsq");
   if (lay.tc)
-    err = launch_score_tc(kd, bd, q, batch->q_off[R], ll, max_tok, lay.chunk, stats, pa, status, cs);
+    err = launch_score_tc(kd, bd, batch->q_off, q, batch->q_off[R], ll, lay.rg_max, pa, status, cs);
   else
     err = launch_score_simt(kd, bd, q, batch->q_off[R], ll, max_rows, max_tok, stats, pa, cs);
   if (err) return cuda_fail(err, "score");
-  if ((err = launch_finalize(pa, ss, bd, ll.n, kd.Hkv, kd.Hq, kd.n_tot, s, attn, g, status, cs)))
+  if ((err = launch_finalize(pa, ss, bd, ll.n, kd.Hkv, kd.Hq, lay.rg_max, lay.group_rows, kd.n_tot,
+                             s, attn, g, status, cs)))
     return cuda_fail(err, "finalize");
   return CONDUIT_OK;
 }

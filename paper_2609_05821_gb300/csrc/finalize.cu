@@ -1,36 +1,60 @@
 // Per-token and per-image reductions of the scoring pass (Conduit Eqs. 6-8).
-//   a_t^(l)  = sum_g pa[l][g][t] / (|Q| Hq)            Eq. 6 (head/query mean)
-//   v_t^(l)  = sqrt(ss[l][t])                           concatenated-head norm
-//   s_t      = (1/|L|) sum_l a_t^(l) v_t^(l)            Eq. 7
+//   a_t^(l)  = sum_g sum_group pa[l][g][group][t] / (|Q| Hq)   Eq. 6 (head/query mean)
+//   v_t^(l)  = sqrt(ss[l][t])                                  concatenated-head norm
+//   s_t      = (1/|L|) sum_l a_t^(l) v_t^(l)                   Eq. 7
 //   A_t      = sum_l a_t^(l)
-//   g_j      = (1/(|L| n_j)) sum_{t in V_j} A_t         Eq. 8
-// Sums run in a fixed order (deterministic).
+//   g_j      = (1/(|L| n_j)) sum_{t in V_j} A_t                Eq. 8
+// A block covers 32 tokens; its 8 warps take every 8th layer (coalesced
+// loads across the 32 tokens of a warp) and combine in a fixed order, so the
+// sums are deterministic.
 #include "internal.cuh"
 
 namespace conduit {
 namespace {
 
+constexpr int kLayerGroups = 8;
+
 __global__ void __launch_bounds__(256) finalize_tokens_kernel(const float* pa, const float* ss,
                                                               BatchDev b, int n_layers, int Hkv,
-                                                              int Hq, int64_t n_tot, float* s,
+                                                              int Hq, int rg_max, int group_rows,
+                                                              int64_t n_tot, float* s,
                                                               float* attn_sum, int32_t* status) {
-  const int64_t tg = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
-  if (tg >= n_tot) return;
-  const int r = request_of(b.tok_off, b.R, tg);
-  const float denom = float((b.q_off[r + 1] - b.q_off[r]) * Hq);
+  __shared__ float part_s[kLayerGroups][32];
+  __shared__ float part_a[kLayerGroups][32];
+  const int lane = threadIdx.x & 31, lg = threadIdx.x >> 5;
+  const int64_t tg = int64_t(blockIdx.x) * 32 + lane;
   float acc_s = 0.f, acc_a = 0.f;
-  for (int li = 0; li < n_layers; ++li) {
-    float col = 0.f;
-    for (int g = 0; g < Hkv; ++g) col += pa[(int64_t(li) * Hkv + g) * n_tot + tg];
-    const float a = col / denom;
-    const float vn = sqrtf(ss[int64_t(li) * n_tot + tg]);
-    acc_s = fmaf(a, vn, acc_s);
-    acc_a += a;
+  if (tg < n_tot) {
+    const int r = request_of(b.tok_off, b.R, tg);
+    const int nq = b.q_off[r + 1] - b.q_off[r];
+    const float denom = float(nq * Hq);
+    const int rows = (Hq / Hkv) * nq;
+    const int n_rg = group_rows ? (rows + group_rows - 1) / group_rows : 1;
+    for (int li = lg; li < n_layers; li += kLayerGroups) {
+      float col = 0.f;
+      for (int g = 0; g < Hkv; ++g)
+        for (int rg = 0; rg < n_rg; ++rg) col += pa[((int64_t(li) * Hkv + g) * rg_max + rg) * n_tot + tg];
+      const float a = col / denom;
+      const float vn = sqrtf(ss[int64_t(li) * n_tot + tg]);
+      acc_s = fmaf(a, vn, acc_s);
+      acc_a += a;
+    }
   }
-  const float sv = acc_s / float(n_layers);
-  if (!isfinite(sv) || !isfinite(acc_a)) flag_status(status, CONDUIT_FLAG_NONFINITE);
-  s[tg] = sv;
-  attn_sum[tg] = acc_a;
+  part_s[lg][lane] = acc_s;
+  part_a[lg][lane] = acc_a;
+  __syncthreads();
+  if (lg == 0 && tg < n_tot) {
+    float ts = 0.f, ta = 0.f;
+#pragma unroll
+    for (int w = 0; w < kLayerGroups; ++w) {
+      ts += part_s[w][lane];
+      ta += part_a[w][lane];
+    }
+    const float sv = ts / float(n_layers);
+    if (!isfinite(sv) || !isfinite(ta)) flag_status(status, CONDUIT_FLAG_NONFINITE);
+    s[tg] = sv;
+    attn_sum[tg] = ta;
+  }
 }
 
 // One CTA per image: g_j by a fixed-order tree reduction of A over its span.
@@ -55,11 +79,11 @@ __global__ void __launch_bounds__(256) image_means_kernel(const float* attn_sum,
 }  // namespace
 
 cudaError_t launch_finalize(const float* pa, const float* ss, const BatchDev& b, int n_layers,
-                            int Hkv, int Hq, int64_t n_tot, float* s, float* attn_sum, float* g,
-                            int32_t* status, cudaStream_t stream) {
+                            int Hkv, int Hq, int rg_max, int group_rows, int64_t n_tot, float* s,
+                            float* attn_sum, float* g, int32_t* status, cudaStream_t stream) {
   if (n_tot == 0) return cudaSuccess;
-  finalize_tokens_kernel<<<unsigned((n_tot + 255) / 256), 256, 0, stream>>>(
-      pa, ss, b, n_layers, Hkv, Hq, n_tot, s, attn_sum, status);
+  finalize_tokens_kernel<<<unsigned((n_tot + 31) / 32), 256, 0, stream>>>(
+      pa, ss, b, n_layers, Hkv, Hq, rg_max, group_rows, n_tot, s, attn_sum, status);
   cudaError_t err = cudaGetLastError();
   if (err) return err;
   image_means_kernel<<<b.K, 256, 0, stream>>>(attn_sum, b, n_layers, g);

@@ -1,25 +1,29 @@
 // Tensor-core scoring pass for bf16 caches with head_dim 128 (Conduit Eq. 6).
 //
-// Per slab (request r, scored layer l, KV head g) the logits are
-// S = Q_g K_g^T over R = G*|Q| scoring rows and the request's N_r keys. Two
-// persistent kernels share one work list of units (slab, token chunk):
+// One persistent, warp-specialised kernel. A work unit is one slab (request
+// r, scored layer l, KV head g) restricted to a group of at most 256 scoring
+// rows (rows = the G query heads of group g times the |Q| span queries).
+// Each unit makes two passes over the request's N_r keys:
 //
-//   rowstats_tc  D[rows x 128 tokens] = Q_rows . K_tile^T on tcgen05 (rows are
-//                the MMA M dimension, so each thread owns one row): running
-//                row max and sum of 2^((S - m) log2(e)/sqrt(d)) over the
-//                chunk -> partial (m, Z) per row and chunk.
-//   colsum_tc    D[128 tokens x rows] = K_tile . Q_rows^T (tokens are M, so
-//                each thread owns one token): merges the chunk statistics
-//                into log2-sum-exp per row, then sums 2^(x - lse) over the
-//                rows -> pa[l][g][t], the group's share of Eq. 6.
+//   pass A   D[rows x 128 tokens] = Q_rows . K_tile^T     (rows are the MMA M)
+//            each epilogue thread owns one row: running max m and sum
+//            z = sum 2^((S - m) log2(e)/sqrt(d)) -> lse = m log2(e)/sqrt(d) + log2 z
+//   pass B   D[128 tokens x rows] = K_tile . Q_rows^T     (tokens are the MMA M)
+//            each epilogue thread owns one token: sum over rows of 2^(x - lse)
+//            -> pa[l][g][group][t], this group's share of sum_q sum_h alpha
 //
-// K tiles (128 tokens x 128 dims) arrive by TMA with 128-byte swizzle into a
-// two-stage ring; scoring rows are staged once per unit by the threads in
-// the same swizzled layout. One thread issues the TMA loads and the MMAs;
-// accumulators live in TMEM (512 columns, double-buffered when a tile needs
-// at most 256) and are read back with tcgen05.ld. Every wait is bounded; on
-// timeout the kernel sets CONDUIT_FLAG_TIMEOUT, drains its copies and frees
-// its TMEM.
+// Pass B walks the tiles in reverse so the most recent K tiles of pass A are
+// still in L2. Roles (192 threads):
+//   warp 0       one thread issues TMA loads of K tiles (128 tokens x 128
+//                dims, 128-byte swizzle) into a four-stage ring
+//   warp 1       one thread issues tcgen05 MMAs into two 256-column TMEM
+//                accumulator slots (it also owns the TMEM allocation)
+//   warps 2-5    epilogue: stage the unit's scoring rows in shared memory
+//                (same swizzle), then read accumulators with tcgen05.ld
+// The roles meet on mbarriers (ring full / empty, accumulator full / empty,
+// rows ready). Every wait is bounded by one second; a role that gives up
+// raises an abort flag the others also watch, the kernel sets
+// CONDUIT_FLAG_TIMEOUT, drains its copies and MMAs, and frees TMEM.
 #include <cuda.h>
 
 #include "internal.cuh"
@@ -30,106 +34,136 @@ namespace {
 
 constexpr int kD = 128;
 constexpr int kTile = 128;
-constexpr int kStages = 2;
-constexpr int kRowGroup = 512;
-constexpr int kThreads = 128;
-constexpr uint32_t kHalfQ = kRowGroup * 128;        // bytes of one 64-dim half of the row tile
-constexpr uint32_t kQBytes = 2 * kHalfQ;            // 128 KB
-constexpr uint32_t kHalfK = kTile * 128;            // 16 KB
-constexpr uint32_t kStageBytes = 2 * kHalfK;        // 32 KB per K tile
-constexpr uint32_t kSmemBytes = 1024 + kQBytes + kStages * kStageBytes + 256 + kRowGroup * 4;
+constexpr int kStages = 4;
+constexpr int kGroupRows = 256;
+constexpr int kThreads = 192;
+constexpr int kEpiThreads = 128;
+constexpr uint32_t kHalfQ = kGroupRows * 128;  // 32 KB: one 64-dim half of the row tile
+constexpr uint32_t kHalfK = kTile * 128;       // 16 KB
+constexpr uint32_t kStageBytes = 2 * kHalfK;   // 32 KB per K tile
+constexpr uint32_t kSlotCols = 256;
+constexpr uint32_t kSmemBytes = 1024 + 2 * kHalfQ + kStages * kStageBytes + 256 + kGroupRows * 4;
 
 struct TcArgs {
   KvDev kv;
   BatchDev b;
   const __nv_bfloat16* q;
   int32_t q_tot;
-  int32_t chunk;        // tokens per unit (multiple of 128)
-  int32_t nchunks_max;  // chunks per slab for the longest request
   int32_t n_units;
-  int64_t total_rows;   // n_layers * Hq * Q_tot
-  float scale_log2;     // log2(e) / sqrt(d)
-  float2* part;         // [nchunks_max][total_rows] partial (max S, sum) per row
-  float* pa;            // [n_layers][Hkv][n_tot]
+  int32_t rg_max;      // row groups per slab, maximum over requests (pa stride)
+  float scale_log2;    // log2(e) / sqrt(d)
+  float* pa;           // [n_layers][Hkv][rg_max][n_tot]
   int32_t* status;
   LayerList layers;
 };
 
 struct Unit {
-  int r, li, l, g, c, t0, N, q0, nq, R, tok0, tiles;
+  int r, li, l, g, rg, t0, N, q0, nq, row0, rows, tiles;
 };
 
+// Row groups of a slab with R scoring rows: ceil(R / 256) groups of equal
+// size rounded up to 16 (the last one takes the rest).
+__host__ __device__ __forceinline__ int n_groups(int R) { return (R + kGroupRows - 1) / kGroupRows; }
+__host__ __device__ __forceinline__ int group_rows(int R) {
+  const int ng = n_groups(R);
+  return ng == 0 ? 0 : (((R + ng - 1) / ng) + 15) & ~15;
+}
+
 __device__ __forceinline__ bool decode_unit(const TcArgs& a, int u, Unit& w) {
-  const int per_slab = a.nchunks_max;
-  int slab = u / per_slab;
-  w.c = u % per_slab;
-  const int Hkv = a.kv.Hkv, nl = a.layers.n;
-  w.g = slab % Hkv;
-  slab /= Hkv;
-  w.li = slab % nl;
-  w.r = slab / nl;
-  w.l = a.layers.ids[w.li];
-  w.t0 = a.b.tok_off[w.r];
-  w.N = a.b.tok_off[w.r + 1] - w.t0;
-  w.q0 = a.b.q_off[w.r];
-  w.nq = a.b.q_off[w.r + 1] - w.q0;
-  w.R = a.kv.G * w.nq;
-  w.tok0 = w.c * a.chunk;
-  if (w.tok0 >= w.N || w.R == 0) return false;
-  w.tiles = (min(a.chunk, w.N - w.tok0) + kTile - 1) / kTile;
-  return true;
+  const int Hkv = a.kv.Hkv, nl = a.layers.n, G = a.kv.G;
+  int base = 0;
+  for (int r = 0; r < a.b.R; ++r) {
+    const int nq = a.b.q_off[r + 1] - a.b.q_off[r];
+    const int R = G * nq;
+    const int ng = n_groups(R);
+    const int cnt = nl * Hkv * ng;
+    if (u < base + cnt) {
+      int local = u - base;
+      w.r = r;
+      w.rg = local % ng;
+      local /= ng;
+      w.g = local % Hkv;
+      w.li = local / Hkv;
+      w.l = a.layers.ids[w.li];
+      w.t0 = a.b.tok_off[r];
+      w.N = a.b.tok_off[r + 1] - w.t0;
+      w.q0 = a.b.q_off[r];
+      w.nq = nq;
+      const int gr = group_rows(R);
+      w.row0 = w.rg * gr;
+      w.rows = min(gr, R - w.row0);
+      w.tiles = (w.N + kTile - 1) / kTile;
+      return w.rows > 0;
+    }
+    base += cnt;
+  }
+  return false;
+}
+
+// Tile index of the i-th K tile of the unit's two passes (pass B in reverse).
+__device__ __forceinline__ int tile_of(const Unit& w, int i) {
+  return i < w.tiles ? i : 2 * w.tiles - 1 - i;
 }
 
 struct Smem {
-  uint8_t* q;        // [2 halves][kRowGroup rows][128 B], 128-byte swizzle
-  uint8_t* k;        // [kStages][2 halves][128 rows][128 B]
-  uint64_t* full;    // [kStages]
-  uint64_t* mma;     // [2]
+  uint8_t* q;          // [2 halves][256 rows][128 B]
+  uint8_t* k;          // [kStages][2 halves][128 rows][128 B]
+  uint64_t* kfull;     // [kStages]
+  uint64_t* kempty;    // [kStages]
+  uint64_t* tfull;     // [2]
+  uint64_t* tempty;    // [2]
+  uint64_t* qready;    // [1]
+  uint64_t* mdone;     // [1]
   uint32_t* tmem_slot;
-  float* lse;        // [kRowGroup]
-  int32_t* pages;    // page ids of the current tile (paged caches)
+  volatile int* abort;
+  uint32_t* counters;  // [0] loads issued, [1] loads consumed
+  float* lse;          // [256]
 };
 
 __device__ __forceinline__ Smem carve(uint8_t* raw) {
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(raw) + 1023) & ~uintptr_t(1023));
   Smem s;
   s.q = base;
-  s.k = base + kQBytes;
+  s.k = base + 2 * kHalfQ;
   uint8_t* tail = s.k + kStages * kStageBytes;
-  s.full = reinterpret_cast<uint64_t*>(tail);
-  s.mma = s.full + kStages;
-  s.tmem_slot = reinterpret_cast<uint32_t*>(s.mma + 2);
-  s.pages = reinterpret_cast<int32_t*>(tail + 64);
+  s.kfull = reinterpret_cast<uint64_t*>(tail);
+  s.kempty = s.kfull + kStages;
+  s.tfull = s.kempty + kStages;
+  s.tempty = s.tfull + 2;
+  s.qready = s.tempty + 2;
+  s.mdone = s.qready + 1;
+  s.tmem_slot = reinterpret_cast<uint32_t*>(s.mdone + 1);
+  s.abort = reinterpret_cast<volatile int*>(s.tmem_slot + 1);
+  s.counters = reinterpret_cast<uint32_t*>(s.tmem_slot + 2);
   s.lse = reinterpret_cast<float*>(tail + 256);
   return s;
 }
 
-// Stage scoring rows [row0, row0 + nrows) of the unit's slab into the swizzled
-// row tile; rows at or beyond R are zero.
-__device__ __forceinline__ void stage_rows(const TcArgs& a, const Unit& w, uint8_t* q_s, int row0,
-                                           int nrows) {
-  const int Hq = a.kv.Hq, G = a.kv.G;
-  for (int idx = threadIdx.x; idx < nrows * 16; idx += blockDim.x) {
-    const int row = idx >> 4, ch = idx & 15;
-    const int j = row0 + row;
-    uint4 val = make_uint4(0u, 0u, 0u, 0u);
-    if (j < w.R) {
-      const int h = w.g * G + j / w.nq, qi = j % w.nq;
-      const __nv_bfloat16* src = a.q + ((int64_t(w.l) * Hq + h) * a.q_tot + w.q0 + qi) * kD + ch * 8;
-      val = *reinterpret_cast<const uint4*>(src);
-    }
-    uint8_t* dst = q_s + (ch >> 3) * kHalfQ + tc::sw128_offset(row, ch & 7);
-    *reinterpret_cast<uint4*>(dst) = val;
+// Bounded wait that also gives up when another role has aborted.
+__device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int* abort) {
+  if (tc::mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = tc::globaltimer_ns();
+  for (uint32_t i = 1; i < tc::kSpinLimit; ++i) {
+    if (tc::mbar_try_wait(bar, parity)) return true;
+    if ((i & 63u) == 0 && (*abort || tc::globaltimer_ns() - t0 > tc::kWaitNs)) return false;
   }
+  return false;
 }
 
-// Issue the TMA loads of K tile `tile` of the unit into ring stage `stage`.
+__device__ __forceinline__ void raise_abort(const TcArgs& a, const Smem& s, int32_t site) {
+  *s.abort = 1;
+  flag_status(a.status, CONDUIT_FLAG_TIMEOUT | site);
+}
+
+__device__ __forceinline__ void epi_barrier() {
+  asm volatile("bar.sync 1, %0;" ::"n"(kEpiThreads) : "memory");
+}
+
+// Issue the TMA loads of K tile `tile` of unit w into ring stage `stage`.
 __device__ __forceinline__ void load_k_tile(const TcArgs& a, const CUtensorMap* kmap, const Unit& w,
-                                            const Smem& s, int tile, int stage) {
-  uint8_t* dst = s.k + stage * kStageBytes;
-  uint64_t* bar = &s.full[stage];
+                                            uint8_t* dst, uint64_t* bar, int tile) {
   tc::mbar_arrive_expect_tx(bar, kStageBytes);
-  const int tok = w.tok0 + tile * kTile;
+  const int tok = tile * kTile;
   const KvDev& kv = a.kv;
   if (kv.page_size == 0) {
     const int32_t y = int32_t((int64_t(w.l) * kv.Hkv + w.g) * kv.n_tot + w.t0 + tok);
@@ -148,285 +182,244 @@ __device__ __forceinline__ void load_k_tile(const TcArgs& a, const CUtensorMap* 
   }
 }
 
-// Row statistics: one unit = (slab, chunk); rows as M.
+// Epilogue threads stage scoring rows [row0, row0 + nrows) of the unit into
+// the swizzled row tile (rows at or beyond the group are zero); eight
+// 16-byte loads per thread are in flight at a time.
+__device__ __forceinline__ void stage_rows(const TcArgs& a, const Unit& w, uint8_t* q_s, int nrows,
+                                           int et) {
+  const int G = a.kv.G, Hq = a.kv.Hq;
+  const int total = nrows * 16;
+  for (int base = 0; base < total; base += kEpiThreads * 8) {
+    uint4 val[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int idx = base + u * kEpiThreads + et;
+      val[u] = make_uint4(0u, 0u, 0u, 0u);
+      if (idx < total) {
+        const int row = idx >> 4, ch = idx & 15;
+        if (row < w.rows) {
+          const int j = w.row0 + row;
+          const int h = w.g * G + j / w.nq, qi = j % w.nq;
+          val[u] = *reinterpret_cast<const uint4*>(
+              a.q + ((int64_t(w.l) * Hq + h) * a.q_tot + w.q0 + qi) * kD + ch * 8);
+        }
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int idx = base + u * kEpiThreads + et;
+      if (idx < total) {
+        const int row = idx >> 4, ch = idx & 15;
+        *reinterpret_cast<uint4*>(q_s + (ch >> 3) * kHalfQ + tc::sw128_offset(row, ch & 7)) = val[u];
+      }
+    }
+  }
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
-    rowstats_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ TcArgs a) {
+    score_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ TcArgs a) {
   extern __shared__ uint8_t smem_raw[];
   const Smem s = carve(smem_raw);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   if (tid == 0) {
-    for (int i = 0; i < kStages; ++i) tc::mbar_init(&s.full[i], 1);
-    tc::mbar_init(&s.mma[0], 1);
-    tc::mbar_init(&s.mma[1], 1);
+    for (int i = 0; i < kStages; ++i) {
+      tc::mbar_init(&s.kfull[i], 1);
+      tc::mbar_init(&s.kempty[i], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      tc::mbar_init(&s.tfull[i], 1);
+      tc::mbar_init(&s.tempty[i], kEpiThreads);
+    }
+    tc::mbar_init(s.qready, 1);
+    tc::mbar_init(s.mdone, 1);
+    *s.abort = 0;
+    s.counters[0] = s.counters[1] = 0;
     tc::fence_barrier_init();
     tc::prefetch_tensormap(&kmap);
   }
-  if (warp == 0) tc::tmem_alloc(s.tmem_slot, 512);
+  if (warp == 1) tc::tmem_alloc(s.tmem_slot, 2 * kSlotCols);
   __syncthreads();
   tc::tc_fence_after();
   const uint32_t tmem = *s.tmem_slot;
-  const uint32_t lane_base = uint32_t(warp * 32) << 16;
 
-  uint32_t ld_seq = 0;          // K tiles issued so far (thread 0's view == everyone's)
-  uint32_t mma_phase[2] = {0u, 0u};
-  bool ok = true;
-  uint32_t pending_lo = 0, pending_hi = 0;  // tiles issued but not yet consumed (for draining)
-
-  for (int u = blockIdx.x; u < a.n_units && ok; u += gridDim.x) {
-    Unit w;
-    if (!decode_unit(a, u, w)) continue;
-    for (int rg0 = 0; rg0 < w.R && ok; rg0 += kRowGroup) {
-      const int rows = min(kRowGroup, w.R - rg0);
-      const int nrb = (rows + 127) / 128;
-      const int nbuf = nrb <= 2 ? 2 : 1;
-      __syncthreads();
-      stage_rows(a, w, s.q, rg0, nrb * 128);
-      tc::fence_proxy_async_smem();
-      __syncthreads();
-      const uint32_t base = ld_seq;
-      const int T = w.tiles;
-      if (tid == 0) {
-        for (int t = 0; t < min(kStages, T); ++t) load_k_tile(a, &kmap, w, s, t, (base + t) % kStages);
-      }
-      ld_seq += min(kStages, T);
-      pending_lo = base;
-      pending_hi = ld_seq;
-
-      auto issue_mma = [&](int t, int buf) {
-        const uint32_t seq = base + t;
+  if (warp == 0 && lane == 0) {
+    // ------------------------------------------------------------ producer
+    uint32_t seq = 0;
+    bool ok = true;
+    for (int u = blockIdx.x; u < a.n_units && ok; u += gridDim.x) {
+      Unit w;
+      if (!decode_unit(a, u, w)) continue;
+      for (int i = 0; i < 2 * w.tiles; ++i, ++seq) {
         const int st = seq % kStages;
-        if (!tc::mbar_wait(&s.full[st], (seq / kStages) & 1)) return false;
+        if (!wait_or_abort(&s.kempty[st], ((seq / kStages) & 1) ^ 1, s.abort)) {
+          if (!*s.abort) raise_abort(a, s, tc::kSiteLoad);
+          ok = false;
+          break;
+        }
+        load_k_tile(a, &kmap, w, s.k + st * kStageBytes, &s.kfull[st], tile_of(w, i));
+      }
+    }
+    s.counters[0] = seq;
+  } else if (warp == 1 && lane == 0) {
+    // ----------------------------------------------------------------- MMA
+    uint32_t kseq = 0, tseq = 0, useq = 0;
+    bool ok = true;
+    const uint32_t qb = tc::smem_u32(s.q);
+    for (int u = blockIdx.x; u < a.n_units && ok; u += gridDim.x) {
+      Unit w;
+      if (!decode_unit(a, u, w)) continue;
+      if (!wait_or_abort(s.qready, useq & 1, s.abort)) {
+        if (!*s.abort) raise_abort(a, s, tc::kSiteMma);
+        break;
+      }
+      ++useq;
+      tc::tc_fence_after();
+      const int nrb = (w.rows + 127) / 128;
+      const int ncols = (w.rows + 15) & ~15;
+      for (int i = 0; i < 2 * w.tiles; ++i) {
+        const int st = kseq % kStages;
+        if (!wait_or_abort(&s.kfull[st], (kseq / kStages) & 1, s.abort)) {
+          if (!*s.abort) raise_abort(a, s, tc::kSiteLoad);
+          ok = false;
+          break;
+        }
+        ++kseq;
+        const int slot = tseq & 1;
+        if (!wait_or_abort(&s.tempty[slot], ((tseq >> 1) & 1) ^ 1, s.abort)) {
+          if (!*s.abort) raise_abort(a, s, tc::kSiteMma);
+          ok = false;
+          break;
+        }
+        ++tseq;
         tc::tc_fence_after();
         const uint32_t kb = tc::smem_u32(s.k + st * kStageBytes);
-        const uint32_t qb = tc::smem_u32(s.q);
-        const uint32_t idesc = tc::idesc_bf16(128, kTile);
-        for (int rb = 0; rb < nrb; ++rb) {
-          const uint32_t d = tmem + uint32_t(buf * nrb * 128 + rb * 128);
+        const uint32_t d = tmem + uint32_t(slot) * kSlotCols;
+        if (i < w.tiles) {  // pass A: rows x tokens
+          const uint32_t idesc = tc::idesc_bf16(128, kTile);
+          for (int rb = 0; rb < nrb; ++rb) {
+#pragma unroll
+            for (int kk = 0; kk < 8; ++kk) {
+              const uint32_t off = (kk >> 2) * 0 + (kk & 3) * 32;
+              tc::mma_bf16(d + rb * 128, tc::desc_sw128(qb + (kk >> 2) * kHalfQ + rb * 128 * 128 + off),
+                           tc::desc_sw128(kb + (kk >> 2) * kHalfK + off), idesc, kk > 0);
+            }
+          }
+        } else {            // pass B: tokens x rows
+          const uint32_t idesc = tc::idesc_bf16(128, ncols);
 #pragma unroll
           for (int kk = 0; kk < 8; ++kk) {
-            const uint32_t off = (kk >> 2) * 0 + (kk & 3) * 32;
-            const uint64_t adesc = tc::desc_sw128(qb + (kk >> 2) * kHalfQ + rb * 128 * 128 + off);
-            const uint64_t bdesc = tc::desc_sw128(kb + (kk >> 2) * kHalfK + off);
-            tc::mma_bf16(d, adesc, bdesc, idesc, kk > 0);
+            const uint32_t off = (kk & 3) * 32;
+            tc::mma_bf16(d, tc::desc_sw128(kb + (kk >> 2) * kHalfK + off),
+                         tc::desc_sw128(qb + (kk >> 2) * kHalfQ + off), idesc, kk > 0);
           }
         }
-        tc::mma_commit(&s.mma[buf]);
-        return true;
-      };
-
-      int mma_ok = 1;
-      if (tid == 0) mma_ok = issue_mma(0, 0);
-      float m[4], z[4];
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        m[i] = -INFINITY;
-        z[i] = 0.f;
+        tc::mma_commit(&s.kempty[st]);
+        tc::mma_commit(&s.tfull[slot]);
       }
-      for (int t = 0; t < T; ++t) {
-        const int buf = nbuf == 2 ? (t & 1) : 0;
-        if (!__syncthreads_and(mma_ok)) { ok = false; break; }
-        if (!tc::mbar_wait(&s.mma[buf], mma_phase[buf])) ok = false;
-        mma_phase[buf] ^= 1u;
-        if (!__syncthreads_and(ok)) { ok = false; break; }
-        tc::tc_fence_after();
-        if (tid == 0) {
-          if (t + kStages < T) {
-            load_k_tile(a, &kmap, w, s, t + kStages, (base + t + kStages) % kStages);
-          }
-          if (nbuf == 2 && t + 1 < T) mma_ok = issue_mma(t + 1, buf ^ 1);
+    }
+    s.counters[1] = kseq;
+    tc::mma_commit(s.mdone);  // every MMA issued above has completed once this arrives
+    tc::mbar_wait(s.mdone, 0);
+  } else if (warp >= 2) {
+    // ------------------------------------------------------------ epilogue
+    // After an abort the epilogue keeps walking its units (skipping the work)
+    // so that every thread reaches every named barrier.
+    const int et = tid - 64;                       // 0..127
+    const int quarter = warp & 3;                  // TMEM lanes 32*quarter .. +31
+    const int lrow = quarter * 32 + lane;          // row (pass A) / token (pass B) in the tile
+    const uint32_t lane_base = uint32_t(quarter * 32) << 16;
+    uint32_t tseq = 0;
+    bool ok = true;
+    for (int u = blockIdx.x; u < a.n_units; u += gridDim.x) {
+      Unit w;
+      if (!decode_unit(a, u, w)) continue;
+      const int nrb = (w.rows + 127) / 128;
+      if (ok && !*s.abort) stage_rows(a, w, s.q, nrb * 128, et);
+      tc::fence_proxy_async_smem();
+      epi_barrier();
+      if (et == 0) tc::mbar_arrive(s.qready);
+      float m0 = -INFINITY, z0 = 0.f, m1 = -INFINITY, z1 = 0.f;
+      for (int i = 0; i < w.tiles; ++i) {            // pass A
+        const int slot = tseq & 1;
+        if (ok && !wait_or_abort(&s.tfull[slot], (tseq >> 1) & 1, s.abort)) {
+          if (!*s.abort) raise_abort(a, s, tc::kSiteMma);
+          ok = false;
         }
-        if (t + kStages < T) ++ld_seq;
-        pending_lo = base + t + 1;
-        pending_hi = ld_seq;
-        // epilogue: this thread's rows are rb*128 + warp*32 + lane
-        const int tok_base = w.tok0 + t * kTile;
+        ++tseq;
+        if (!ok) continue;
+        tc::tc_fence_after();
+        const int tok0 = i * kTile;
         for (int rb = 0; rb < nrb; ++rb) {
+          float mr = rb == 0 ? m0 : m1, zr = rb == 0 ? z0 : z1;
+#pragma unroll 1
           for (int cc = 0; cc < 4; ++cc) {
             float v[32];
-            tc::tmem_ld32(tmem + lane_base + uint32_t(buf * nrb * 128 + rb * 128 + cc * 32), v);
-            const int tok = tok_base + cc * 32;
+            tc::tmem_ld32(tmem + lane_base + uint32_t(slot) * kSlotCols + rb * 128 + cc * 32, v);
             float cmax = -INFINITY;
+            const int tok = tok0 + cc * 32;
 #pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              if (tok + i >= w.N) v[i] = -INFINITY;
-              cmax = fmaxf(cmax, v[i]);
+            for (int x = 0; x < 32; ++x) {
+              if (tok + x >= w.N) v[x] = -INFINITY;
+              cmax = fmaxf(cmax, v[x]);
             }
-            float mr = m[0], zr = z[0];
-            if (rb == 1) { mr = m[1]; zr = z[1]; }
-            if (rb == 2) { mr = m[2]; zr = z[2]; }
-            if (rb == 3) { mr = m[3]; zr = z[3]; }
             const float mn = fmaxf(mr, cmax);
             if (mn != -INFINITY) {
               const float nb = -mn * a.scale_log2;
               float acc = 0.f;
 #pragma unroll
-              for (int i = 0; i < 32; ++i) acc += exp2f(fmaf(v[i], a.scale_log2, nb));
+              for (int x = 0; x < 32; ++x) acc += exp2f(fmaf(v[x], a.scale_log2, nb));
               zr = zr * exp2f((mr - mn) * a.scale_log2) + acc;
               mr = mn;
             }
-            if (rb == 0) { m[0] = mr; z[0] = zr; }
-            if (rb == 1) { m[1] = mr; z[1] = zr; }
-            if (rb == 2) { m[2] = mr; z[2] = zr; }
-            if (rb == 3) { m[3] = mr; z[3] = zr; }
           }
+          if (rb == 0) { m0 = mr; z0 = zr; } else { m1 = mr; z1 = zr; }
         }
         tc::tc_fence_before();
-        __syncthreads();
-        if (tid == 0 && nbuf == 1 && t + 1 < T) mma_ok = issue_mma(t + 1, 0);
+        tc::mbar_arrive(&s.tempty[slot]);
       }
-      if (!ok) break;
-      const int64_t srow0 = (int64_t(w.li) * a.kv.Hkv + w.g) * a.kv.G * a.q_tot + int64_t(a.kv.G) * w.q0;
-      for (int rb = 0; rb < nrb; ++rb) {
-        const int j = rg0 + rb * 128 + warp * 32 + lane;
-        if (j < w.R) {
-          float mr = rb == 0 ? m[0] : rb == 1 ? m[1] : rb == 2 ? m[2] : m[3];
-          float zr = rb == 0 ? z[0] : rb == 1 ? z[1] : rb == 2 ? z[2] : z[3];
-          a.part[int64_t(w.c) * a.total_rows + srow0 + j] = make_float2(mr, zr);
+      // log2-sum-exp of this thread's rows, shared with the token-owning threads of pass B
+      if (lrow < w.rows) s.lse[lrow] = m0 * a.scale_log2 + log2f(z0);
+      if (nrb > 1 && 128 + lrow < w.rows) s.lse[128 + lrow] = m1 * a.scale_log2 + log2f(z1);
+      epi_barrier();
+      float* pa_out = a.pa + ((int64_t(w.li) * a.kv.Hkv + w.g) * a.rg_max + w.rg) * a.kv.n_tot + w.t0;
+      const int nchunk = (w.rows + 31) / 32;
+      for (int i = w.tiles; i < 2 * w.tiles; ++i) {  // pass B
+        const int slot = tseq & 1;
+        if (ok && !wait_or_abort(&s.tfull[slot], (tseq >> 1) & 1, s.abort)) {
+          if (!*s.abort) raise_abort(a, s, tc::kSiteMma);
+          ok = false;
         }
-      }
-    }
-  }
-  if (!ok) {
-    flag_status(a.status, CONDUIT_FLAG_TIMEOUT);
-    if (tid == 0) {  // drain TMA copies still in flight into this CTA's shared memory
-      for (uint32_t seq = pending_lo; seq < pending_hi; ++seq)
-        tc::mbar_wait(&s.full[seq % kStages], (seq / kStages) & 1);
-    }
-  }
-  tc::tc_fence_before();
-  __syncthreads();
-  if (warp == 0) tc::tmem_dealloc(tmem, 512);
-}
-
-// Column sums: one unit = (slab, chunk); tokens as M.
-__global__ void __launch_bounds__(kThreads, 1)
-    colsum_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ TcArgs a) {
-  extern __shared__ uint8_t smem_raw[];
-  const Smem s = carve(smem_raw);
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  if (tid == 0) {
-    for (int i = 0; i < kStages; ++i) tc::mbar_init(&s.full[i], 1);
-    tc::mbar_init(&s.mma[0], 1);
-    tc::mbar_init(&s.mma[1], 1);
-    tc::fence_barrier_init();
-    tc::prefetch_tensormap(&kmap);
-  }
-  if (warp == 0) tc::tmem_alloc(s.tmem_slot, 512);
-  __syncthreads();
-  tc::tc_fence_after();
-  const uint32_t tmem = *s.tmem_slot;
-  const uint32_t lane_base = uint32_t(warp * 32) << 16;
-
-  uint32_t ld_seq = 0;
-  uint32_t mma_phase[2] = {0u, 0u};
-  bool ok = true;
-  uint32_t pending_lo = 0, pending_hi = 0;
-
-  for (int u = blockIdx.x; u < a.n_units && ok; u += gridDim.x) {
-    Unit w;
-    if (!decode_unit(a, u, w)) continue;
-    const int nch = (w.N + a.chunk - 1) / a.chunk;
-    const int64_t srow0 = (int64_t(w.li) * a.kv.Hkv + w.g) * a.kv.G * a.q_tot + int64_t(a.kv.G) * w.q0;
-    float* pa_out = a.pa + (int64_t(w.li) * a.kv.Hkv + w.g) * a.kv.n_tot + w.t0;
-    for (int rg0 = 0; rg0 < w.R && ok; rg0 += kRowGroup) {
-      const int rows = min(kRowGroup, w.R - rg0);
-      const int ncols = (rows + 15) & ~15;
-      const int nbuf = ncols <= 256 ? 2 : 1;
-      __syncthreads();
-      // log2-sum-exp of each row from the chunk statistics of rowstats_tc
-      for (int j = tid; j < rows; j += blockDim.x) {
-        float M = -INFINITY;
-        for (int c = 0; c < nch; ++c) M = fmaxf(M, a.part[int64_t(c) * a.total_rows + srow0 + rg0 + j].x);
-        float Z = 0.f;
-        for (int c = 0; c < nch; ++c) {
-          const float2 st = a.part[int64_t(c) * a.total_rows + srow0 + rg0 + j];
-          Z += st.y * exp2f((st.x - M) * a.scale_log2);
-        }
-        s.lse[j] = M * a.scale_log2 + log2f(Z);
-      }
-      stage_rows(a, w, s.q, rg0, ncols);
-      tc::fence_proxy_async_smem();
-      __syncthreads();
-      const uint32_t base = ld_seq;
-      const int T = w.tiles;
-      if (tid == 0) {
-        for (int t = 0; t < min(kStages, T); ++t) load_k_tile(a, &kmap, w, s, t, (base + t) % kStages);
-      }
-      ld_seq += min(kStages, T);
-      pending_lo = base;
-      pending_hi = ld_seq;
-
-      auto issue_mma = [&](int t, int buf) {
-        const uint32_t seq = base + t;
-        const int st = seq % kStages;
-        if (!tc::mbar_wait(&s.full[st], (seq / kStages) & 1)) return false;
+        ++tseq;
+        if (!ok) continue;
         tc::tc_fence_after();
-        const uint32_t kb = tc::smem_u32(s.k + st * kStageBytes);
-        const uint32_t qb = tc::smem_u32(s.q);
-        for (int n0 = 0; n0 < ncols; n0 += 256) {
-          const int nn = min(256, ncols - n0);
-          const uint32_t idesc = tc::idesc_bf16(128, nn);
-          const uint32_t d = tmem + uint32_t(buf * 256 + n0);
-#pragma unroll
-          for (int kk = 0; kk < 8; ++kk) {
-            const uint32_t off = (kk & 3) * 32;
-            const uint64_t adesc = tc::desc_sw128(kb + (kk >> 2) * kHalfK + off);
-            const uint64_t bdesc = tc::desc_sw128(qb + (kk >> 2) * kHalfQ + n0 * 128 + off);
-            tc::mma_bf16(d, adesc, bdesc, idesc, kk > 0);
-          }
-        }
-        tc::mma_commit(&s.mma[buf]);
-        return true;
-      };
-
-      int mma_ok = 1;
-      if (tid == 0) mma_ok = issue_mma(0, 0);
-      for (int t = 0; t < T; ++t) {
-        const int buf = nbuf == 2 ? (t & 1) : 0;
-        if (!__syncthreads_and(mma_ok)) { ok = false; break; }
-        if (!tc::mbar_wait(&s.mma[buf], mma_phase[buf])) ok = false;
-        mma_phase[buf] ^= 1u;
-        if (!__syncthreads_and(ok)) { ok = false; break; }
-        tc::tc_fence_after();
-        if (tid == 0) {
-          if (t + kStages < T) load_k_tile(a, &kmap, w, s, t + kStages, (base + t + kStages) % kStages);
-          if (nbuf == 2 && t + 1 < T) mma_ok = issue_mma(t + 1, buf ^ 1);
-        }
-        if (t + kStages < T) ++ld_seq;
-        pending_lo = base + t + 1;
-        pending_hi = ld_seq;
-        // epilogue: this thread's token is warp*32 + lane of the tile
         float acc = 0.f;
-        const int nchunk32 = (rows + 31) / 32;
-        for (int cc = 0; cc < nchunk32; ++cc) {
+        for (int cc = 0; cc < nchunk; ++cc) {
           float v[32];
-          tc::tmem_ld32(tmem + lane_base + uint32_t(buf * 256 + cc * 32), v);
+          tc::tmem_ld32(tmem + lane_base + uint32_t(slot) * kSlotCols + cc * 32, v);
           const int jb = cc * 32;
-          if (jb + 32 <= rows) {
+          if (jb + 32 <= w.rows) {
 #pragma unroll
-            for (int i = 0; i < 32; ++i) acc += exp2f(fmaf(v[i], a.scale_log2, -s.lse[jb + i]));
+            for (int x = 0; x < 32; ++x) acc += exp2f(fmaf(v[x], a.scale_log2, -s.lse[jb + x]));
           } else {
-            for (int i = 0; i < rows - jb; ++i) acc += exp2f(fmaf(v[i], a.scale_log2, -s.lse[jb + i]));
+            for (int x = 0; x < w.rows - jb; ++x) acc += exp2f(fmaf(v[x], a.scale_log2, -s.lse[jb + x]));
           }
         }
-        const int tok = w.tok0 + t * kTile + warp * 32 + lane;
-        if (tok < w.N) pa_out[tok] = rg0 == 0 ? acc : pa_out[tok] + acc;
         tc::tc_fence_before();
-        __syncthreads();
-        if (tid == 0 && nbuf == 1 && t + 1 < T) mma_ok = issue_mma(t + 1, 0);
+        tc::mbar_arrive(&s.tempty[slot]);
+        const int tok = tile_of(w, i) * kTile + lrow;
+        if (tok < w.N) pa_out[tok] = acc;
       }
+      epi_barrier();  // every thread is done with this unit's rows and lse
     }
   }
-  if (!ok) {
-    flag_status(a.status, CONDUIT_FLAG_TIMEOUT);
-    if (tid == 0) {
-      for (uint32_t seq = pending_lo; seq < pending_hi; ++seq)
-        tc::mbar_wait(&s.full[seq % kStages], (seq / kStages) & 1);
-    }
+  __syncthreads();
+  if (tid == 0) {  // drain TMA copies issued but never consumed (only after an abort)
+    for (uint32_t n = s.counters[1]; n < s.counters[0]; ++n)
+      tc::mbar_wait(&s.kfull[n % kStages], (n / kStages) & 1);
   }
   tc::tc_fence_before();
   __syncthreads();
-  if (warp == 0) tc::tmem_dealloc(tmem, 512);
+  if (warp == 1) tc::tmem_dealloc(tmem, 2 * kSlotCols);
 }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
@@ -455,78 +448,55 @@ bool score_tc_supported(const KvDev& kv) {
   return true;
 }
 
-int score_tc_chunk(int R, const int32_t* tok_off_host, int n_layers, int Hkv) {
-  // largest chunk that still gives at least two units per SM of a 152-SM part
-  for (int chunk = 1024; chunk > kTile; chunk >>= 1) {
-    int64_t units = 0;
-    for (int r = 0; r < R; ++r)
-      units += int64_t(n_layers) * Hkv * ((tok_off_host[r + 1] - tok_off_host[r] + chunk - 1) / chunk);
-    if (units >= 304) return chunk;
-  }
-  return kTile;
-}
+int score_tc_groups(int rows) { return n_groups(rows); }
 
-size_t score_tc_part_bytes(int chunk, int max_tokens, int64_t total_rows) {
-  const int nch = (max_tokens + chunk - 1) / chunk;
-  return size_t(nch) * size_t(total_rows) * sizeof(float2);
-}
-
-cudaError_t launch_score_tc(const KvDev& kv, const BatchDev& b, const void* q, int32_t q_tot,
-                            const LayerList& layers, int max_tokens, int chunk, float2* part,
+cudaError_t launch_score_tc(const KvDev& kv, const BatchDev& b, const int32_t* q_off_host,
+                            const void* q, int32_t q_tot, const LayerList& layers, int rg_max,
                             float* pa, int32_t* status, cudaStream_t stream) {
   EncodeTiledFn enc = encode_fn();
   if (!enc) return cudaErrorNotSupported;
   CUtensorMap kmap;
-  cuuint64_t dims[2];
+  cuuint64_t dims[2] = {cuuint64_t(kD), 0};
   cuuint64_t strides[1] = {cuuint64_t(kD) * 2};
-  cuuint32_t box[2];
+  cuuint32_t box[2] = {64, 0};
   cuuint32_t estr[2] = {1, 1};
   if (kv.page_size == 0) {
-    dims[0] = kD;
     dims[1] = cuuint64_t(kv.L) * kv.Hkv * kv.n_tot;
-    box[0] = 64;
     box[1] = kTile;
   } else {
-    dims[0] = kD;
     dims[1] = cuuint64_t(kv.L) * kv.num_pages * kv.Hkv * kv.page_size;
-    box[0] = 64;
     box[1] = kv.page_size;
   }
-  CUresult cr = enc(&kmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, kv.k, dims, strides, box, estr,
-                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-  if (cr != CUDA_SUCCESS) return cudaErrorInvalidValue;
+  if (enc(&kmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, kv.k, dims, strides, box, estr,
+          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    return cudaErrorInvalidValue;
 
   TcArgs a{};
   a.kv = kv;
   a.b = b;
   a.q = static_cast<const __nv_bfloat16*>(q);
   a.q_tot = q_tot;
-  a.chunk = chunk;
-  a.nchunks_max = (max_tokens + chunk - 1) / chunk;
-  a.n_units = b.R * layers.n * kv.Hkv * a.nchunks_max;
-  a.total_rows = int64_t(layers.n) * kv.Hq * q_tot;
+  int units = 0;
+  for (int r = 0; r < b.R; ++r)
+    units += layers.n * kv.Hkv * n_groups(kv.G * (q_off_host[r + 1] - q_off_host[r]));
+  a.n_units = units;
+  a.rg_max = rg_max;
   a.scale_log2 = kLog2e / sqrtf(float(kD));
-  a.part = part;
   a.pa = pa;
   a.status = status;
   a.layers = layers;
+  if (units == 0) return cudaSuccess;
 
   int dev = 0, sms = 0;
   cudaError_t err;
   if ((err = cudaGetDevice(&dev))) return err;
   if ((err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev))) return err;
-  const int grid = std::max(1, std::min(a.n_units, sms));
-  if ((err = cudaFuncSetAttribute(rowstats_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  if ((err = cudaFuncSetAttribute(score_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                   int(kSmemBytes))))
     return err;
-  if ((err = cudaFuncSetAttribute(colsum_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                  int(kSmemBytes))))
-    return err;
-  rowstats_tc_kernel<<<grid, kThreads, kSmemBytes, stream>>>(kmap, a);
-  if ((err = cudaGetLastError())) return err;
-  colsum_tc_kernel<<<grid, kThreads, kSmemBytes, stream>>>(kmap, a);
-  count_launches(2);
+  score_tc_kernel<<<std::min(units, sms), kThreads, kSmemBytes, stream>>>(kmap, a);
+  count_launches(1);
   return cudaGetLastError();
 }
 

@@ -119,15 +119,33 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(BatchDev b, const f
       if ((key & pmask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
     }
     __syncthreads();
-    if (threadIdx.x == 0) {
-      int rem = remaining_s, digit = 255;
-      for (; digit > 0; --digit) {
-        const int c = int(hist[digit]);
-        if (c >= rem) break;
-        rem -= c;
+    if (threadIdx.x < 32) {
+      // Lane l holds digits 255-8l .. 248-8l (highest first); a warp scan of
+      // the lane totals finds the lane whose bins reach the remaining count.
+      const int lane = threadIdx.x;
+      int cnt[8], lsum = 0;
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        cnt[q] = int(hist[255 - 8 * lane - q]);
+        lsum += cnt[q];
       }
-      remaining_s = rem;
-      prefix_s = prefix | (uint32_t(digit) << shift);
+      int incl = lsum;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+      }
+      const int rem = remaining_s, excl = incl - lsum;
+      const unsigned hit = __ballot_sync(0xffffffffu, excl < rem && rem <= incl);
+      if (lane == __ffs(hit) - 1) {
+        int r2 = rem - excl, q = 0;
+        for (; q < 7; ++q) {
+          if (cnt[q] >= r2) break;
+          r2 -= cnt[q];
+        }
+        remaining_s = r2;
+        prefix_s = prefix | (uint32_t(255 - 8 * lane - q) << shift);
+      }
     }
     pmask |= 255u << shift;
     __syncthreads();
