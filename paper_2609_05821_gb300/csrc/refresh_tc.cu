@@ -4,18 +4,23 @@
 //
 // One CTA owns a block of 128 query rows of one (layer, KV head, request):
 // floor(128/G) consecutive selected rows times the G query heads that share
-// the KV head. Keys stream in tiles of 64 through a two-stage TMA ring:
-//   S = Q K_tile^T          tcgen05, rows as M, into TMEM columns [0, 64)
-//   softmax                 each thread owns one row: causal mask j <= p_i,
-//                           running max kept lazily (O and the row sum are
-//                           rescaled only when the max grows by 2^8), P in bf16
-//                           written into the K half of the tile's stage
-//   O += P V_tile           tcgen05 with V as an MN-major operand, TMEM
-//                           columns [64, 192)
-// then O / rowsum is written in bf16. Rows are sorted by position, so a
-// block needs keys up to its last row's position only. Two CTAs fit an SM
-// (96 KB shared, 256 TMEM columns each), so one CTA's softmax overlaps the
-// other's MMAs. Every wait is bounded (CONDUIT_FLAG_TIMEOUT on expiry).
+// the KV head. Keys stream in tiles of 64. Roles (192 threads):
+//   warp 0     one thread issues TMA loads of K and V tiles into two
+//              three-stage rings (K frees after S, V after P.V)
+//   warp 1     one thread issues tcgen05 MMAs: S(t) = Q K(t)^T into one of two
+//              TMEM S buffers (columns [0,64) / [64,128)), and O += P(t) V(t)
+//              into TMEM columns [128,256); S(t+2) is issued right after
+//              P.V(t), so the softmax of tile t+1 overlaps the tensor work
+//   warps 2-5  softmax: stage the query rows, then per tile read S(t) (one
+//              row per thread), apply the causal mask j <= p_i, keep a lazy
+//              running max (O and the row sum are rescaled only when the
+//              max grows by 2^8; the rescale is warp-uniform because
+//              tcgen05.ld/st are warp-collective), write P(t) in bf16 to one
+//              of two shared buffers, and finally write O / rowsum in bf16
+// Rows are sorted by position, so a block needs keys up to its last row's
+// position only. Every wait is bounded by one second; a role that gives up
+// raises an abort flag the others watch, the kernel sets
+// CONDUIT_FLAG_TIMEOUT, drains its copies and MMAs, and frees TMEM.
 #include <cuda.h>
 
 #include "internal.cuh"
@@ -27,13 +32,16 @@ namespace {
 constexpr int kD = 128;
 constexpr int kKT = 64;                          // keys per tile
 constexpr int kRows = 128;
-constexpr int kThreads = 128;
+constexpr int kThreads = 192;
+constexpr int kSoftThreads = 128;
+constexpr int kStages = 3;
 constexpr uint32_t kQHalf = kRows * 128;         // 16 KB: one 64-dim half of the query tile
-constexpr uint32_t kKVHalf = kKT * 128;          // 8 KB: one 64-dim half of a K or V tile
-constexpr uint32_t kStage = 4 * kKVHalf;         // K (2 halves) then V (2 halves)
-constexpr uint32_t kSmem = 1024 + 2 * kQHalf + 2 * kStage + 128;
+constexpr uint32_t kTileHalf = kKT * 128;        // 8 KB: one 64-dim half of a K or V tile
+constexpr uint32_t kTileBytes = 2 * kTileHalf;   // 16 KB
+constexpr uint32_t kPBytes = kRows * 128;        // 16 KB: 128 rows x 64 keys
+constexpr uint32_t kSmem = 1024 + 2 * kQHalf + 2 * kStages * kTileBytes + 2 * kPBytes + 256;
 constexpr uint32_t kTmemCols = 256;
-constexpr uint32_t kOCol = 64;
+constexpr uint32_t kOCol = 128;
 constexpr float kRescaleLog2 = 8.f;
 
 struct RefArgs {
@@ -50,17 +58,71 @@ struct RefArgs {
   int32_t* status;
 };
 
-__device__ __forceinline__ void load_kv_tile(const RefArgs& a, const CUtensorMap* kmap,
-                                             const CUtensorMap* vmap, uint8_t* st, uint64_t* bar,
-                                             int l, int g, int r, int t0, int N, int j0) {
+struct Smem {
+  uint8_t* q;        // [2 halves][128 rows][128 B]
+  uint8_t* k;        // [kStages][2 halves][64 keys][128 B]
+  uint8_t* v;        // [kStages][2 halves][64 keys][128 B]
+  uint8_t* p;        // [2][128 rows][128 B]
+  uint64_t *kfull, *kempty, *vfull, *vempty;  // [kStages] each
+  uint64_t *sfull, *pfull, *pempty;           // [2] each
+  uint64_t *obar, *qready, *mdone;
+  uint32_t* tmem_slot;
+  volatile int* abort;
+  uint32_t* counters;  // [0] K loads, [1] V loads, [2] K consumed, [3] V consumed
+};
+
+__device__ __forceinline__ Smem carve(uint8_t* raw) {
+  uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(raw) + 1023) & ~uintptr_t(1023));
+  Smem s;
+  s.q = base;
+  s.k = s.q + 2 * kQHalf;
+  s.v = s.k + kStages * kTileBytes;
+  s.p = s.v + kStages * kTileBytes;
+  uint64_t* bar = reinterpret_cast<uint64_t*>(s.p + 2 * kPBytes);
+  s.kfull = bar;
+  s.kempty = bar + kStages;
+  s.vfull = bar + 2 * kStages;
+  s.vempty = bar + 3 * kStages;
+  s.sfull = bar + 4 * kStages;
+  s.pfull = s.sfull + 2;
+  s.pempty = s.pfull + 2;
+  s.obar = s.pempty + 2;
+  s.qready = s.obar + 1;
+  s.mdone = s.qready + 1;
+  s.tmem_slot = reinterpret_cast<uint32_t*>(s.mdone + 1);
+  s.abort = reinterpret_cast<volatile int*>(s.tmem_slot + 1);
+  s.counters = reinterpret_cast<uint32_t*>(s.tmem_slot + 2);
+  return s;
+}
+
+__device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int* abort) {
+  if (tc::mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = tc::globaltimer_ns();
+  for (uint32_t i = 1; i < tc::kSpinLimit; ++i) {
+    if (tc::mbar_try_wait(bar, parity)) return true;
+    if ((i & 7u) == 0 && (*abort || tc::globaltimer_ns() - t0 > tc::kWaitNs)) return false;
+  }
+  return false;
+}
+
+__device__ __forceinline__ void raise_abort(const RefArgs& a, const Smem& s, int32_t site) {
+  if (!*s.abort) flag_status(a.status, CONDUIT_FLAG_TIMEOUT | site);
+  *s.abort = 1;
+}
+
+__device__ __forceinline__ void soft_barrier() {
+  asm volatile("bar.sync 1, %0;" ::"n"(kSoftThreads) : "memory");
+}
+
+// TMA of the 64-key tile starting at request-local key j0 (one 64-dim half per box).
+__device__ __forceinline__ void load_tile(const RefArgs& a, const CUtensorMap* map, uint8_t* dst,
+                                          uint64_t* bar, int l, int g, int r, int t0, int N, int j0) {
   const KvDev& kv = a.kv;
-  tc::mbar_arrive_expect_tx(bar, kStage);
+  tc::mbar_arrive_expect_tx(bar, kTileBytes);
   if (kv.page_size == 0) {
     const int32_t y = int32_t((int64_t(l) * kv.Hkv + g) * kv.n_tot + t0 + j0);
-    tc::tma_load_2d(st, kmap, bar, 0, y);
-    tc::tma_load_2d(st + kKVHalf, kmap, bar, 64, y);
-    tc::tma_load_2d(st + 2 * kKVHalf, vmap, bar, 0, y);
-    tc::tma_load_2d(st + 3 * kKVHalf, vmap, bar, 64, y);
+    tc::tma_load_2d(dst, map, bar, 0, y);
+    tc::tma_load_2d(dst + kTileHalf, map, bar, 64, y);
   } else {
     const int ps = kv.page_size;
     const int last_page = (N - 1) / ps;
@@ -68,25 +130,17 @@ __device__ __forceinline__ void load_kv_tile(const RefArgs& a, const CUtensorMap
       const int lp = min((j0 + i * ps) / ps, last_page);
       const int page = kv.page_table[int64_t(r) * kv.max_pages + lp];
       const int32_t y = int32_t(((int64_t(l) * kv.num_pages + page) * kv.Hkv + g) * ps);
-      tc::tma_load_2d(st + i * ps * 128, kmap, bar, 0, y);
-      tc::tma_load_2d(st + kKVHalf + i * ps * 128, kmap, bar, 64, y);
-      tc::tma_load_2d(st + 2 * kKVHalf + i * ps * 128, vmap, bar, 0, y);
-      tc::tma_load_2d(st + 3 * kKVHalf + i * ps * 128, vmap, bar, 64, y);
+      tc::tma_load_2d(dst + i * ps * 128, map, bar, 0, y);
+      tc::tma_load_2d(dst + kTileHalf + i * ps * 128, map, bar, 64, y);
     }
   }
 }
 
-__global__ void __launch_bounds__(kThreads, 2)
+__global__ void __launch_bounds__(kThreads, 1)
     refresh_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
                       const __grid_constant__ RefArgs a) {
   extern __shared__ uint8_t smem_raw[];
-  uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* q_s = base;                       // [2][128 rows][128 B]
-  uint8_t* stages = base + 2 * kQHalf;       // [2][K half0, K half1, V half0, V half1]
-  uint64_t* full = reinterpret_cast<uint64_t*>(stages + 2 * kStage);  // [2]
-  uint64_t* s_bar = full + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(s_bar + 1);
-
+  const Smem s = carve(smem_raw);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int l = blockIdx.z, g = blockIdx.y;
   const KvDev& kv = a.kv;
@@ -112,179 +166,260 @@ __global__ void __launch_bounds__(kThreads, 2)
   if (p_max < 0) return;
   const int ntiles = p_max / kKT + 1;
 
-  // this thread's row: selected row i0 + row / G, query head g*G + row % G
-  const int row = warp * 32 + lane;
-  const bool row_ok = row < cnt * G;
-  const int i_row = i0 + (row_ok ? row / G : 0);
-  const int h_row = g * G + (row_ok ? row % G : 0);
-  int p_row = row_ok ? a.idx[i_row] : -1;
-  if (p_row >= N) p_row = -1;
-
   if (tid == 0) {
-    tc::mbar_init(&full[0], 1);
-    tc::mbar_init(&full[1], 1);
-    tc::mbar_init(s_bar, 1);
+    for (int i = 0; i < kStages; ++i) {
+      tc::mbar_init(&s.kfull[i], 1);
+      tc::mbar_init(&s.kempty[i], 1);
+      tc::mbar_init(&s.vfull[i], 1);
+      tc::mbar_init(&s.vempty[i], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      tc::mbar_init(&s.sfull[i], 1);
+      tc::mbar_init(&s.pfull[i], kSoftThreads);
+      tc::mbar_init(&s.pempty[i], 1);
+    }
+    tc::mbar_init(s.obar, 1);
+    tc::mbar_init(s.qready, 1);
+    tc::mbar_init(s.mdone, 1);
+    *s.abort = 0;
+    for (int i = 0; i < 4; ++i) s.counters[i] = 0;
     tc::fence_barrier_init();
     tc::prefetch_tensormap(&kmap);
     tc::prefetch_tensormap(&vmap);
   }
-  if (warp == 0) tc::tmem_alloc(tmem_slot, kTmemCols);
-  // query tile: rows as above, zero beyond cnt * G
-  for (int x = tid; x < kRows * 16; x += kThreads) {
-    const int rr = x >> 4, ch = x & 15;
-    uint4 val = make_uint4(0u, 0u, 0u, 0u);
-    if (rr < cnt * G) {
-      const int ii = i0 + rr / G, hh = g * G + rr % G;
-      val = *reinterpret_cast<const uint4*>(a.q_rows + ((int64_t(l) * a.n_sel + ii) * Hq + hh) * kD + ch * 8);
-    }
-    *reinterpret_cast<uint4*>(q_s + (ch >> 3) * kQHalf + tc::sw128_offset(rr, ch & 7)) = val;
-  }
-  tc::fence_proxy_async_smem();
+  if (warp == 1) tc::tmem_alloc(s.tmem_slot, kTmemCols);
   __syncthreads();
   tc::tc_fence_after();
-  const uint32_t tmem = *tmem_slot;
-  const uint32_t lane_base = uint32_t(warp * 32) << 16;
+  const uint32_t tmem = *s.tmem_slot;
 
-  bool ok = true;
-  int32_t site = 0;
-  if (tid == 0) {
-    load_kv_tile(a, &kmap, &vmap, stages, &full[0], l, g, r, t0, N, 0);
-    if (ntiles > 1) load_kv_tile(a, &kmap, &vmap, stages + kStage, &full[1], l, g, r, t0, N, kKT);
-  }
-  int loads_issued = min(ntiles, 2);
-
-  float m_ref = -INFINITY, lsum = 0.f;
-  const uint32_t q_addr = tc::smem_u32(q_s);
-  const uint32_t idesc_s = tc::idesc_bf16(kRows, kKT);
-  const uint32_t idesc_o = tc::idesc_bf16(kRows, kD, /*b_mn_major=*/true);
-  int t = 0;
-  for (; t < ntiles; ++t) {
-    const int st = t & 1;
-    uint8_t* stage = stages + st * kStage;
-    const uint32_t k_addr = tc::smem_u32(stage);
-    int issued = 1;
-    if (tid == 0) {
-      if (!tc::mbar_wait(&full[st], (t >> 1) & 1)) {
-        issued = 0;
-      } else {
-        tc::tc_fence_after();
-#pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {
-          const uint32_t off = (kk & 3) * 32;
-          tc::mma_bf16(tmem, tc::desc_sw128(q_addr + (kk >> 2) * kQHalf + off),
-                       tc::desc_sw128(k_addr + (kk >> 2) * kKVHalf + off), idesc_s, kk > 0);
-        }
-        tc::mma_commit(s_bar);
-      }
+  if (warp == 0 && lane == 0) {
+    // ---------------------------------------------------------------- loads
+    uint32_t nk = 0, nv = 0;
+    for (int t = 0; t < ntiles; ++t) {
+      const int st = t % kStages;
+      const uint32_t ph = ((t / kStages) & 1) ^ 1;
+      if (!wait_or_abort(&s.kempty[st], ph, s.abort)) { raise_abort(a, s, tc::kSiteLoad); break; }
+      load_tile(a, &kmap, s.k + st * kTileBytes, &s.kfull[st], l, g, r, t0, N, t * kKT);
+      ++nk;
+      if (!wait_or_abort(&s.vempty[st], ph, s.abort)) { raise_abort(a, s, tc::kSiteLoad); break; }
+      load_tile(a, &vmap, s.v + st * kTileBytes, &s.vfull[st], l, g, r, t0, N, t * kKT);
+      ++nv;
     }
-    if (!__syncthreads_and(issued)) { ok = false; site = tc::kSiteLoad; break; }
-    // S of tile t ready, and every earlier MMA (the P.V of tile t-1) is complete
-    if (!__syncthreads_and(tc::mbar_wait(s_bar, t & 1))) { ok = false; site = tc::kSiteMma; break; }
-    tc::tc_fence_after();
-    if (tid == 0 && t >= 1 && t + 1 < ntiles) {  // stage of tile t-1 is free again
-      load_kv_tile(a, &kmap, &vmap, stages + ((t + 1) & 1) * kStage, &full[(t + 1) & 1], l, g, r, t0,
-                   N, (t + 1) * kKT);
-    }
-    if (t >= 1 && t + 1 < ntiles) ++loads_issued;
-
-    float sv[2][32];
-    tc::tmem_ld32(tmem + lane_base + 0, sv[0]);
-    tc::tmem_ld32(tmem + lane_base + 32, sv[1]);
-    const int j0 = t * kKT;
-    float tmax = -INFINITY;
-#pragma unroll
-    for (int h2 = 0; h2 < 2; ++h2)
-#pragma unroll
-      for (int i = 0; i < 32; ++i) {
-        const float x = (j0 + h2 * 32 + i <= p_row) ? sv[h2][i] * a.scale_log2 : -INFINITY;
-        sv[h2][i] = x;
-        tmax = fmaxf(tmax, x);
-      }
-    // Lazy rescale of this row's O and sum when its max grew by more than 2^8.
-    // tcgen05.ld / st are warp-collective, so the TMEM pass runs for the whole
-    // warp whenever any lane needs it; lanes that do not rescale use alpha = 1.
-    const bool need = tmax > m_ref + kRescaleLog2 || (m_ref == -INFINITY && tmax != -INFINITY);
-    const float alpha = need ? exp2f(m_ref - tmax) : 1.f;  // 0 when m_ref is -inf
-    if (__any_sync(0xffffffffu, need) && t > 0) {
-      for (int c = 0; c < kD; c += 32) {
-        float o[32];
-        tc::tmem_ld32(tmem + lane_base + kOCol + c, o);
-#pragma unroll
-        for (int i = 0; i < 32; ++i) o[i] *= alpha;
-        tc::tmem_st32(tmem + lane_base + kOCol + c, o);
-      }
-    }
-    if (need) {
-      lsum *= alpha;
-      m_ref = tmax;
-    }
-    // P = 2^(x - m_ref) in bf16 into the K half of this stage (K is consumed)
-#pragma unroll
-    for (int h2 = 0; h2 < 2; ++h2) {
-#pragma unroll
-      for (int c8 = 0; c8 < 4; ++c8) {
-        uint32_t w4[4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const float p0 = (m_ref == -INFINITY) ? 0.f : exp2f(sv[h2][c8 * 8 + 2 * u] - m_ref);
-          const float p1 = (m_ref == -INFINITY) ? 0.f : exp2f(sv[h2][c8 * 8 + 2 * u + 1] - m_ref);
-          lsum += p0 + p1;
-          __nv_bfloat162 pr = __floats2bfloat162_rn(p0, p1);
-          w4[u] = *reinterpret_cast<uint32_t*>(&pr);
-        }
-        const int chunk = h2 * 4 + c8;  // 16-byte chunk of the 128-byte P row
-        *reinterpret_cast<uint4*>(stage + tc::sw128_offset(row, chunk)) =
-            make_uint4(w4[0], w4[1], w4[2], w4[3]);
-      }
-    }
-    tc::fence_proxy_async_smem();
-    tc::tc_fence_before();
-    __syncthreads();
-    if (tid == 0) {
+    s.counters[0] = nk;
+    s.counters[1] = nv;
+  } else if (warp == 1 && lane == 0) {
+    // ------------------------------------------------------------------ MMA
+    uint32_t ck = 0, cv = 0;
+    const uint32_t q_addr = tc::smem_u32(s.q);
+    const uint32_t idesc_s = tc::idesc_bf16(kRows, kKT);
+    const uint32_t idesc_o = tc::idesc_bf16(kRows, kD, /*b_mn_major=*/true);
+    auto issue_s = [&](int t) -> bool {  // S(t) = Q K(t)^T into S buffer t & 1
+      const int st = t % kStages;
+      if (!wait_or_abort(&s.kfull[st], (t / kStages) & 1, s.abort)) return false;
+      ++ck;
       tc::tc_fence_after();
-      const uint32_t p_addr = k_addr;                       // P: [128 rows][64 keys] K-major
-      const uint32_t v_addr = k_addr + 2 * kKVHalf;          // V: [64 keys][128 dims] MN-major
+      const uint32_t k_addr = tc::smem_u32(s.k + st * kTileBytes);
+#pragma unroll
+      for (int kk = 0; kk < 8; ++kk) {
+        const uint32_t off = (kk & 3) * 32;
+        tc::mma_bf16(tmem + uint32_t(t & 1) * kKT, tc::desc_sw128(q_addr + (kk >> 2) * kQHalf + off),
+                     tc::desc_sw128(k_addr + (kk >> 2) * kTileHalf + off), idesc_s, kk > 0);
+      }
+      tc::mma_commit(&s.kempty[st]);
+      tc::mma_commit(&s.sfull[t & 1]);
+      return true;
+    };
+    bool ok = wait_or_abort(s.qready, 0, s.abort);
+    if (ok) ok = issue_s(0);
+    if (ok && ntiles > 1) ok = issue_s(1);
+    for (int t = 0; t < ntiles && ok; ++t) {
+      const int b = t & 1, st = t % kStages;
+      if (!wait_or_abort(&s.pfull[b], (t >> 1) & 1, s.abort)) { ok = false; break; }
+      if (!wait_or_abort(&s.vfull[st], (t / kStages) & 1, s.abort)) { ok = false; break; }
+      ++cv;
+      tc::tc_fence_after();
+      const uint32_t p_addr = tc::smem_u32(s.p + b * kPBytes);
+      const uint32_t v_addr = tc::smem_u32(s.v + st * kTileBytes);
 #pragma unroll
       for (int kk = 0; kk < kKT / 16; ++kk) {
         tc::mma_bf16(tmem + kOCol, tc::desc_sw128(p_addr + kk * 32),
-                     tc::desc_sw128_mn(v_addr + kk * 2048, kKVHalf), idesc_o, t > 0 || kk > 0);
+                     tc::desc_sw128_mn(v_addr + kk * 2048, kTileHalf), idesc_o, t > 0 || kk > 0);
+      }
+      tc::mma_commit(&s.vempty[st]);
+      tc::mma_commit(&s.pempty[b]);
+      tc::mma_commit(s.obar);
+      if (t + 2 < ntiles && !issue_s(t + 2)) { ok = false; break; }
+    }
+    if (!ok) raise_abort(a, s, tc::kSiteMma);
+    s.counters[2] = ck;
+    s.counters[3] = cv;
+    tc::mma_commit(s.mdone);  // every MMA issued above has completed once this arrives
+    tc::mbar_wait(s.mdone, 0);
+  } else if (warp >= 2) {
+    // -------------------------------------------------------------- softmax
+    const int et = tid - 64;
+    const int quarter = warp & 3;
+    const int row = quarter * 32 + lane;                 // TMEM lane = query row of the tile
+    const uint32_t lane_base = uint32_t(quarter * 32) << 16;
+    const bool row_ok = row < cnt * G;
+    const int i_row = i0 + (row_ok ? row / G : 0);
+    const int h_row = g * G + (row_ok ? row % G : 0);
+    int p_row = row_ok ? a.idx[i_row] : -1;
+    if (p_row >= N) p_row = -1;
+    // query tile: row ρ = (i0 + ρ / G, head g*G + ρ % G), zero beyond cnt * G
+    for (int base = 0; base < kRows * 16; base += kSoftThreads * 8) {
+      uint4 val[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int x = base + u * kSoftThreads + et;
+        const int rr = x >> 4, ch = x & 15;
+        val[u] = make_uint4(0u, 0u, 0u, 0u);
+        if (rr < cnt * G) {
+          const int ii = i0 + rr / G, hh = g * G + rr % G;
+          val[u] = *reinterpret_cast<const uint4*>(a.q_rows + ((int64_t(l) * a.n_sel + ii) * Hq + hh) * kD + ch * 8);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int x = base + u * kSoftThreads + et;
+        const int rr = x >> 4, ch = x & 15;
+        *reinterpret_cast<uint4*>(s.q + (ch >> 3) * kQHalf + tc::sw128_offset(rr, ch & 7)) = val[u];
       }
     }
-  }
-  // final P.V -> O ready
-  if (ok) {
-    if (tid == 0) tc::mma_commit(s_bar);
-    if (!__syncthreads_and(tc::mbar_wait(s_bar, ntiles & 1))) { ok = false; site = tc::kSiteFinal; }
-  }
-  if (ok) {
-    tc::tc_fence_after();
-    const float inv = lsum > 0.f ? 1.f / lsum : 0.f;
-    __nv_bfloat16* dst = a.out + ((int64_t(l) * a.n_sel + i_row) * Hq + h_row) * kD;
-    for (int c = 0; c < kD; c += 32) {
-      float o[32];
-      tc::tmem_ld32(tmem + lane_base + kOCol + c, o);
-      if (row_ok && p_row >= 0) {
+    tc::fence_proxy_async_smem();
+    soft_barrier();
+    if (et == 0) tc::mbar_arrive(s.qready);
+
+    bool ok = true;
+    float m_ref = -INFINITY, lsum = 0.f;
+    for (int t = 0; t < ntiles; ++t) {
+      const int b = t & 1;
+      // the tcgen05.ld below is warp-collective: the whole warp goes on or stops
+      const bool got = __all_sync(0xffffffffu, ok && wait_or_abort(&s.sfull[b], (t >> 1) & 1, s.abort));
+      if (!got) {
+        if (ok) raise_abort(a, s, tc::kSiteMma);
+        ok = false;
+        continue;
+      }
+      tc::tc_fence_after();
+      float sv[2][32];
+      tc::tmem_ld32(tmem + lane_base + uint32_t(b) * kKT, sv[0]);
+      tc::tmem_ld32(tmem + lane_base + uint32_t(b) * kKT + 32, sv[1]);
+      const int j0 = t * kKT;
+      float tm[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+      if (j0 + kKT - 1 <= p_row) {  // the whole tile is visible to this row
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
+        for (int h2 = 0; h2 < 2; ++h2)
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            sv[h2][i] *= a.scale_log2;
+            tm[i & 3] = fmaxf(tm[i & 3], sv[h2][i]);
+          }
+      } else {
+#pragma unroll
+        for (int h2 = 0; h2 < 2; ++h2)
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const float x = (j0 + h2 * 32 + i <= p_row) ? sv[h2][i] * a.scale_log2 : -INFINITY;
+            sv[h2][i] = x;
+            tm[i & 3] = fmaxf(tm[i & 3], x);
+          }
+      }
+      const float tmax = fmaxf(fmaxf(tm[0], tm[1]), fmaxf(tm[2], tm[3]));
+      const bool need = tmax > m_ref + kRescaleLog2 || (m_ref == -INFINITY && tmax != -INFINITY);
+      const float alpha = need ? exp2f(m_ref - tmax) : 1.f;  // 0 when m_ref is -inf
+      if (__any_sync(0xffffffffu, need) && t > 0) {
+        // P.V(t-1) must be complete before this warp rescales its rows of O.
+        // S(t) was issued after P.V(t-2), so obar is at most one phase behind
+        // here and its parity cannot alias.
+        if (!__all_sync(0xffffffffu, wait_or_abort(s.obar, (t - 1) & 1, s.abort))) {
+          raise_abort(a, s, tc::kSiteMma);
+          ok = false;
+          continue;
+        }
+        tc::tc_fence_after();
+        for (int c = 0; c < kD; c += 32) {
+          float o[32];
+          tc::tmem_ld32(tmem + lane_base + kOCol + c, o);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) o[i] *= alpha;
+          tc::tmem_st32(tmem + lane_base + kOCol + c, o);
+        }
+      }
+      if (need) {
+        lsum *= alpha;
+        m_ref = tmax;
+      }
+      // the P buffer of tile t was last read by P.V(t-2)
+      if (!wait_or_abort(&s.pempty[b], ((t >> 1) & 1) ^ 1, s.abort)) {
+        raise_abort(a, s, tc::kSiteMma);
+        ok = false;
+        continue;
+      }
+      uint8_t* pb = s.p + b * kPBytes;
+      float ls[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int h2 = 0; h2 < 2; ++h2) {
+#pragma unroll
+        for (int c8 = 0; c8 < 4; ++c8) {
           uint32_t w4[4];
 #pragma unroll
-          for (int k2 = 0; k2 < 4; ++k2) {
-            __nv_bfloat162 pr = __floats2bfloat162_rn(o[u * 8 + 2 * k2] * inv, o[u * 8 + 2 * k2 + 1] * inv);
-            w4[k2] = *reinterpret_cast<uint32_t*>(&pr);
+          for (int u = 0; u < 4; ++u) {
+            const float p0 = (m_ref == -INFINITY) ? 0.f : tc::ex2(sv[h2][c8 * 8 + 2 * u] - m_ref);
+            const float p1 = (m_ref == -INFINITY) ? 0.f : tc::ex2(sv[h2][c8 * 8 + 2 * u + 1] - m_ref);
+            ls[u] += p0 + p1;
+            __nv_bfloat162 pr = __floats2bfloat162_rn(p0, p1);
+            w4[u] = *reinterpret_cast<uint32_t*>(&pr);
           }
-          *reinterpret_cast<uint4*>(dst + c + u * 8) = make_uint4(w4[0], w4[1], w4[2], w4[3]);
+          *reinterpret_cast<uint4*>(pb + tc::sw128_offset(row, h2 * 4 + c8)) =
+              make_uint4(w4[0], w4[1], w4[2], w4[3]);
+        }
+      }
+      lsum += (ls[0] + ls[1]) + (ls[2] + ls[3]);
+      tc::fence_proxy_async_smem();
+      tc::tc_fence_before();
+      tc::mbar_arrive(&s.pfull[b]);
+    }
+    // O is complete once the MMA thread's final commit arrives. (The obar phase
+    // of the last P.V could alias: after this warp's last tile only P.V up to
+    // ntiles-3 is known to be done, two phases behind.)
+    if (ok && !wait_or_abort(s.mdone, 0, s.abort)) {
+      raise_abort(a, s, tc::kSiteFinal);
+      ok = false;
+    }
+    const bool all_ok = !__any_sync(0xffffffffu, !ok);
+    if (all_ok) {
+      tc::tc_fence_after();
+      const float inv = lsum > 0.f ? 1.f / lsum : 0.f;
+      __nv_bfloat16* dst = a.out + ((int64_t(l) * a.n_sel + i_row) * Hq + h_row) * kD;
+      for (int c = 0; c < kD; c += 32) {
+        float o[32];
+        tc::tmem_ld32(tmem + lane_base + kOCol + c, o);
+        if (row_ok && p_row >= 0) {
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            uint32_t w4[4];
+#pragma unroll
+            for (int k2 = 0; k2 < 4; ++k2) {
+              __nv_bfloat162 pr = __floats2bfloat162_rn(o[u * 8 + 2 * k2] * inv, o[u * 8 + 2 * k2 + 1] * inv);
+              w4[k2] = *reinterpret_cast<uint32_t*>(&pr);
+            }
+            *reinterpret_cast<uint4*>(dst + c + u * 8) = make_uint4(w4[0], w4[1], w4[2], w4[3]);
+          }
         }
       }
     }
-  } else {
-    flag_status(a.status, CONDUIT_FLAG_TIMEOUT | site);
-    if (tid == 0) {  // drain loads still in flight into this CTA's shared memory
-      for (int tt = t; tt < loads_issued; ++tt) tc::mbar_wait(&full[tt & 1], (tt >> 1) & 1);
-    }
+  }
+  __syncthreads();
+  if (tid == 0) {  // drain loads issued but never consumed (only after an abort)
+    for (uint32_t n = s.counters[2]; n < s.counters[0]; ++n)
+      tc::mbar_wait(&s.kfull[n % kStages], (n / kStages) & 1);
+    for (uint32_t n = s.counters[3]; n < s.counters[1]; ++n)
+      tc::mbar_wait(&s.vfull[n % kStages], (n / kStages) & 1);
   }
   tc::tc_fence_before();
   __syncthreads();
-  if (warp == 0) tc::tmem_dealloc(tmem, kTmemCols);
+  if (warp == 1) tc::tmem_dealloc(tmem, kTmemCols);
 }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,

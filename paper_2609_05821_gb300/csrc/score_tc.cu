@@ -145,7 +145,7 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, vo
   const uint64_t t0 = tc::globaltimer_ns();
   for (uint32_t i = 1; i < tc::kSpinLimit; ++i) {
     if (tc::mbar_try_wait(bar, parity)) return true;
-    if ((i & 63u) == 0 && (*abort || tc::globaltimer_ns() - t0 > tc::kWaitNs)) return false;
+    if ((i & 7u) == 0 && (*abort || tc::globaltimer_ns() - t0 > tc::kWaitNs)) return false;
   }
   return false;
 }
@@ -341,12 +341,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       float m0 = -INFINITY, z0 = 0.f, m1 = -INFINITY, z1 = 0.f;
       for (int i = 0; i < w.tiles; ++i) {            // pass A
         const int slot = tseq & 1;
-        if (ok && !wait_or_abort(&s.tfull[slot], (tseq >> 1) & 1, s.abort)) {
-          if (!*s.abort) raise_abort(a, s, tc::kSiteMma);
-          ok = false;
-        }
+        // tcgen05.ld is warp-collective: the whole warp goes on or stops
+        const bool got = __all_sync(0xffffffffu, ok && wait_or_abort(&s.tfull[slot], (tseq >> 1) & 1, s.abort));
         ++tseq;
-        if (!ok) continue;
+        if (!got) {
+          if (ok && !*s.abort) raise_abort(a, s, tc::kSiteMma);
+          ok = false;
+          continue;
+        }
         tc::tc_fence_after();
         const int tok0 = i * kTile;
         for (int rb = 0; rb < nrb; ++rb) {
@@ -355,20 +357,23 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int cc = 0; cc < 4; ++cc) {
             float v[32];
             tc::tmem_ld32(tmem + lane_base + uint32_t(slot) * kSlotCols + rb * 128 + cc * 32, v);
-            float cmax = -INFINITY;
             const int tok = tok0 + cc * 32;
+            if (tok + 32 > w.N) {  // ragged last tile only
 #pragma unroll
-            for (int x = 0; x < 32; ++x) {
-              if (tok + x >= w.N) v[x] = -INFINITY;
-              cmax = fmaxf(cmax, v[x]);
+              for (int x = 0; x < 32; ++x)
+                if (tok + x >= w.N) v[x] = -INFINITY;
             }
+            float cm[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+            for (int x = 0; x < 32; ++x) cm[x & 3] = fmaxf(cm[x & 3], v[x]);
+            const float cmax = fmaxf(fmaxf(cm[0], cm[1]), fmaxf(cm[2], cm[3]));
             const float mn = fmaxf(mr, cmax);
             if (mn != -INFINITY) {
               const float nb = -mn * a.scale_log2;
-              float acc = 0.f;
+              float ac[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-              for (int x = 0; x < 32; ++x) acc += exp2f(fmaf(v[x], a.scale_log2, nb));
-              zr = zr * exp2f((mr - mn) * a.scale_log2) + acc;
+              for (int x = 0; x < 32; ++x) ac[x & 3] += tc::ex2(fmaf(v[x], a.scale_log2, nb));
+              zr = zr * exp2f((mr - mn) * a.scale_log2) + ((ac[0] + ac[1]) + (ac[2] + ac[3]));
               mr = mn;
             }
           }
@@ -385,25 +390,35 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int nchunk = (w.rows + 31) / 32;
       for (int i = w.tiles; i < 2 * w.tiles; ++i) {  // pass B
         const int slot = tseq & 1;
-        if (ok && !wait_or_abort(&s.tfull[slot], (tseq >> 1) & 1, s.abort)) {
-          if (!*s.abort) raise_abort(a, s, tc::kSiteMma);
-          ok = false;
-        }
+        // tcgen05.ld is warp-collective: the whole warp goes on or stops
+        const bool got = __all_sync(0xffffffffu, ok && wait_or_abort(&s.tfull[slot], (tseq >> 1) & 1, s.abort));
         ++tseq;
-        if (!ok) continue;
+        if (!got) {
+          if (ok && !*s.abort) raise_abort(a, s, tc::kSiteMma);
+          ok = false;
+          continue;
+        }
         tc::tc_fence_after();
-        float acc = 0.f;
+        float ac[4] = {0.f, 0.f, 0.f, 0.f};
         for (int cc = 0; cc < nchunk; ++cc) {
           float v[32];
           tc::tmem_ld32(tmem + lane_base + uint32_t(slot) * kSlotCols + cc * 32, v);
           const int jb = cc * 32;
+          const float4* l4 = reinterpret_cast<const float4*>(s.lse + jb);
           if (jb + 32 <= w.rows) {
 #pragma unroll
-            for (int x = 0; x < 32; ++x) acc += exp2f(fmaf(v[x], a.scale_log2, -s.lse[jb + x]));
+            for (int x4 = 0; x4 < 8; ++x4) {
+              const float4 lv = l4[x4];
+              ac[0] += tc::ex2(fmaf(v[4 * x4 + 0], a.scale_log2, -lv.x));
+              ac[1] += tc::ex2(fmaf(v[4 * x4 + 1], a.scale_log2, -lv.y));
+              ac[2] += tc::ex2(fmaf(v[4 * x4 + 2], a.scale_log2, -lv.z));
+              ac[3] += tc::ex2(fmaf(v[4 * x4 + 3], a.scale_log2, -lv.w));
+            }
           } else {
-            for (int x = 0; x < w.rows - jb; ++x) acc += exp2f(fmaf(v[x], a.scale_log2, -s.lse[jb + x]));
+            for (int x = 0; x < w.rows - jb; ++x) ac[x & 3] += tc::ex2(fmaf(v[x], a.scale_log2, -s.lse[jb + x]));
           }
         }
+        const float acc = (ac[0] + ac[1]) + (ac[2] + ac[3]);
         tc::tc_fence_before();
         tc::mbar_arrive(&s.tempty[slot]);
         const int tok = tile_of(w, i) * kTile + lrow;

@@ -15,6 +15,7 @@ namespace tc {
 #define CONDUIT_WAIT_NS 1000000000ull
 #endif
 constexpr uint32_t kSpinLimit = 1u << 26;        // hard cap on polls of one wait
+constexpr uint32_t kSuspendNs = 1000000;         // a polling thread sleeps up to 1 ms per try
 constexpr uint64_t kWaitNs = CONDUIT_WAIT_NS;    // polling time before a wait gives up (1 s)
 
 // Diagnostic bits of the status word, set next to CONDUIT_FLAG_TIMEOUT to
@@ -25,6 +26,14 @@ constexpr int32_t kSiteFinal = 1 << 10;  // the last commit of a CTA never arriv
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+// 2^x by the SFU's approximate exp2 with subnormal results flushed to zero
+// (softmax weights below 2^-126 of the row maximum are dropped).
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
 }
 
 // ------------------------------------------------------------------ mbarrier
@@ -51,11 +60,11 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   asm volatile(
       "{\n"
       ".reg .pred p;\n"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n"
       "selp.u32 %0, 1, 0, p;\n"
       "}\n"
       : "=r"(done)
-      : "r"(smem_u32(bar)), "r"(parity)
+      : "r"(smem_u32(bar)), "r"(parity), "r"(kSuspendNs)
       : "memory");
   return done != 0;
 }
@@ -73,7 +82,7 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
   const uint64_t t0 = globaltimer_ns();
   for (uint32_t i = 1; i < kSpinLimit; ++i) {
     if (mbar_try_wait(bar, parity)) return true;
-    if ((i & 255u) == 0 && globaltimer_ns() - t0 > kWaitNs) return false;
+    if ((i & 7u) == 0 && globaltimer_ns() - t0 > kWaitNs) return false;
   }
   return false;
 }
