@@ -189,7 +189,7 @@ def call_kernels(pipe) -> dict:
     tc = pipe.kv.k.dtype == torch.bfloat16 and pipe.kv.head_dim == 128
     tail = ["finalize_tokens_kernel", "image_means_kernel"]
     if tc:
-        score = (["value_sumsq_kernel", "score_tc_kernel"] + tail, "hbm", "score_tc.cu")
+        score = (["score_tc_kernel"] + tail, "hbm", "score_tc.cu")
         refresh = (["refresh_tc_kernel"], "tensor", "refresh_tc.cu")
     else:
         score = (["value_sumsq_kernel", "rowstats_kernel", "colsum_kernel"] + tail, "alu", "score_simt.cu")

@@ -170,7 +170,7 @@ ScoreLayout score_layout(const conduit_kv* kv, const conduit_batch* b, int n_lay
   s.pa = off;
   off += align_up(size_t(n_layers) * kv->num_kv_heads * s.rg_max * n_tot * sizeof(float));
   s.ss = off;
-  off += align_up(size_t(n_layers) * n_tot * sizeof(float));
+  off += align_up(size_t(n_layers) * kv->num_kv_heads * n_tot * sizeof(float));
   s.attn = off;
   off += align_up(n_tot * sizeof(float));
   s.total = off;
@@ -269,11 +269,12 @@ conduit_status conduit_score(const conduit_kv* kv, const conduit_batch* batch, c
   float* attn = attn_sum ? attn_sum : reinterpret_cast<float*>(ws + lay.attn);
   cudaStream_t cs = static_cast<cudaStream_t>(stream);
   cudaError_t err;
-  if ((err = launch_value_sumsq(kd, bd, ll, max_tok, ss, cs))) return cuda_fail(err, "value_sumsq");
-  if (lay.tc)
-    err = launch_score_tc(kd, bd, batch->q_off, q, batch->q_off[R], ll, lay.rg_max, pa, status, cs);
-  else
+  if (lay.tc) {  // the tensor-core kernel also streams V for the value norms
+    err = launch_score_tc(kd, bd, batch->q_off, q, batch->q_off[R], ll, lay.rg_max, pa, ss, status, cs);
+  } else {
+    if ((err = launch_value_sumsq(kd, bd, ll, max_tok, ss, cs))) return cuda_fail(err, "value_sumsq");
     err = launch_score_simt(kd, bd, q, batch->q_off[R], ll, max_rows, max_tok, stats, pa, cs);
+  }
   if (err) return cuda_fail(err, "score");
   if ((err = launch_finalize(pa, ss, bd, ll.n, kd.Hkv, kd.Hq, lay.rg_max, lay.group_rows, kd.n_tot,
                              s, attn, g, status, cs)))

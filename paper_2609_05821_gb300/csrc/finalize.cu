@@ -1,27 +1,27 @@
 // Per-token and per-image reductions of the scoring pass (Conduit Eqs. 6-8).
 //   a_t^(l)  = sum_g sum_group pa[l][g][group][t] / (|Q| Hq)   Eq. 6 (head/query mean)
-//   v_t^(l)  = sqrt(ss[l][t])                                  concatenated-head norm
+//   v_t^(l)  = sqrt(sum_g ss[l][g][t])                        norm of the concatenated heads
 //   s_t      = (1/|L|) sum_l a_t^(l) v_t^(l)                   Eq. 7
 //   A_t      = sum_l a_t^(l)
 //   g_j      = (1/(|L| n_j)) sum_{t in V_j} A_t                Eq. 8
-// A block covers 32 tokens; its 8 warps take every 8th layer (coalesced
-// loads across the 32 tokens of a warp) and combine in a fixed order, so the
-// sums are deterministic.
+// A block covers 32 tokens with one warp per layer slot (layers l, l+32, ...;
+// coalesced loads across the 32 tokens of a warp), then combines the layer
+// slots in a fixed order, so the sums are deterministic.
 #include "internal.cuh"
 
 namespace conduit {
 namespace {
 
-constexpr int kLayerGroups = 8;
+constexpr int kLayerSlots = 32;
 
-__global__ void __launch_bounds__(256) finalize_tokens_kernel(const float* pa, const float* ss,
-                                                              BatchDev b, int n_layers, int Hkv,
-                                                              int Hq, int rg_max, int group_rows,
-                                                              int64_t n_tot, float* s,
-                                                              float* attn_sum, int32_t* status) {
-  __shared__ float part_s[kLayerGroups][32];
-  __shared__ float part_a[kLayerGroups][32];
-  const int lane = threadIdx.x & 31, lg = threadIdx.x >> 5;
+__global__ void __launch_bounds__(1024) finalize_tokens_kernel(const float* pa, const float* ss,
+                                                               BatchDev b, int n_layers, int Hkv,
+                                                               int Hq, int rg_max, int group_rows,
+                                                               int64_t n_tot, float* s,
+                                                               float* attn_sum, int32_t* status) {
+  __shared__ float part_s[kLayerSlots][33];
+  __shared__ float part_a[kLayerSlots][33];
+  const int lane = threadIdx.x & 31, slot = threadIdx.x >> 5;
   const int64_t tg = int64_t(blockIdx.x) * 32 + lane;
   float acc_s = 0.f, acc_a = 0.f;
   if (tg < n_tot) {
@@ -30,23 +30,25 @@ __global__ void __launch_bounds__(256) finalize_tokens_kernel(const float* pa, c
     const float denom = float(nq * Hq);
     const int rows = (Hq / Hkv) * nq;
     const int n_rg = group_rows ? (rows + group_rows - 1) / group_rows : 1;
-    for (int li = lg; li < n_layers; li += kLayerGroups) {
-      float col = 0.f;
-      for (int g = 0; g < Hkv; ++g)
-        for (int rg = 0; rg < n_rg; ++rg) col += pa[((int64_t(li) * Hkv + g) * rg_max + rg) * n_tot + tg];
+    for (int li = slot; li < n_layers; li += kLayerSlots) {
+      float col = 0.f, sq = 0.f;
+      for (int g = 0; g < Hkv; ++g) {
+        const int64_t lg = int64_t(li) * Hkv + g;
+        for (int rg = 0; rg < n_rg; ++rg) col += pa[(lg * rg_max + rg) * n_tot + tg];
+        sq += ss[lg * n_tot + tg];
+      }
       const float a = col / denom;
-      const float vn = sqrtf(ss[int64_t(li) * n_tot + tg]);
-      acc_s = fmaf(a, vn, acc_s);
+      acc_s = fmaf(a, sqrtf(sq), acc_s);
       acc_a += a;
     }
   }
-  part_s[lg][lane] = acc_s;
-  part_a[lg][lane] = acc_a;
+  part_s[slot][lane] = acc_s;
+  part_a[slot][lane] = acc_a;
   __syncthreads();
-  if (lg == 0 && tg < n_tot) {
+  if (slot == 0 && tg < n_tot) {
     float ts = 0.f, ta = 0.f;
-#pragma unroll
-    for (int w = 0; w < kLayerGroups; ++w) {
+    const int used = min(kLayerSlots, n_layers);
+    for (int w = 0; w < used; ++w) {
       ts += part_s[w][lane];
       ta += part_a[w][lane];
     }
@@ -82,7 +84,8 @@ cudaError_t launch_finalize(const float* pa, const float* ss, const BatchDev& b,
                             int Hkv, int Hq, int rg_max, int group_rows, int64_t n_tot, float* s,
                             float* attn_sum, float* g, int32_t* status, cudaStream_t stream) {
   if (n_tot == 0) return cudaSuccess;
-  finalize_tokens_kernel<<<unsigned((n_tot + 31) / 32), 256, 0, stream>>>(
+  const int threads = 32 * std::min(kLayerSlots, n_layers);
+  finalize_tokens_kernel<<<unsigned((n_tot + 31) / 32), threads, 0, stream>>>(
       pa, ss, b, n_layers, Hkv, Hq, rg_max, group_rows, n_tot, s, attn_sum, status);
   cudaError_t err = cudaGetLastError();
   if (err) return err;

@@ -89,8 +89,9 @@ bool score_tc_supported(const KvDev& kv);
 int score_tc_groups(int rows);
 cudaError_t launch_score_tc(const KvDev& kv, const BatchDev& b, const int32_t* q_off_host,
                             const void* q, int32_t q_tot, const LayerList& layers, int rg_max,
-                            float* pa, int32_t* status, cudaStream_t stream);
-// pa is [n_layers][Hkv][rg_max][n_tot]; request r contributes
+                            float* pa, float* ss, int32_t* status, cudaStream_t stream);
+// pa is [n_layers][Hkv][rg_max][n_tot] and ss [n_layers][Hkv][n_tot] (sum of
+// squares of V per KV head); request r contributes
 // ceil(G n_q_r / group_rows) row groups (one when group_rows == 0).
 cudaError_t launch_finalize(const float* pa, const float* ss, const BatchDev& b, int n_layers,
                             int Hkv, int Hq, int rg_max, int group_rows, int64_t n_tot, float* s,

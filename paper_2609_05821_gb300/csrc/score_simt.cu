@@ -194,7 +194,7 @@ __global__ void __launch_bounds__(kThreads) colsum_kernel(KvDev kv, BatchDev b, 
   }
 }
 
-// ss[li][tg] = sum over KV heads g and e of V[l][g][t][e]^2; one warp per token.
+// ss[li][g][tg] = sum over e of V[l][g][t][e]^2 for every KV head g; one warp per token.
 template <typename T>
 __global__ void __launch_bounds__(256) value_sumsq_kernel(KvDev kv, BatchDev b, LayerList layers,
                                                           float* ss) {
@@ -204,23 +204,23 @@ __global__ void __launch_bounds__(256) value_sumsq_kernel(KvDev kv, BatchDev b, 
   const int t = blockIdx.x * 8 + threadIdx.x / 32, lane = threadIdx.x % 32;
   if (t >= N) return;
   const int cpr = kv.d / VEC;            // 16-byte chunks per head row
-  const int chunks = kv.Hkv * cpr;
   const T* vb = static_cast<const T*>(kv.v);
-  float acc = 0.f;
-  for (int c = lane; c < chunks; c += 32) {
-    const int g = c / cpr, e = (c % cpr) * VEC;
-    const int64_t off = kv.row(l, g, r, int64_t(t0) + t, t) + e;
-    const uint4 raw = *reinterpret_cast<const uint4*>(vb + off);
-    const T* vals = reinterpret_cast<const T*>(&raw);
+  for (int g = 0; g < kv.Hkv; ++g) {
+    const int64_t base = kv.row(l, g, r, int64_t(t0) + t, t);
+    float acc = 0.f;
+    for (int c = lane; c < cpr; c += 32) {
+      const uint4 raw = *reinterpret_cast<const uint4*>(vb + base + c * VEC);
+      const T* vals = reinterpret_cast<const T*>(&raw);
 #pragma unroll
-    for (int u = 0; u < VEC; ++u) {
-      const float x = to_float(vals[u]);
-      acc = fmaf(x, x, acc);
+      for (int u = 0; u < VEC; ++u) {
+        const float x = to_float(vals[u]);
+        acc = fmaf(x, x, acc);
+      }
     }
-  }
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-  if (lane == 0) ss[int64_t(li) * kv.n_tot + t0 + t] = acc;
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if (lane == 0) ss[(int64_t(li) * kv.Hkv + g) * kv.n_tot + t0 + t] = acc;
+  }
 }
 
 }  // namespace

@@ -53,6 +53,7 @@ struct TcArgs {
   int32_t rg_max;      // row groups per slab, maximum over requests (pa stride)
   float scale_log2;    // log2(e) / sqrt(d)
   float* pa;           // [n_layers][Hkv][rg_max][n_tot]
+  float* ss;           // [n_layers][Hkv][n_tot] sum of squares of V per KV head
   int32_t* status;
   LayerList layers;
 };
@@ -387,9 +388,21 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (nrb > 1 && 128 + lrow < w.rows) s.lse[128 + lrow] = m1 * a.scale_log2 + log2f(z1);
       epi_barrier();
       float* pa_out = a.pa + ((int64_t(w.li) * a.kv.Hkv + w.g) * a.rg_max + w.rg) * a.kv.n_tot + w.t0;
+      float* ss_out = a.ss + (int64_t(w.li) * a.kv.Hkv + w.g) * a.kv.n_tot + w.t0;
+      const bool do_norm = w.rg == 0;  // one row group of each slab also streams V
       const int nchunk = (w.rows + 31) / 32;
       for (int i = w.tiles; i < 2 * w.tiles; ++i) {  // pass B
         const int slot = tseq & 1;
+        const int tok = tile_of(w, i) * kTile + lrow;
+        // this thread's V row (256 bytes), loaded before the wait to hide its latency
+        uint4 vrow[16];
+        const bool vload = ok && do_norm && tok < w.N;
+        if (vload) {
+          const uint4* src = reinterpret_cast<const uint4*>(
+              static_cast<const __nv_bfloat16*>(a.kv.v) + a.kv.row(w.l, w.g, w.r, int64_t(w.t0) + tok, tok));
+#pragma unroll
+          for (int c = 0; c < 16; ++c) vrow[c] = src[c];
+        }
         // tcgen05.ld is warp-collective: the whole warp goes on or stops
         const bool got = __all_sync(0xffffffffu, ok && wait_or_abort(&s.tfull[slot], (tseq >> 1) & 1, s.abort));
         ++tseq;
@@ -397,6 +410,19 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (ok && !*s.abort) raise_abort(a, s, tc::kSiteMma);
           ok = false;
           continue;
+        }
+        if (vload) {  // sum of squares of the cached value of (layer, KV head, token)
+          float sq[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+          for (int c = 0; c < 16; ++c) {
+            const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&vrow[c]);
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const float2 f = __bfloat1622float2(h[e]);
+              sq[e] = fmaf(f.x, f.x, fmaf(f.y, f.y, sq[e]));
+            }
+          }
+          ss_out[tok] = (sq[0] + sq[1]) + (sq[2] + sq[3]);
         }
         tc::tc_fence_after();
         float ac[4] = {0.f, 0.f, 0.f, 0.f};
@@ -421,7 +447,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float acc = (ac[0] + ac[1]) + (ac[2] + ac[3]);
         tc::tc_fence_before();
         tc::mbar_arrive(&s.tempty[slot]);
-        const int tok = tile_of(w, i) * kTile + lrow;
         if (tok < w.N) pa_out[tok] = acc;
       }
       epi_barrier();  // every thread is done with this unit's rows and lse
@@ -467,7 +492,7 @@ int score_tc_groups(int rows) { return n_groups(rows); }
 
 cudaError_t launch_score_tc(const KvDev& kv, const BatchDev& b, const int32_t* q_off_host,
                             const void* q, int32_t q_tot, const LayerList& layers, int rg_max,
-                            float* pa, int32_t* status, cudaStream_t stream) {
+                            float* pa, float* ss, int32_t* status, cudaStream_t stream) {
   EncodeTiledFn enc = encode_fn();
   if (!enc) return cudaErrorNotSupported;
   CUtensorMap kmap;
@@ -499,6 +524,7 @@ cudaError_t launch_score_tc(const KvDev& kv, const BatchDev& b, const int32_t* q
   a.rg_max = rg_max;
   a.scale_log2 = kLog2e / sqrtf(float(kD));
   a.pa = pa;
+  a.ss = ss;
   a.status = status;
   a.layers = layers;
   if (units == 0) return cudaSuccess;
