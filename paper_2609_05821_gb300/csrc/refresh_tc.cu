@@ -2,25 +2,26 @@
 // (selective recompute, Conduit Sec. 3.1 / 4.3):
 //   out[l][i][h] = sum_{j <= p_i} softmax_j(<q[l][i][h], K'[l][h/G][j]> / sqrt(d)) V'[l][h/G][j]
 //
-// One CTA owns a block of 128 query rows of one (layer, KV head, request):
-// floor(128/G) consecutive selected rows times the G query heads that share
-// the KV head. Keys stream in tiles of 64. Roles (192 threads):
+// One CTA owns up to two query tiles of 128 rows of one (layer, KV head,
+// request); a tile holds floor(128/G) consecutive selected rows times the G
+// query heads that share the KV head, and both tiles share every K/V tile.
+// Keys stream in tiles of 64. Roles (320 threads):
 //   warp 0     one thread issues TMA loads of K and V tiles into two
-//              three-stage rings (K frees after S, V after P.V)
-//   warp 1     one thread issues tcgen05 MMAs: S(t) = Q K(t)^T into one of two
-//              TMEM S buffers (columns [0,64) / [64,128)), and O += P(t) V(t)
-//              into TMEM columns [128,256); S(t+2) is issued right after
-//              P.V(t), so the softmax of tile t+1 overlaps the tensor work
-//   warps 2-5  softmax: stage the query rows, then per tile read S(t) (one
-//              row per thread), apply the causal mask j <= p_i, keep a lazy
-//              running max (O and the row sum are rescaled only when the
-//              max grows by 2^8; the rescale is warp-uniform because
+//              three-stage rings (K frees after both S, V after both P.V)
+//   warp 1     one thread issues tcgen05 MMAs: per query tile, S(t) = Q K(t)^T
+//              into one of two TMEM S buffers and O += P(t) V(t); S(t+2) is
+//              issued right after P.V(t), so softmax overlaps tensor work
+//   warps 2-5, 6-9   softmax of tile 0 and tile 1: stage the query rows, then
+//              per key tile read S(t) (one row per thread), apply the causal
+//              mask j <= p_i, keep a lazy running max (O and the row sum are
+//              rescaled only when the max grows by 2^8; warp-uniform, since
 //              tcgen05.ld/st are warp-collective), write P(t) in bf16 to one
 //              of two shared buffers, and finally write O / rowsum in bf16
-// Rows are sorted by position, so a block needs keys up to its last row's
-// position only. Every wait is bounded by one second; a role that gives up
-// raises an abort flag the others watch, the kernel sets
-// CONDUIT_FLAG_TIMEOUT, drains its copies and MMAs, and frees TMEM.
+// TMEM: tile q uses columns [256q, 256q + 128) for its two S buffers and
+// [256q + 128, 256q + 256) for O. Rows are sorted by position, so a CTA needs
+// keys up to its last row's position only. Every wait is bounded by one
+// second; a role that gives up raises an abort flag the others watch, the
+// kernel sets CONDUIT_FLAG_TIMEOUT, drains its copies and MMAs, frees TMEM.
 #include <cuda.h>
 
 #include "internal.cuh"
@@ -31,17 +32,21 @@ namespace {
 
 constexpr int kD = 128;
 constexpr int kKT = 64;                          // keys per tile
-constexpr int kRows = 128;
-constexpr int kThreads = 192;
+constexpr int kRows = 128;                       // rows per query tile
+constexpr int kTiles = 2;                        // query tiles per CTA
 constexpr int kSoftThreads = 128;
+constexpr int kThreads = 64 + kTiles * kSoftThreads;
 constexpr int kStages = 3;
-constexpr uint32_t kQHalf = kRows * 128;         // 16 KB: one 64-dim half of the query tile
+constexpr uint32_t kQHalf = kRows * 128;         // 16 KB: one 64-dim half of a query tile
+constexpr uint32_t kQBytes = 2 * kQHalf;         // 32 KB
 constexpr uint32_t kTileHalf = kKT * 128;        // 8 KB: one 64-dim half of a K or V tile
 constexpr uint32_t kTileBytes = 2 * kTileHalf;   // 16 KB
 constexpr uint32_t kPBytes = kRows * 128;        // 16 KB: 128 rows x 64 keys
-constexpr uint32_t kSmem = 1024 + 2 * kQHalf + 2 * kStages * kTileBytes + 2 * kPBytes + 256;
-constexpr uint32_t kTmemCols = 256;
-constexpr uint32_t kOCol = 128;
+constexpr uint32_t kSmem =
+    1024 + kTiles * kQBytes + 2 * kStages * kTileBytes + kTiles * 2 * kPBytes + 512;
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kTileCols = 256;              // TMEM columns per query tile
+constexpr uint32_t kOCol = 128;                  // O offset inside a tile's columns
 constexpr float kRescaleLog2 = 8.f;
 
 struct RefArgs {
@@ -52,20 +57,21 @@ struct RefArgs {
   const __nv_bfloat16* q_rows;
   __nv_bfloat16* out;
   int32_t n_sel;
-  int32_t rows_per_block;  // selected rows per CTA, floor(128 / G)
-  int32_t n_blocks;        // CTA blocks per (layer, KV head)
+  int32_t rows_per_tile;   // selected rows per query tile, floor(128 / G)
+  int32_t n_blocks;        // CTAs per (layer, KV head)
   float scale_log2;
   int32_t* status;
 };
 
 struct Smem {
-  uint8_t* q;        // [2 halves][128 rows][128 B]
+  uint8_t* q;        // [kTiles][2 halves][128 rows][128 B]
   uint8_t* k;        // [kStages][2 halves][64 keys][128 B]
   uint8_t* v;        // [kStages][2 halves][64 keys][128 B]
-  uint8_t* p;        // [2][128 rows][128 B]
+  uint8_t* p;        // [kTiles][2][128 rows][128 B]
   uint64_t *kfull, *kempty, *vfull, *vempty;  // [kStages] each
-  uint64_t *sfull, *pfull, *pempty;           // [2] each
-  uint64_t *obar, *qready, *mdone;
+  uint64_t *sfull, *pfull, *pempty;           // [kTiles][2] each
+  uint64_t *obar;                             // [kTiles]
+  uint64_t *qready, *mdone;
   uint32_t* tmem_slot;
   volatile int* abort;
   uint32_t* counters;  // [0] K loads, [1] V loads, [2] K consumed, [3] V consumed
@@ -75,19 +81,19 @@ __device__ __forceinline__ Smem carve(uint8_t* raw) {
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(raw) + 1023) & ~uintptr_t(1023));
   Smem s;
   s.q = base;
-  s.k = s.q + 2 * kQHalf;
+  s.k = s.q + kTiles * kQBytes;
   s.v = s.k + kStages * kTileBytes;
   s.p = s.v + kStages * kTileBytes;
-  uint64_t* bar = reinterpret_cast<uint64_t*>(s.p + 2 * kPBytes);
+  uint64_t* bar = reinterpret_cast<uint64_t*>(s.p + kTiles * 2 * kPBytes);
   s.kfull = bar;
   s.kempty = bar + kStages;
   s.vfull = bar + 2 * kStages;
   s.vempty = bar + 3 * kStages;
   s.sfull = bar + 4 * kStages;
-  s.pfull = s.sfull + 2;
-  s.pempty = s.pfull + 2;
-  s.obar = s.pempty + 2;
-  s.qready = s.obar + 1;
+  s.pfull = s.sfull + 2 * kTiles;
+  s.pempty = s.pfull + 2 * kTiles;
+  s.obar = s.pempty + 2 * kTiles;
+  s.qready = s.obar + kTiles;
   s.mdone = s.qready + 1;
   s.tmem_slot = reinterpret_cast<uint32_t*>(s.mdone + 1);
   s.abort = reinterpret_cast<volatile int*>(s.tmem_slot + 1);
@@ -108,10 +114,6 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, vo
 __device__ __forceinline__ void raise_abort(const RefArgs& a, const Smem& s, int32_t site) {
   if (!*s.abort) flag_status(a.status, CONDUIT_FLAG_TIMEOUT | site);
   *s.abort = 1;
-}
-
-__device__ __forceinline__ void soft_barrier() {
-  asm volatile("bar.sync 1, %0;" ::"n"(kSoftThreads) : "memory");
 }
 
 // TMA of the 64-key tile starting at request-local key j0 (one 64-dim half per box).
@@ -146,16 +148,17 @@ __global__ void __launch_bounds__(kThreads, 1)
   const KvDev& kv = a.kv;
   const int G = kv.G, Hq = kv.Hq;
 
-  // block -> (request, first selected row); larger positions first
+  // CTA -> (request, first selected row, row count); larger positions first
+  const int span = kTiles * a.rows_per_tile;
   int blk = a.n_blocks - 1 - int(blockIdx.x);
   int r = 0, i0 = -1, cnt = 0;
   for (int rr = 0; rr < a.b.R; ++rr) {
     const int k0 = a.idx_off[rr], kr = a.idx_off[rr + 1] - k0;
-    const int nb = (kr + a.rows_per_block - 1) / a.rows_per_block;
+    const int nb = (kr + span - 1) / span;
     if (blk < nb) {
       r = rr;
-      i0 = k0 + blk * a.rows_per_block;
-      cnt = min(a.rows_per_block, kr - blk * a.rows_per_block);
+      i0 = k0 + blk * span;
+      cnt = min(span, kr - blk * span);
       break;
     }
     blk -= nb;
@@ -165,6 +168,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int p_max = min(a.idx[i0 + cnt - 1], N - 1);
   if (p_max < 0) return;
   const int ntiles = p_max / kKT + 1;
+  const int nq = cnt > a.rows_per_tile ? 2 : 1;   // query tiles in use (CTA-uniform)
 
   if (tid == 0) {
     for (int i = 0; i < kStages; ++i) {
@@ -173,13 +177,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::mbar_init(&s.vfull[i], 1);
       tc::mbar_init(&s.vempty[i], 1);
     }
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < 2 * kTiles; ++i) {
       tc::mbar_init(&s.sfull[i], 1);
       tc::mbar_init(&s.pfull[i], kSoftThreads);
       tc::mbar_init(&s.pempty[i], 1);
     }
-    tc::mbar_init(s.obar, 1);
-    tc::mbar_init(s.qready, 1);
+    for (int i = 0; i < kTiles; ++i) tc::mbar_init(&s.obar[i], 1);
+    tc::mbar_init(s.qready, kTiles);
     tc::mbar_init(s.mdone, 1);
     *s.abort = 0;
     for (int i = 0; i < 4; ++i) s.counters[i] = 0;
@@ -210,23 +214,26 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == 1 && lane == 0) {
     // ------------------------------------------------------------------ MMA
     uint32_t ck = 0, cv = 0;
-    const uint32_t q_addr = tc::smem_u32(s.q);
     const uint32_t idesc_s = tc::idesc_bf16(kRows, kKT);
     const uint32_t idesc_o = tc::idesc_bf16(kRows, kD, /*b_mn_major=*/true);
-    auto issue_s = [&](int t) -> bool {  // S(t) = Q K(t)^T into S buffer t & 1
+    auto issue_s = [&](int t) -> bool {  // S(t) of every query tile into its S buffer t & 1
       const int st = t % kStages;
       if (!wait_or_abort(&s.kfull[st], (t / kStages) & 1, s.abort)) return false;
       ++ck;
       tc::tc_fence_after();
       const uint32_t k_addr = tc::smem_u32(s.k + st * kTileBytes);
+      for (int qi = 0; qi < nq; ++qi) {
+        const uint32_t q_addr = tc::smem_u32(s.q + qi * kQBytes);
 #pragma unroll
-      for (int kk = 0; kk < 8; ++kk) {
-        const uint32_t off = (kk & 3) * 32;
-        tc::mma_bf16(tmem + uint32_t(t & 1) * kKT, tc::desc_sw128(q_addr + (kk >> 2) * kQHalf + off),
-                     tc::desc_sw128(k_addr + (kk >> 2) * kTileHalf + off), idesc_s, kk > 0);
+        for (int kk = 0; kk < 8; ++kk) {
+          const uint32_t off = (kk & 3) * 32;
+          tc::mma_bf16(tmem + qi * kTileCols + uint32_t(t & 1) * kKT,
+                       tc::desc_sw128(q_addr + (kk >> 2) * kQHalf + off),
+                       tc::desc_sw128(k_addr + (kk >> 2) * kTileHalf + off), idesc_s, kk > 0);
+        }
+        tc::mma_commit(&s.sfull[qi * 2 + (t & 1)]);
       }
       tc::mma_commit(&s.kempty[st]);
-      tc::mma_commit(&s.sfull[t & 1]);
       return true;
     };
     bool ok = wait_or_abort(s.qready, 0, s.abort);
@@ -234,20 +241,23 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (ok && ntiles > 1) ok = issue_s(1);
     for (int t = 0; t < ntiles && ok; ++t) {
       const int b = t & 1, st = t % kStages;
-      if (!wait_or_abort(&s.pfull[b], (t >> 1) & 1, s.abort)) { ok = false; break; }
       if (!wait_or_abort(&s.vfull[st], (t / kStages) & 1, s.abort)) { ok = false; break; }
       ++cv;
-      tc::tc_fence_after();
-      const uint32_t p_addr = tc::smem_u32(s.p + b * kPBytes);
       const uint32_t v_addr = tc::smem_u32(s.v + st * kTileBytes);
+      for (int qi = 0; qi < nq && ok; ++qi) {
+        if (!wait_or_abort(&s.pfull[qi * 2 + b], (t >> 1) & 1, s.abort)) { ok = false; break; }
+        tc::tc_fence_after();
+        const uint32_t p_addr = tc::smem_u32(s.p + (qi * 2 + b) * kPBytes);
 #pragma unroll
-      for (int kk = 0; kk < kKT / 16; ++kk) {
-        tc::mma_bf16(tmem + kOCol, tc::desc_sw128(p_addr + kk * 32),
-                     tc::desc_sw128_mn(v_addr + kk * 2048, kTileHalf), idesc_o, t > 0 || kk > 0);
+        for (int kk = 0; kk < kKT / 16; ++kk) {
+          tc::mma_bf16(tmem + qi * kTileCols + kOCol, tc::desc_sw128(p_addr + kk * 32),
+                       tc::desc_sw128_mn(v_addr + kk * 2048, kTileHalf), idesc_o, t > 0 || kk > 0);
+        }
+        tc::mma_commit(&s.pempty[qi * 2 + b]);
+        tc::mma_commit(&s.obar[qi]);
       }
+      if (!ok) break;
       tc::mma_commit(&s.vempty[st]);
-      tc::mma_commit(&s.pempty[b]);
-      tc::mma_commit(s.obar);
       if (t + 2 < ntiles && !issue_s(t + 2)) { ok = false; break; }
     }
     if (!ok) raise_abort(a, s, tc::kSiteMma);
@@ -257,45 +267,52 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc::mbar_wait(s.mdone, 0);
   } else if (warp >= 2) {
     // -------------------------------------------------------------- softmax
-    const int et = tid - 64;
+    const int qi = (warp - 2) >> 2;                      // query tile of this warp
+    const int et = tid - 64 - qi * kSoftThreads;         // 0..127 within the tile
     const int quarter = warp & 3;
     const int row = quarter * 32 + lane;                 // TMEM lane = query row of the tile
     const uint32_t lane_base = uint32_t(quarter * 32) << 16;
-    const bool row_ok = row < cnt * G;
-    const int i_row = i0 + (row_ok ? row / G : 0);
+    const uint32_t tcol = qi * kTileCols;
+    const int ti0 = i0 + qi * a.rows_per_tile;           // first selected row of the tile
+    const int tcnt = max(0, min(a.rows_per_tile, cnt - qi * a.rows_per_tile));
+    const bool active = qi < nq;
+    const bool row_ok = row < tcnt * G;
+    const int i_row = ti0 + (row_ok ? row / G : 0);
     const int h_row = g * G + (row_ok ? row % G : 0);
     int p_row = row_ok ? a.idx[i_row] : -1;
     if (p_row >= N) p_row = -1;
-    // query tile: row ρ = (i0 + ρ / G, head g*G + ρ % G), zero beyond cnt * G
-    for (int base = 0; base < kRows * 16; base += kSoftThreads * 8) {
-      uint4 val[8];
+    uint8_t* q_s = s.q + qi * kQBytes;
+    if (active) {  // query tile: row = (ti0 + row / G, head g*G + row % G), zero beyond tcnt * G
+      for (int base = 0; base < kRows * 16; base += kSoftThreads * 8) {
+        uint4 val[8];
 #pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const int x = base + u * kSoftThreads + et;
-        const int rr = x >> 4, ch = x & 15;
-        val[u] = make_uint4(0u, 0u, 0u, 0u);
-        if (rr < cnt * G) {
-          const int ii = i0 + rr / G, hh = g * G + rr % G;
-          val[u] = *reinterpret_cast<const uint4*>(a.q_rows + ((int64_t(l) * a.n_sel + ii) * Hq + hh) * kD + ch * 8);
+        for (int u = 0; u < 8; ++u) {
+          const int x = base + u * kSoftThreads + et;
+          const int rr = x >> 4, ch = x & 15;
+          val[u] = make_uint4(0u, 0u, 0u, 0u);
+          if (rr < tcnt * G) {
+            const int ii = ti0 + rr / G, hh = g * G + rr % G;
+            val[u] = *reinterpret_cast<const uint4*>(a.q_rows + ((int64_t(l) * a.n_sel + ii) * Hq + hh) * kD + ch * 8);
+          }
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const int x = base + u * kSoftThreads + et;
+          const int rr = x >> 4, ch = x & 15;
+          *reinterpret_cast<uint4*>(q_s + (ch >> 3) * kQHalf + tc::sw128_offset(rr, ch & 7)) = val[u];
         }
       }
-#pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const int x = base + u * kSoftThreads + et;
-        const int rr = x >> 4, ch = x & 15;
-        *reinterpret_cast<uint4*>(s.q + (ch >> 3) * kQHalf + tc::sw128_offset(rr, ch & 7)) = val[u];
-      }
+      tc::fence_proxy_async_smem();
     }
-    tc::fence_proxy_async_smem();
-    soft_barrier();
+    asm volatile("bar.sync %0, %1;" ::"r"(1 + qi), "n"(kSoftThreads) : "memory");
     if (et == 0) tc::mbar_arrive(s.qready);
 
-    bool ok = true;
+    bool ok = active;
     float m_ref = -INFINITY, lsum = 0.f;
-    for (int t = 0; t < ntiles; ++t) {
+    for (int t = 0; t < ntiles && active; ++t) {
       const int b = t & 1;
       // the tcgen05.ld below is warp-collective: the whole warp goes on or stops
-      const bool got = __all_sync(0xffffffffu, ok && wait_or_abort(&s.sfull[b], (t >> 1) & 1, s.abort));
+      const bool got = __all_sync(0xffffffffu, ok && wait_or_abort(&s.sfull[qi * 2 + b], (t >> 1) & 1, s.abort));
       if (!got) {
         if (ok) raise_abort(a, s, tc::kSiteMma);
         ok = false;
@@ -303,8 +320,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       tc::tc_fence_after();
       float sv[2][32];
-      tc::tmem_ld32(tmem + lane_base + uint32_t(b) * kKT, sv[0]);
-      tc::tmem_ld32(tmem + lane_base + uint32_t(b) * kKT + 32, sv[1]);
+      tc::tmem_ld32(tmem + lane_base + tcol + uint32_t(b) * kKT, sv[0]);
+      tc::tmem_ld32(tmem + lane_base + tcol + uint32_t(b) * kKT + 32, sv[1]);
       const int j0 = t * kKT;
       float tm[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
       if (j0 + kKT - 1 <= p_row) {  // the whole tile is visible to this row
@@ -332,7 +349,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // P.V(t-1) must be complete before this warp rescales its rows of O.
         // S(t) was issued after P.V(t-2), so obar is at most one phase behind
         // here and its parity cannot alias.
-        if (!__all_sync(0xffffffffu, wait_or_abort(s.obar, (t - 1) & 1, s.abort))) {
+        if (!__all_sync(0xffffffffu, wait_or_abort(&s.obar[qi], (t - 1) & 1, s.abort))) {
           raise_abort(a, s, tc::kSiteMma);
           ok = false;
           continue;
@@ -340,10 +357,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc::tc_fence_after();
         for (int c = 0; c < kD; c += 32) {
           float o[32];
-          tc::tmem_ld32(tmem + lane_base + kOCol + c, o);
+          tc::tmem_ld32(tmem + lane_base + tcol + kOCol + c, o);
 #pragma unroll
           for (int i = 0; i < 32; ++i) o[i] *= alpha;
-          tc::tmem_st32(tmem + lane_base + kOCol + c, o);
+          tc::tmem_st32(tmem + lane_base + tcol + kOCol + c, o);
         }
       }
       if (need) {
@@ -351,12 +368,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         m_ref = tmax;
       }
       // the P buffer of tile t was last read by P.V(t-2)
-      if (!wait_or_abort(&s.pempty[b], ((t >> 1) & 1) ^ 1, s.abort)) {
+      if (!wait_or_abort(&s.pempty[qi * 2 + b], ((t >> 1) & 1) ^ 1, s.abort)) {
         raise_abort(a, s, tc::kSiteMma);
         ok = false;
         continue;
       }
-      uint8_t* pb = s.p + b * kPBytes;
+      uint8_t* pb = s.p + (qi * 2 + b) * kPBytes;
       float ls[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
       for (int h2 = 0; h2 < 2; ++h2) {
@@ -378,33 +395,35 @@ __global__ void __launch_bounds__(kThreads, 1)
       lsum += (ls[0] + ls[1]) + (ls[2] + ls[3]);
       tc::fence_proxy_async_smem();
       tc::tc_fence_before();
-      tc::mbar_arrive(&s.pfull[b]);
+      tc::mbar_arrive(&s.pfull[qi * 2 + b]);
     }
-    // O is complete once the MMA thread's final commit arrives. (The obar phase
-    // of the last P.V could alias: after this warp's last tile only P.V up to
-    // ntiles-3 is known to be done, two phases behind.)
-    if (ok && !wait_or_abort(s.mdone, 0, s.abort)) {
-      raise_abort(a, s, tc::kSiteFinal);
-      ok = false;
-    }
-    const bool all_ok = !__any_sync(0xffffffffu, !ok);
-    if (all_ok) {
-      tc::tc_fence_after();
-      const float inv = lsum > 0.f ? 1.f / lsum : 0.f;
-      __nv_bfloat16* dst = a.out + ((int64_t(l) * a.n_sel + i_row) * Hq + h_row) * kD;
-      for (int c = 0; c < kD; c += 32) {
-        float o[32];
-        tc::tmem_ld32(tmem + lane_base + kOCol + c, o);
-        if (row_ok && p_row >= 0) {
+    if (active) {
+      // O is complete once the MMA thread's final commit arrives. (The obar
+      // phase of the last P.V could alias: after this warp's last tile only
+      // P.V up to ntiles-3 is known to be done, two phases behind.)
+      if (ok && !wait_or_abort(s.mdone, 0, s.abort)) {
+        raise_abort(a, s, tc::kSiteFinal);
+        ok = false;
+      }
+      const bool all_ok = !__any_sync(0xffffffffu, !ok);
+      if (all_ok) {
+        tc::tc_fence_after();
+        const float inv = lsum > 0.f ? 1.f / lsum : 0.f;
+        __nv_bfloat16* dst = a.out + ((int64_t(l) * a.n_sel + i_row) * Hq + h_row) * kD;
+        for (int c = 0; c < kD; c += 32) {
+          float o[32];
+          tc::tmem_ld32(tmem + lane_base + tcol + kOCol + c, o);
+          if (row_ok && p_row >= 0) {
 #pragma unroll
-          for (int u = 0; u < 4; ++u) {
-            uint32_t w4[4];
+            for (int u = 0; u < 4; ++u) {
+              uint32_t w4[4];
 #pragma unroll
-            for (int k2 = 0; k2 < 4; ++k2) {
-              __nv_bfloat162 pr = __floats2bfloat162_rn(o[u * 8 + 2 * k2] * inv, o[u * 8 + 2 * k2 + 1] * inv);
-              w4[k2] = *reinterpret_cast<uint32_t*>(&pr);
+              for (int k2 = 0; k2 < 4; ++k2) {
+                __nv_bfloat162 pr = __floats2bfloat162_rn(o[u * 8 + 2 * k2] * inv, o[u * 8 + 2 * k2 + 1] * inv);
+                w4[k2] = *reinterpret_cast<uint32_t*>(&pr);
+              }
+              *reinterpret_cast<uint4*>(dst + c + u * 8) = make_uint4(w4[0], w4[1], w4[2], w4[3]);
             }
-            *reinterpret_cast<uint4*>(dst + c + u * 8) = make_uint4(w4[0], w4[1], w4[2], w4[3]);
           }
         }
       }
@@ -481,11 +500,11 @@ cudaError_t launch_refresh_tc(const KvDev& kv, const BatchDev& b, const int32_t*
   a.q_rows = static_cast<const __nv_bfloat16*>(q_rows);
   a.out = static_cast<__nv_bfloat16*>(out);
   a.n_sel = n_sel;
-  a.rows_per_block = kRows / kv.G;
+  a.rows_per_tile = kRows / kv.G;
   int blocks = 0;
   for (int r = 0; r < b.R; ++r) {
     const int kr = idx_off_host[r + 1] - idx_off_host[r];
-    blocks += (kr + a.rows_per_block - 1) / a.rows_per_block;
+    blocks += (kr + kTiles * a.rows_per_tile - 1) / (kTiles * a.rows_per_tile);
   }
   a.n_blocks = blocks;
   a.scale_log2 = kLog2e / sqrtf(float(kD));
