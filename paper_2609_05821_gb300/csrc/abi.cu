@@ -147,6 +147,7 @@ struct ScoreLayout {
   bool tc;     // tensor-core kernel (bf16, head_dim 128) or the CUDA-core ones
   int rg_max;  // row groups per slab (column-sum partials per KV head)
   int group_rows;
+  int parts;   // partials per row group and per value norm (2 for the tensor-core kernel)
   size_t stats, pa, ss, attn, total;
 };
 
@@ -157,6 +158,7 @@ ScoreLayout score_layout(const conduit_kv* kv, const conduit_batch* b, int n_lay
   ScoreLayout s{};
   s.tc = score_tc_supported(make_kv(kv, b));
   s.rg_max = 1;
+  s.parts = s.tc ? 2 : 1;
   if (s.tc) {
     s.group_rows = kScoreGroupRows;
     const int G = kv->num_q_heads / kv->num_kv_heads;
@@ -168,9 +170,9 @@ ScoreLayout score_layout(const conduit_kv* kv, const conduit_batch* b, int n_lay
   s.stats = off;
   if (!s.tc) off += align_up(size_t(total_rows) * sizeof(float2));  // (max, sum) per row
   s.pa = off;
-  off += align_up(size_t(n_layers) * kv->num_kv_heads * s.rg_max * n_tot * sizeof(float));
+  off += align_up(size_t(n_layers) * kv->num_kv_heads * s.rg_max * s.parts * n_tot * sizeof(float));
   s.ss = off;
-  off += align_up(size_t(n_layers) * kv->num_kv_heads * n_tot * sizeof(float));
+  off += align_up(size_t(n_layers) * kv->num_kv_heads * s.parts * n_tot * sizeof(float));
   s.attn = off;
   off += align_up(n_tot * sizeof(float));
   s.total = off;
@@ -276,7 +278,7 @@ conduit_status conduit_score(const conduit_kv* kv, const conduit_batch* batch, c
     err = launch_score_simt(kd, bd, q, batch->q_off[R], ll, max_rows, max_tok, stats, pa, cs);
   }
   if (err) return cuda_fail(err, "score");
-  if ((err = launch_finalize(pa, ss, bd, ll.n, kd.Hkv, kd.Hq, lay.rg_max, lay.group_rows, kd.n_tot,
+  if ((err = launch_finalize(pa, ss, bd, ll.n, kd.Hkv, kd.Hq, lay.rg_max, lay.group_rows, lay.parts, kd.n_tot,
                              s, attn, g, status, cs)))
     return cuda_fail(err, "finalize");
   return CONDUIT_OK;

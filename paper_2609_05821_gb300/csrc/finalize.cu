@@ -1,6 +1,6 @@
 // Per-token and per-image reductions of the scoring pass (Conduit Eqs. 6-8).
-//   a_t^(l)  = sum_g sum_group pa[l][g][group][t] / (|Q| Hq)   Eq. 6 (head/query mean)
-//   v_t^(l)  = sqrt(sum_g ss[l][g][t])                        norm of the concatenated heads
+//   a_t^(l)  = sum_g sum_group,part pa[l][g][group][part][t] / (|Q| Hq)   Eq. 6 (head/query mean)
+//   v_t^(l)  = sqrt(sum_g,part ss[l][g][part][t])                     norm of the concatenated heads
 //   s_t      = (1/|L|) sum_l a_t^(l) v_t^(l)                   Eq. 7
 //   A_t      = sum_l a_t^(l)
 //   g_j      = (1/(|L| n_j)) sum_{t in V_j} A_t                Eq. 8
@@ -17,7 +17,7 @@ constexpr int kLayerSlots = 32;
 __global__ void __launch_bounds__(1024) finalize_tokens_kernel(const float* pa, const float* ss,
                                                                BatchDev b, int n_layers, int Hkv,
                                                                int Hq, int rg_max, int group_rows,
-                                                               int64_t n_tot, float* s,
+                                                               int parts, int64_t n_tot, float* s,
                                                                float* attn_sum, int32_t* status) {
   __shared__ float part_s[kLayerSlots][33];
   __shared__ float part_a[kLayerSlots][33];
@@ -29,13 +29,13 @@ __global__ void __launch_bounds__(1024) finalize_tokens_kernel(const float* pa, 
     const int nq = b.q_off[r + 1] - b.q_off[r];
     const float denom = float(nq * Hq);
     const int rows = (Hq / Hkv) * nq;
-    const int n_rg = group_rows ? (rows + group_rows - 1) / group_rows : 1;
+    const int n_sl = (group_rows ? (rows + group_rows - 1) / group_rows : 1) * parts;
     for (int li = slot; li < n_layers; li += kLayerSlots) {
       float col = 0.f, sq = 0.f;
       for (int g = 0; g < Hkv; ++g) {
         const int64_t lg = int64_t(li) * Hkv + g;
-        for (int rg = 0; rg < n_rg; ++rg) col += pa[(lg * rg_max + rg) * n_tot + tg];
-        sq += ss[lg * n_tot + tg];
+        for (int sl = 0; sl < n_sl; ++sl) col += pa[(lg * rg_max * parts + sl) * n_tot + tg];
+        for (int p = 0; p < parts; ++p) sq += ss[(lg * parts + p) * n_tot + tg];
       }
       const float a = col / denom;
       acc_s = fmaf(a, sqrtf(sq), acc_s);
@@ -81,12 +81,12 @@ __global__ void __launch_bounds__(256) image_means_kernel(const float* attn_sum,
 }  // namespace
 
 cudaError_t launch_finalize(const float* pa, const float* ss, const BatchDev& b, int n_layers,
-                            int Hkv, int Hq, int rg_max, int group_rows, int64_t n_tot, float* s,
+                            int Hkv, int Hq, int rg_max, int group_rows, int parts, int64_t n_tot, float* s,
                             float* attn_sum, float* g, int32_t* status, cudaStream_t stream) {
   if (n_tot == 0) return cudaSuccess;
   const int threads = 32 * std::min(kLayerSlots, n_layers);
   finalize_tokens_kernel<<<unsigned((n_tot + 31) / 32), threads, 0, stream>>>(
-      pa, ss, b, n_layers, Hkv, Hq, rg_max, group_rows, n_tot, s, attn_sum, status);
+      pa, ss, b, n_layers, Hkv, Hq, rg_max, group_rows, parts, n_tot, s, attn_sum, status);
   cudaError_t err = cudaGetLastError();
   if (err) return err;
   image_means_kernel<<<b.K, 256, 0, stream>>>(attn_sum, b, n_layers, g);

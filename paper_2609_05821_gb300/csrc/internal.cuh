@@ -83,18 +83,19 @@ cudaError_t launch_score_simt(const KvDev& kv, const BatchDev& b, const void* q,
                               const LayerList& layers, int max_rows, int max_tokens,
                               float2* stats, float* pa, cudaStream_t stream);
 // Tensor-core scoring (bf16, head_dim 128): one kernel, row statistics then
-// column sums per (slab, group of at most 256 scoring rows).
+// column sums per (slab, group of at most 256 scoring rows); it writes two
+// partials per row group into pa and two half-row partials into ss.
 constexpr int kScoreGroupRows = 256;
 bool score_tc_supported(const KvDev& kv);
 int score_tc_groups(int rows);
 cudaError_t launch_score_tc(const KvDev& kv, const BatchDev& b, const int32_t* q_off_host,
                             const void* q, int32_t q_tot, const LayerList& layers, int rg_max,
                             float* pa, float* ss, int32_t* status, cudaStream_t stream);
-// pa is [n_layers][Hkv][rg_max][n_tot] and ss [n_layers][Hkv][n_tot] (sum of
-// squares of V per KV head); request r contributes
+// pa is [n_layers][Hkv][rg_max][parts][n_tot] and ss [n_layers][Hkv][parts][n_tot]
+// (partial sums of squares of V per KV head); request r contributes
 // ceil(G n_q_r / group_rows) row groups (one when group_rows == 0).
 cudaError_t launch_finalize(const float* pa, const float* ss, const BatchDev& b, int n_layers,
-                            int Hkv, int Hq, int rg_max, int group_rows, int64_t n_tot, float* s,
+                            int Hkv, int Hq, int rg_max, int group_rows, int parts, int64_t n_tot, float* s,
                             float* attn_sum, float* g, int32_t* status, cudaStream_t stream);
 cudaError_t launch_select(const BatchDev& b, const float* s, const float* g, float lambda,
                           const int32_t* idx_off_dev, int32_t* idx, uint8_t* mask, float* s_hat,

@@ -6,20 +6,25 @@
 // Each unit makes two passes over the request's N_r keys:
 //
 //   pass A   D[rows x 128 tokens] = Q_rows . K_tile^T     (rows are the MMA M)
-//            each epilogue thread owns one row: running max m and sum
-//            z = sum 2^((S - m) log2(e)/sqrt(d)) -> lse = m log2(e)/sqrt(d) + log2 z
+//            each epilogue thread owns one row and a share of the columns:
+//            running max m and sum z = sum 2^((S - m) log2(e)/sqrt(d)), merged
+//            into lse = m log2(e)/sqrt(d) + log2 z; the same threads also
+//            stream the tile's V rows for the value norms (ss)
 //   pass B   D[128 tokens x rows] = K_tile . Q_rows^T     (tokens are the MMA M)
-//            each epilogue thread owns one token: sum over rows of 2^(x - lse)
-//            -> pa[l][g][group][t], this group's share of sum_q sum_h alpha
+//            each epilogue thread owns one token and half of the rows: sum of
+//            2^(x - lse) -> pa[l][g][group][half][t], this share of
+//            sum_q sum_h alpha
 //
 // Pass B walks the tiles in reverse so the most recent K tiles of pass A are
-// still in L2. Roles (192 threads):
+// still in L2. Roles (320 threads):
 //   warp 0       one thread issues TMA loads of K tiles (128 tokens x 128
 //                dims, 128-byte swizzle) into a four-stage ring
 //   warp 1       one thread issues tcgen05 MMAs into two 256-column TMEM
 //                accumulator slots (it also owns the TMEM allocation)
-//   warps 2-5    epilogue: stage the unit's scoring rows in shared memory
-//                (same swizzle), then read accumulators with tcgen05.ld
+//   warps 2-9    epilogue, two warps per TMEM lane quarter (warp group h
+//                = 0, 1 splits each tile's columns, or takes row block h):
+//                stage the unit's scoring rows in shared memory (same
+//                swizzle), then read accumulators with tcgen05.ld
 // The roles meet on mbarriers (ring full / empty, accumulator full / empty,
 // rows ready). Every wait is bounded by one second; a role that gives up
 // raises an abort flag the others also watch, the kernel sets
@@ -36,13 +41,13 @@ constexpr int kD = 128;
 constexpr int kTile = 128;
 constexpr int kStages = 4;
 constexpr int kGroupRows = 256;
-constexpr int kThreads = 192;
-constexpr int kEpiThreads = 128;
+constexpr int kThreads = 320;
+constexpr int kEpiThreads = 256;
 constexpr uint32_t kHalfQ = kGroupRows * 128;  // 32 KB: one 64-dim half of the row tile
 constexpr uint32_t kHalfK = kTile * 128;       // 16 KB
 constexpr uint32_t kStageBytes = 2 * kHalfK;   // 32 KB per K tile
 constexpr uint32_t kSlotCols = 256;
-constexpr uint32_t kSmemBytes = 1024 + 2 * kHalfQ + kStages * kStageBytes + 256 + kGroupRows * 4;
+constexpr uint32_t kSmemBytes = 1024 + 2 * kHalfQ + kStages * kStageBytes + 256 + kGroupRows * 4 + 128 * 8;
 
 struct TcArgs {
   KvDev kv;
@@ -52,8 +57,8 @@ struct TcArgs {
   int32_t n_units;
   int32_t rg_max;      // row groups per slab, maximum over requests (pa stride)
   float scale_log2;    // log2(e) / sqrt(d)
-  float* pa;           // [n_layers][Hkv][rg_max][n_tot]
-  float* ss;           // [n_layers][Hkv][n_tot] sum of squares of V per KV head
+  float* pa;           // [n_layers][Hkv][rg_max][2][n_tot]
+  float* ss;           // [n_layers][Hkv][2][n_tot] sum of squares of V, per half of the head
   int32_t* status;
   LayerList layers;
 };
@@ -119,6 +124,7 @@ struct Smem {
   volatile int* abort;
   uint32_t* counters;  // [0] loads issued, [1] loads consumed
   float* lse;          // [256]
+  float2* part;        // [128] (m, z) of the second column half
 };
 
 __device__ __forceinline__ Smem carve(uint8_t* raw) {
@@ -137,6 +143,7 @@ __device__ __forceinline__ Smem carve(uint8_t* raw) {
   s.abort = reinterpret_cast<volatile int*>(s.tmem_slot + 1);
   s.counters = reinterpret_cast<uint32_t*>(s.tmem_slot + 2);
   s.lse = reinterpret_cast<float*>(tail + 256);
+  s.part = reinterpret_cast<float2*>(tail + 256 + kGroupRows * 4);
   return s;
 }
 
@@ -325,10 +332,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------------------ epilogue
     // After an abort the epilogue keeps walking its units (skipping the work)
     // so that every thread reaches every named barrier.
-    const int et = tid - 64;                       // 0..127
+    const int et = tid - 64;                       // 0..255
+    const int h = et >> 7;                         // warp group: column half or row block
     const int quarter = warp & 3;                  // TMEM lanes 32*quarter .. +31
     const int lrow = quarter * 32 + lane;          // row (pass A) / token (pass B) in the tile
     const uint32_t lane_base = uint32_t(quarter * 32) << 16;
+    const int64_t n_tot = a.kv.n_tot;
     uint32_t tseq = 0;
     bool ok = true;
     for (int u = blockIdx.x; u < a.n_units; u += gridDim.x) {
@@ -339,9 +348,26 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::fence_proxy_async_smem();
       epi_barrier();
       if (et == 0) tc::mbar_arrive(s.qready);
-      float m0 = -INFINITY, z0 = 0.f, m1 = -INFINITY, z1 = 0.f;
+      // pass A share: row block rb, 32-column chunks [cc0, cc0 + ncc)
+      const int rb = nrb == 2 ? h : 0;
+      const int cc0 = nrb == 2 ? 0 : 2 * h;
+      const int ncc = nrb == 2 ? 4 : 2;
+      const bool do_norm = w.rg == 0;  // one row group of each slab also streams V
+      const int64_t lg = int64_t(w.li) * a.kv.Hkv + w.g;
+      float* ss_out = a.ss + (lg * 2 + h) * n_tot + w.t0;
+      float m = -INFINITY, z = 0.f;
       for (int i = 0; i < w.tiles; ++i) {            // pass A
         const int slot = tseq & 1;
+        // half (64 dims) of this thread's V row, loaded before the wait to hide its latency
+        const int tok_v = i * kTile + lrow;
+        uint4 vrow[8];
+        const bool vload = ok && do_norm && tok_v < w.N;
+        if (vload) {
+          const uint4* src = reinterpret_cast<const uint4*>(
+              static_cast<const __nv_bfloat16*>(a.kv.v) + a.kv.row(w.l, w.g, w.r, int64_t(w.t0) + tok_v, tok_v) + h * 64);
+#pragma unroll
+          for (int c = 0; c < 8; ++c) vrow[c] = src[c];
+        }
         // tcgen05.ld is warp-collective: the whole warp goes on or stops
         const bool got = __all_sync(0xffffffffu, ok && wait_or_abort(&s.tfull[slot], (tseq >> 1) & 1, s.abort));
         ++tseq;
@@ -352,57 +378,68 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tc::tc_fence_after();
         const int tok0 = i * kTile;
-        for (int rb = 0; rb < nrb; ++rb) {
-          float mr = rb == 0 ? m0 : m1, zr = rb == 0 ? z0 : z1;
 #pragma unroll 1
-          for (int cc = 0; cc < 4; ++cc) {
-            float v[32];
-            tc::tmem_ld32(tmem + lane_base + uint32_t(slot) * kSlotCols + rb * 128 + cc * 32, v);
-            const int tok = tok0 + cc * 32;
-            if (tok + 32 > w.N) {  // ragged last tile only
+        for (int cc = cc0; cc < cc0 + ncc; ++cc) {
+          float v[32];
+          tc::tmem_ld32(tmem + lane_base + uint32_t(slot) * kSlotCols + rb * 128 + cc * 32, v);
+          const int tok = tok0 + cc * 32;
+          if (tok + 32 > w.N) {  // ragged last tile only
 #pragma unroll
-              for (int x = 0; x < 32; ++x)
-                if (tok + x >= w.N) v[x] = -INFINITY;
-            }
-            float cm[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-#pragma unroll
-            for (int x = 0; x < 32; ++x) cm[x & 3] = fmaxf(cm[x & 3], v[x]);
-            const float cmax = fmaxf(fmaxf(cm[0], cm[1]), fmaxf(cm[2], cm[3]));
-            const float mn = fmaxf(mr, cmax);
-            if (mn != -INFINITY) {
-              const float nb = -mn * a.scale_log2;
-              float ac[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-              for (int x = 0; x < 32; ++x) ac[x & 3] += tc::ex2(fmaf(v[x], a.scale_log2, nb));
-              zr = zr * exp2f((mr - mn) * a.scale_log2) + ((ac[0] + ac[1]) + (ac[2] + ac[3]));
-              mr = mn;
-            }
+            for (int x = 0; x < 32; ++x)
+              if (tok + x >= w.N) v[x] = -INFINITY;
           }
-          if (rb == 0) { m0 = mr; z0 = zr; } else { m1 = mr; z1 = zr; }
+          float cm[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+          for (int x = 0; x < 32; ++x) cm[x & 3] = fmaxf(cm[x & 3], v[x]);
+          const float cmax = fmaxf(fmaxf(cm[0], cm[1]), fmaxf(cm[2], cm[3]));
+          const float mn = fmaxf(m, cmax);
+          if (mn != -INFINITY) {
+            const float nb = -mn * a.scale_log2;
+            float ac[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+            for (int x = 0; x < 32; ++x) ac[x & 3] += tc::ex2(fmaf(v[x], a.scale_log2, nb));
+            z = z * exp2f((m - mn) * a.scale_log2) + ((ac[0] + ac[1]) + (ac[2] + ac[3]));
+            m = mn;
+          }
         }
         tc::tc_fence_before();
         tc::mbar_arrive(&s.tempty[slot]);
+        if (vload) {  // sum of squares of this half of the cached value row
+          float sq[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+          for (int c = 0; c < 8; ++c) {
+            const __nv_bfloat162* hv = reinterpret_cast<const __nv_bfloat162*>(&vrow[c]);
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const float2 f = __bfloat1622float2(hv[e]);
+              sq[e] = fmaf(f.x, f.x, fmaf(f.y, f.y, sq[e]));
+            }
+          }
+          ss_out[tok_v] = (sq[0] + sq[1]) + (sq[2] + sq[3]);
+        }
       }
-      // log2-sum-exp of this thread's rows, shared with the token-owning threads of pass B
-      if (lrow < w.rows) s.lse[lrow] = m0 * a.scale_log2 + log2f(z0);
-      if (nrb > 1 && 128 + lrow < w.rows) s.lse[128 + lrow] = m1 * a.scale_log2 + log2f(z1);
+      // log2-sum-exp of each row, shared with the token-owning threads of pass B
+      if (nrb == 1 && h == 1) s.part[lrow] = make_float2(m, z);
       epi_barrier();
-      float* pa_out = a.pa + ((int64_t(w.li) * a.kv.Hkv + w.g) * a.rg_max + w.rg) * a.kv.n_tot + w.t0;
-      float* ss_out = a.ss + (int64_t(w.li) * a.kv.Hkv + w.g) * a.kv.n_tot + w.t0;
-      const bool do_norm = w.rg == 0;  // one row group of each slab also streams V
+      if (nrb == 2) {
+        s.lse[h * 128 + lrow] = m * a.scale_log2 + log2f(z);
+      } else if (h == 0) {
+        const float2 o = s.part[lrow];
+        const float mm = fmaxf(m, o.x);
+        float zz = 0.f;
+        if (m != -INFINITY) zz += z * exp2f((m - mm) * a.scale_log2);
+        if (o.x != -INFINITY) zz += o.y * exp2f((o.x - mm) * a.scale_log2);
+        s.lse[lrow] = mm * a.scale_log2 + log2f(zz);
+      }
+      epi_barrier();
+      // pass B share: 32-row chunks [cb0, cb1)
       const int nchunk = (w.rows + 31) / 32;
+      const int hc = (nchunk + 1) / 2;
+      const int cb0 = h * hc, cb1 = min(nchunk, cb0 + hc);
+      float* pa_out = a.pa + ((lg * a.rg_max + w.rg) * 2 + h) * n_tot + w.t0;
       for (int i = w.tiles; i < 2 * w.tiles; ++i) {  // pass B
         const int slot = tseq & 1;
         const int tok = tile_of(w, i) * kTile + lrow;
-        // this thread's V row (256 bytes), loaded before the wait to hide its latency
-        uint4 vrow[16];
-        const bool vload = ok && do_norm && tok < w.N;
-        if (vload) {
-          const uint4* src = reinterpret_cast<const uint4*>(
-              static_cast<const __nv_bfloat16*>(a.kv.v) + a.kv.row(w.l, w.g, w.r, int64_t(w.t0) + tok, tok));
-#pragma unroll
-          for (int c = 0; c < 16; ++c) vrow[c] = src[c];
-        }
         // tcgen05.ld is warp-collective: the whole warp goes on or stops
         const bool got = __all_sync(0xffffffffu, ok && wait_or_abort(&s.tfull[slot], (tseq >> 1) & 1, s.abort));
         ++tseq;
@@ -411,22 +448,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           ok = false;
           continue;
         }
-        if (vload) {  // sum of squares of the cached value of (layer, KV head, token)
-          float sq[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-          for (int c = 0; c < 16; ++c) {
-            const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&vrow[c]);
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const float2 f = __bfloat1622float2(h[e]);
-              sq[e] = fmaf(f.x, f.x, fmaf(f.y, f.y, sq[e]));
-            }
-          }
-          ss_out[tok] = (sq[0] + sq[1]) + (sq[2] + sq[3]);
-        }
         tc::tc_fence_after();
         float ac[4] = {0.f, 0.f, 0.f, 0.f};
-        for (int cc = 0; cc < nchunk; ++cc) {
+        for (int cc = cb0; cc < cb1; ++cc) {
           float v[32];
           tc::tmem_ld32(tmem + lane_base + uint32_t(slot) * kSlotCols + cc * 32, v);
           const int jb = cc * 32;
@@ -441,7 +465,9 @@ __global__ void __launch_bounds__(kThreads, 1)
               ac[3] += tc::ex2(fmaf(v[4 * x4 + 3], a.scale_log2, -lv.w));
             }
           } else {
-            for (int x = 0; x < w.rows - jb; ++x) ac[x & 3] += tc::ex2(fmaf(v[x], a.scale_log2, -s.lse[jb + x]));
+#pragma unroll
+            for (int x = 0; x < 32; ++x)
+              if (jb + x < w.rows) ac[x & 3] += tc::ex2(fmaf(v[x], a.scale_log2, -s.lse[jb + x]));
           }
         }
         const float acc = (ac[0] + ac[1]) + (ac[2] + ac[3]);
