@@ -13,6 +13,7 @@ namespace conduit {
 namespace {
 
 constexpr int kLayerSlots = 32;
+constexpr int kBatch = 8;
 
 __global__ void __launch_bounds__(1024) finalize_tokens_kernel(const float* pa, const float* ss,
                                                                BatchDev b, int n_layers, int Hkv,
@@ -30,12 +31,28 @@ __global__ void __launch_bounds__(1024) finalize_tokens_kernel(const float* pa, 
     const float denom = float(nq * Hq);
     const int rows = (Hq / Hkv) * nq;
     const int n_sl = (group_rows ? (rows + group_rows - 1) / group_rows : 1) * parts;
+    const int npa = Hkv * n_sl, nss = Hkv * parts;  // partials of one layer
     for (int li = slot; li < n_layers; li += kLayerSlots) {
+      // loads go out in batches of eight, so their latencies overlap
+      const float* pa_l = pa + int64_t(li) * Hkv * rg_max * parts * n_tot + tg;
+      const float* ss_l = ss + int64_t(li) * nss * n_tot + tg;
       float col = 0.f, sq = 0.f;
-      for (int g = 0; g < Hkv; ++g) {
-        const int64_t lg = int64_t(li) * Hkv + g;
-        for (int sl = 0; sl < n_sl; ++sl) col += pa[(lg * rg_max * parts + sl) * n_tot + tg];
-        for (int p = 0; p < parts; ++p) sq += ss[(lg * parts + p) * n_tot + tg];
+      for (int q0 = 0; q0 < npa; q0 += kBatch) {
+        float x[kBatch];
+#pragma unroll
+        for (int k = 0; k < kBatch; ++k) {
+          const int q = q0 + k;
+          x[k] = q < npa ? pa_l[(int64_t(q / n_sl) * rg_max * parts + q % n_sl) * n_tot] : 0.f;
+        }
+#pragma unroll
+        for (int k = 0; k < kBatch; ++k) col += x[k];
+      }
+      for (int q0 = 0; q0 < nss; q0 += kBatch) {
+        float x[kBatch];
+#pragma unroll
+        for (int k = 0; k < kBatch; ++k) x[k] = q0 + k < nss ? ss_l[int64_t(q0 + k) * n_tot] : 0.f;
+#pragma unroll
+        for (int k = 0; k < kBatch; ++k) sq += x[k];
       }
       const float a = col / denom;
       acc_s = fmaf(a, sqrtf(sq), acc_s);

@@ -8,8 +8,8 @@
 //   pass A   D[rows x 128 tokens] = Q_rows . K_tile^T     (rows are the MMA M)
 //            each epilogue thread owns one row and a share of the columns:
 //            running max m and sum z = sum 2^((S - m) log2(e)/sqrt(d)), merged
-//            into lse = m log2(e)/sqrt(d) + log2 z; the same threads also
-//            stream the tile's V rows for the value norms (ss)
+//            into lse = m log2(e)/sqrt(d) + log2 z; the same threads read the
+//            tile's V rows (loaded by TMA) for the value norms (ss)
 //   pass B   D[128 tokens x rows] = K_tile . Q_rows^T     (tokens are the MMA M)
 //            each epilogue thread owns one token and half of the rows: sum of
 //            2^(x - lse) -> pa[l][g][group][half][t], this share of
@@ -18,7 +18,8 @@
 // Pass B walks the tiles in reverse so the most recent K tiles of pass A are
 // still in L2. Roles (320 threads):
 //   warp 0       one thread issues TMA loads of K tiles (128 tokens x 128
-//                dims, 128-byte swizzle) into a four-stage ring
+//                dims, 128-byte swizzle) into a three-stage ring, and of the
+//                matching V tiles into two buffers during pass A
 //   warp 1       one thread issues tcgen05 MMAs into two 256-column TMEM
 //                accumulator slots (it also owns the TMEM allocation)
 //   warps 2-9    epilogue, two warps per TMEM lane quarter (warp group h
@@ -39,7 +40,8 @@ namespace {
 
 constexpr int kD = 128;
 constexpr int kTile = 128;
-constexpr int kStages = 4;
+constexpr int kStages = 3;                     // K ring
+constexpr int kVBufs = 2;                      // V tiles (value norms, pass A)
 constexpr int kGroupRows = 256;
 constexpr int kThreads = 320;
 constexpr int kEpiThreads = 256;
@@ -47,7 +49,7 @@ constexpr uint32_t kHalfQ = kGroupRows * 128;  // 32 KB: one 64-dim half of the 
 constexpr uint32_t kHalfK = kTile * 128;       // 16 KB
 constexpr uint32_t kStageBytes = 2 * kHalfK;   // 32 KB per K tile
 constexpr uint32_t kSlotCols = 256;
-constexpr uint32_t kSmemBytes = 1024 + 2 * kHalfQ + kStages * kStageBytes + 256 + kGroupRows * 4 + 128 * 8;
+constexpr uint32_t kSmemBytes = 1024 + 2 * kHalfQ + (kStages + kVBufs) * kStageBytes + 256 + kGroupRows * 4;
 
 struct TcArgs {
   KvDev kv;
@@ -116,15 +118,17 @@ struct Smem {
   uint8_t* k;          // [kStages][2 halves][128 rows][128 B]
   uint64_t* kfull;     // [kStages]
   uint64_t* kempty;    // [kStages]
+  uint8_t* v;          // [kVBufs][2 halves][128 rows][128 B]
+  uint64_t* vfull;     // [kVBufs]
+  uint64_t* vempty;    // [kVBufs]
   uint64_t* tfull;     // [2]
   uint64_t* tempty;    // [2]
   uint64_t* qready;    // [1]
   uint64_t* mdone;     // [1]
   uint32_t* tmem_slot;
   volatile int* abort;
-  uint32_t* counters;  // [0] loads issued, [1] loads consumed
+  uint32_t* counters;  // [0] K loads issued, [1] K loads consumed, [2] V issued, [3] V consumed
   float* lse;          // [256]
-  float2* part;        // [128] (m, z) of the second column half
 };
 
 __device__ __forceinline__ Smem carve(uint8_t* raw) {
@@ -132,10 +136,13 @@ __device__ __forceinline__ Smem carve(uint8_t* raw) {
   Smem s;
   s.q = base;
   s.k = base + 2 * kHalfQ;
-  uint8_t* tail = s.k + kStages * kStageBytes;
+  s.v = s.k + kStages * kStageBytes;
+  uint8_t* tail = s.v + kVBufs * kStageBytes;
   s.kfull = reinterpret_cast<uint64_t*>(tail);
   s.kempty = s.kfull + kStages;
-  s.tfull = s.kempty + kStages;
+  s.vfull = s.kempty + kStages;
+  s.vempty = s.vfull + kVBufs;
+  s.tfull = s.vempty + kVBufs;
   s.tempty = s.tfull + 2;
   s.qready = s.tempty + 2;
   s.mdone = s.qready + 1;
@@ -143,7 +150,6 @@ __device__ __forceinline__ Smem carve(uint8_t* raw) {
   s.abort = reinterpret_cast<volatile int*>(s.tmem_slot + 1);
   s.counters = reinterpret_cast<uint32_t*>(s.tmem_slot + 2);
   s.lse = reinterpret_cast<float*>(tail + 256);
-  s.part = reinterpret_cast<float2*>(tail + 256 + kGroupRows * 4);
   return s;
 }
 
@@ -167,7 +173,7 @@ __device__ __forceinline__ void epi_barrier() {
   asm volatile("bar.sync 1, %0;" ::"n"(kEpiThreads) : "memory");
 }
 
-// Issue the TMA loads of K tile `tile` of unit w into ring stage `stage`.
+// Issue the TMA loads of K (or V) tile `tile` of unit w into `dst`.
 __device__ __forceinline__ void load_k_tile(const TcArgs& a, const CUtensorMap* kmap, const Unit& w,
                                             uint8_t* dst, uint64_t* bar, int tile) {
   tc::mbar_arrive_expect_tx(bar, kStageBytes);
@@ -224,8 +230,50 @@ __device__ __forceinline__ void stage_rows(const TcArgs& a, const Unit& w, uint8
   }
 }
 
+// Online row statistics over NC accumulator columns of which the first
+// `valid` are tokens of the slab: running max m (raw logit) and
+// z = sum 2^((S - m) scale). Only a ragged last tile takes the masked path.
+template <int NC>
+__device__ __forceinline__ void row_stats(float (&v)[NC], int valid, float scale, float& m,
+                                          float& z) {
+  if (valid < NC) {
+#pragma unroll
+    for (int x = 0; x < NC; ++x)
+      if (x >= valid) v[x] = -INFINITY;
+  }
+  float cm[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+  for (int x = 0; x < NC; ++x) cm[x & 3] = fmaxf(cm[x & 3], v[x]);
+  const float mn = fmaxf(m, fmaxf(fmaxf(cm[0], cm[1]), fmaxf(cm[2], cm[3])));
+  if (mn == -INFINITY) return;
+  const float nb = -mn * scale;
+  float ac[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+  for (int x = 0; x < NC; ++x) ac[x & 3] += tc::ex2(fmaf(v[x], scale, nb));
+  z = z * tc::ex2((m - mn) * scale) + ((ac[0] + ac[1]) + (ac[2] + ac[3]));
+  m = mn;
+}
+
+// Sum over NC accumulator columns (scoring rows c0 ...) of 2^(S scale - lse_row).
+// Columns past the row group carry lse = +inf and add exactly zero (the
+// accumulator columns there hold finite values: TMEM is zeroed at start).
+template <int NC>
+__device__ __forceinline__ float col_sum(const float (&v)[NC], const float* lse, float scale) {
+  float ac[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+  for (int x4 = 0; x4 < NC / 4; ++x4) {
+    const float4 lv = reinterpret_cast<const float4*>(lse)[x4];
+    ac[0] += tc::ex2(fmaf(v[4 * x4 + 0], scale, -lv.x));
+    ac[1] += tc::ex2(fmaf(v[4 * x4 + 1], scale, -lv.y));
+    ac[2] += tc::ex2(fmaf(v[4 * x4 + 2], scale, -lv.z));
+    ac[3] += tc::ex2(fmaf(v[4 * x4 + 3], scale, -lv.w));
+  }
+  return (ac[0] + ac[1]) + (ac[2] + ac[3]);
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
-    score_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ TcArgs a) {
+    score_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
+                    const __grid_constant__ TcArgs a) {
   extern __shared__ uint8_t smem_raw[];
   const Smem s = carve(smem_raw);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -234,6 +282,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::mbar_init(&s.kfull[i], 1);
       tc::mbar_init(&s.kempty[i], 1);
     }
+    for (int i = 0; i < kVBufs; ++i) {
+      tc::mbar_init(&s.vfull[i], 1);
+      tc::mbar_init(&s.vempty[i], kEpiThreads);
+    }
     for (int i = 0; i < 2; ++i) {
       tc::mbar_init(&s.tfull[i], 1);
       tc::mbar_init(&s.tempty[i], kEpiThreads);
@@ -241,9 +293,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc::mbar_init(s.qready, 1);
     tc::mbar_init(s.mdone, 1);
     *s.abort = 0;
-    s.counters[0] = s.counters[1] = 0;
+    for (int i = 0; i < 4; ++i) s.counters[i] = 0;
     tc::fence_barrier_init();
     tc::prefetch_tensormap(&kmap);
+    tc::prefetch_tensormap(&vmap);
   }
   if (warp == 1) tc::tmem_alloc(s.tmem_slot, 2 * kSlotCols);
   __syncthreads();
@@ -252,7 +305,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0 && lane == 0) {
     // ------------------------------------------------------------ producer
-    uint32_t seq = 0;
+    uint32_t seq = 0, vseq = 0;
     bool ok = true;
     for (int u = blockIdx.x; u < a.n_units && ok; u += gridDim.x) {
       Unit w;
@@ -265,9 +318,21 @@ __global__ void __launch_bounds__(kThreads, 1)
           break;
         }
         load_k_tile(a, &kmap, w, s.k + st * kStageBytes, &s.kfull[st], tile_of(w, i));
+        if (i < w.tiles && w.rg == 0) {  // V tile for the value norms, read by the epilogue in pass A
+          const int vb = vseq % kVBufs;
+          if (!wait_or_abort(&s.vempty[vb], ((vseq / kVBufs) & 1) ^ 1, s.abort)) {
+            if (!*s.abort) raise_abort(a, s, tc::kSiteLoad);
+            ok = false;
+            ++seq;
+            break;
+          }
+          load_k_tile(a, &vmap, w, s.v + vb * kStageBytes, &s.vfull[vb], i);
+          ++vseq;
+        }
       }
     }
     s.counters[0] = seq;
+    s.counters[2] = vseq;
   } else if (warp == 1 && lane == 0) {
     // ----------------------------------------------------------------- MMA
     uint32_t kseq = 0, tseq = 0, useq = 0;
@@ -338,8 +403,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int lrow = quarter * 32 + lane;          // row (pass A) / token (pass B) in the tile
     const uint32_t lane_base = uint32_t(quarter * 32) << 16;
     const int64_t n_tot = a.kv.n_tot;
-    uint32_t tseq = 0;
+    uint32_t tseq = 0, vcons = 0;
     bool ok = true;
+    {  // zero this warp's TMEM lanes once, so unwritten accumulator columns hold finite values
+      uint32_t zero[64];
+#pragma unroll
+      for (int i = 0; i < 64; ++i) zero[i] = 0u;
+      for (int c = h * 256; c < h * 256 + 256; c += 64) tc::tmem_st64(tmem + lane_base + c, zero);
+      tc::tc_fence_before();
+    }
     for (int u = blockIdx.x; u < a.n_units; u += gridDim.x) {
       Unit w;
       if (!decode_unit(a, u, w)) continue;
@@ -348,26 +420,16 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::fence_proxy_async_smem();
       epi_barrier();
       if (et == 0) tc::mbar_arrive(s.qready);
-      // pass A share: row block rb, 32-column chunks [cc0, cc0 + ncc)
+      // pass A share: row block rb (with one row block the second warp group
+      // only does value norms) and this thread's half of each V row
+      const bool do_rows = nrb == 2 || h == 0;
       const int rb = nrb == 2 ? h : 0;
-      const int cc0 = nrb == 2 ? 0 : 2 * h;
-      const int ncc = nrb == 2 ? 4 : 2;
       const bool do_norm = w.rg == 0;  // one row group of each slab also streams V
       const int64_t lg = int64_t(w.li) * a.kv.Hkv + w.g;
       float* ss_out = a.ss + (lg * 2 + h) * n_tot + w.t0;
       float m = -INFINITY, z = 0.f;
       for (int i = 0; i < w.tiles; ++i) {            // pass A
         const int slot = tseq & 1;
-        // half (64 dims) of this thread's V row, loaded before the wait to hide its latency
-        const int tok_v = i * kTile + lrow;
-        uint4 vrow[8];
-        const bool vload = ok && do_norm && tok_v < w.N;
-        if (vload) {
-          const uint4* src = reinterpret_cast<const uint4*>(
-              static_cast<const __nv_bfloat16*>(a.kv.v) + a.kv.row(w.l, w.g, w.r, int64_t(w.t0) + tok_v, tok_v) + h * 64);
-#pragma unroll
-          for (int c = 0; c < 8; ++c) vrow[c] = src[c];
-        }
         // tcgen05.ld is warp-collective: the whole warp goes on or stops
         const bool got = __all_sync(0xffffffffu, ok && wait_or_abort(&s.tfull[slot], (tseq >> 1) & 1, s.abort));
         ++tseq;
@@ -377,59 +439,50 @@ __global__ void __launch_bounds__(kThreads, 1)
           continue;
         }
         tc::tc_fence_after();
-        const int tok0 = i * kTile;
-#pragma unroll 1
-        for (int cc = cc0; cc < cc0 + ncc; ++cc) {
-          float v[32];
-          tc::tmem_ld32(tmem + lane_base + uint32_t(slot) * kSlotCols + rb * 128 + cc * 32, v);
-          const int tok = tok0 + cc * 32;
-          if (tok + 32 > w.N) {  // ragged last tile only
-#pragma unroll
-            for (int x = 0; x < 32; ++x)
-              if (tok + x >= w.N) v[x] = -INFINITY;
-          }
-          float cm[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-#pragma unroll
-          for (int x = 0; x < 32; ++x) cm[x & 3] = fmaxf(cm[x & 3], v[x]);
-          const float cmax = fmaxf(fmaxf(cm[0], cm[1]), fmaxf(cm[2], cm[3]));
-          const float mn = fmaxf(m, cmax);
-          if (mn != -INFINITY) {
-            const float nb = -mn * a.scale_log2;
-            float ac[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-            for (int x = 0; x < 32; ++x) ac[x & 3] += tc::ex2(fmaf(v[x], a.scale_log2, nb));
-            z = z * exp2f((m - mn) * a.scale_log2) + ((ac[0] + ac[1]) + (ac[2] + ac[3]));
-            m = mn;
-          }
+        const uint32_t col0 = uint32_t(slot) * kSlotCols + rb * 128;
+        const int valid = w.N - i * kTile;
+        if (do_rows) {  // 128 columns in two loads; the slot is free again after the second
+          float v[64];
+          tc::tmem_ld64(tmem + lane_base + col0, v);
+          row_stats<64>(v, valid, a.scale_log2, m, z);
+          tc::tmem_ld64(tmem + lane_base + col0 + 64, v);
+          tc::tc_fence_before();
+          tc::mbar_arrive(&s.tempty[slot]);
+          row_stats<64>(v, valid - 64, a.scale_log2, m, z);
+        } else {
+          tc::tc_fence_before();
+          tc::mbar_arrive(&s.tempty[slot]);
         }
-        tc::tc_fence_before();
-        tc::mbar_arrive(&s.tempty[slot]);
-        if (vload) {  // sum of squares of this half of the cached value row
+        if (do_norm) {  // half (64 dims) of V row lrow of the tile, from shared memory
+          const int vb = vcons % kVBufs;
+          if (!wait_or_abort(&s.vfull[vb], (vcons / kVBufs) & 1, s.abort)) {
+            if (!*s.abort) raise_abort(a, s, tc::kSiteLoad);
+            ok = false;
+            continue;
+          }
+          ++vcons;
+          const uint8_t* vh = s.v + vb * kStageBytes + h * kHalfK;
           float sq[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
           for (int c = 0; c < 8; ++c) {
-            const __nv_bfloat162* hv = reinterpret_cast<const __nv_bfloat162*>(&vrow[c]);
+            const uint4 x = *reinterpret_cast<const uint4*>(vh + tc::sw128_offset(lrow, c));
+            const __nv_bfloat162* hv = reinterpret_cast<const __nv_bfloat162*>(&x);
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
               const float2 f = __bfloat1622float2(hv[e]);
               sq[e] = fmaf(f.x, f.x, fmaf(f.y, f.y, sq[e]));
             }
           }
-          ss_out[tok_v] = (sq[0] + sq[1]) + (sq[2] + sq[3]);
+          tc::mbar_arrive(&s.vempty[vb]);
+          const int tok = i * kTile + lrow;
+          if (tok < w.N) ss_out[tok] = (sq[0] + sq[1]) + (sq[2] + sq[3]);
         }
       }
       // log2-sum-exp of each row, shared with the token-owning threads of pass B
-      if (nrb == 1 && h == 1) s.part[lrow] = make_float2(m, z);
-      epi_barrier();
-      if (nrb == 2) {
-        s.lse[h * 128 + lrow] = m * a.scale_log2 + log2f(z);
-      } else if (h == 0) {
-        const float2 o = s.part[lrow];
-        const float mm = fmaxf(m, o.x);
-        float zz = 0.f;
-        if (m != -INFINITY) zz += z * exp2f((m - mm) * a.scale_log2);
-        if (o.x != -INFINITY) zz += o.y * exp2f((o.x - mm) * a.scale_log2);
-        s.lse[lrow] = mm * a.scale_log2 + log2f(zz);
+      // (+inf past the row group: those columns then add zero)
+      {
+        const int row = (do_rows ? rb : 1) * 128 + lrow;
+        s.lse[row] = (do_rows && row < w.rows) ? m * a.scale_log2 + log2f(z) : INFINITY;
       }
       epi_barrier();
       // pass B share: 32-row chunks [cb0, cb1)
@@ -449,39 +502,44 @@ __global__ void __launch_bounds__(kThreads, 1)
           continue;
         }
         tc::tc_fence_after();
-        float ac[4] = {0.f, 0.f, 0.f, 0.f};
-        for (int cc = cb0; cc < cb1; ++cc) {
-          float v[32];
-          tc::tmem_ld32(tmem + lane_base + uint32_t(slot) * kSlotCols + cc * 32, v);
-          const int jb = cc * 32;
-          const float4* l4 = reinterpret_cast<const float4*>(s.lse + jb);
-          if (jb + 32 <= w.rows) {
-#pragma unroll
-            for (int x4 = 0; x4 < 8; ++x4) {
-              const float4 lv = l4[x4];
-              ac[0] += tc::ex2(fmaf(v[4 * x4 + 0], a.scale_log2, -lv.x));
-              ac[1] += tc::ex2(fmaf(v[4 * x4 + 1], a.scale_log2, -lv.y));
-              ac[2] += tc::ex2(fmaf(v[4 * x4 + 2], a.scale_log2, -lv.z));
-              ac[3] += tc::ex2(fmaf(v[4 * x4 + 3], a.scale_log2, -lv.w));
-            }
-          } else {
-#pragma unroll
-            for (int x = 0; x < 32; ++x)
-              if (jb + x < w.rows) ac[x & 3] += tc::ex2(fmaf(v[x], a.scale_log2, -s.lse[jb + x]));
+        // this thread's columns [32 cb0, 32 cb1) in loads of 64 (and one of 32);
+        // the slot is free again after the last load
+        const uint32_t col0 = uint32_t(slot) * kSlotCols + cb0 * 32;
+        const int ncol = (cb1 - cb0) * 32;
+        const float* lse = s.lse + cb0 * 32;
+        float acc = 0.f;
+        int c = 0;
+        for (; c + 64 <= ncol; c += 64) {
+          float v[64];
+          tc::tmem_ld64(tmem + lane_base + col0 + c, v);
+          if (c + 64 == ncol) {
+            tc::tc_fence_before();
+            tc::mbar_arrive(&s.tempty[slot]);
           }
+          acc += col_sum<64>(v, lse + c, a.scale_log2);
         }
-        const float acc = (ac[0] + ac[1]) + (ac[2] + ac[3]);
-        tc::tc_fence_before();
-        tc::mbar_arrive(&s.tempty[slot]);
+        if (c < ncol) {
+          float v[32];
+          tc::tmem_ld32(tmem + lane_base + col0 + c, v);
+          tc::tc_fence_before();
+          tc::mbar_arrive(&s.tempty[slot]);
+          acc += col_sum<32>(v, lse + c, a.scale_log2);
+        } else if (ncol == 0) {
+          tc::tc_fence_before();
+          tc::mbar_arrive(&s.tempty[slot]);
+        }
         if (tok < w.N) pa_out[tok] = acc;
       }
       epi_barrier();  // every thread is done with this unit's rows and lse
     }
+    if (et == 0) s.counters[3] = vcons;
   }
   __syncthreads();
   if (tid == 0) {  // drain TMA copies issued but never consumed (only after an abort)
     for (uint32_t n = s.counters[1]; n < s.counters[0]; ++n)
       tc::mbar_wait(&s.kfull[n % kStages], (n / kStages) & 1);
+    for (uint32_t n = s.counters[3]; n < s.counters[2]; ++n)
+      tc::mbar_wait(&s.vfull[n % kVBufs], (n / kVBufs) & 1);
   }
   tc::tc_fence_before();
   __syncthreads();
@@ -521,7 +579,7 @@ cudaError_t launch_score_tc(const KvDev& kv, const BatchDev& b, const int32_t* q
                             float* pa, float* ss, int32_t* status, cudaStream_t stream) {
   EncodeTiledFn enc = encode_fn();
   if (!enc) return cudaErrorNotSupported;
-  CUtensorMap kmap;
+  CUtensorMap kmap, vmap;
   cuuint64_t dims[2] = {cuuint64_t(kD), 0};
   cuuint64_t strides[1] = {cuuint64_t(kD) * 2};
   cuuint32_t box[2] = {64, 0};
@@ -534,6 +592,10 @@ cudaError_t launch_score_tc(const KvDev& kv, const BatchDev& b, const int32_t* q
     box[1] = kv.page_size;
   }
   if (enc(&kmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, kv.k, dims, strides, box, estr,
+          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    return cudaErrorInvalidValue;
+  if (enc(&vmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, kv.v, dims, strides, box, estr,
           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
     return cudaErrorInvalidValue;
@@ -562,7 +624,7 @@ cudaError_t launch_score_tc(const KvDev& kv, const BatchDev& b, const int32_t* q
   if ((err = cudaFuncSetAttribute(score_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                   int(kSmemBytes))))
     return err;
-  score_tc_kernel<<<std::min(units, sms), kThreads, kSmemBytes, stream>>>(kmap, a);
+  score_tc_kernel<<<std::min(units, sms), kThreads, kSmemBytes, stream>>>(kmap, vmap, a);
   count_launches(1);
   return cudaGetLastError();
 }
