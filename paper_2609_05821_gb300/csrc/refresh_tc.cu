@@ -5,23 +5,29 @@
 // One CTA owns up to two query tiles of 128 rows of one (layer, KV head,
 // request); a tile holds floor(128/G) consecutive selected rows times the G
 // query heads that share the KV head, and both tiles share every K/V tile.
-// Keys stream in tiles of 64. Roles (320 threads):
-//   warp 0     one thread issues TMA loads of K and V tiles into two
-//              three-stage rings (K frees after both S, V after both P.V)
-//   warp 1     one thread issues tcgen05 MMAs: per query tile, S(t) = Q K(t)^T
-//              into one of two TMEM S buffers and O += P(t) V(t); S(t+2) is
-//              issued right after P.V(t), so softmax overlaps tensor work
-//   warps 2-5, 6-9   softmax of tile 0 and tile 1: stage the query rows, then
-//              per key tile read S(t) (one row per thread), apply the causal
-//              mask j <= p_i, keep a lazy running max (O and the row sum are
-//              rescaled only when the max grows by 2^8; warp-uniform, since
-//              tcgen05.ld/st are warp-collective), write P(t) in bf16 to one
-//              of two shared buffers, and finally write O / rowsum in bf16
-// TMEM: tile q uses columns [256q, 256q + 128) for its two S buffers and
-// [256q + 128, 256q + 256) for O. Rows are sorted by position, so a CTA needs
-// keys up to its last row's position only. Every wait is bounded by one
-// second; a role that gives up raises an abort flag the others watch, the
-// kernel sets CONDUIT_FLAG_TIMEOUT, drains its copies and MMAs, frees TMEM.
+// Keys stream in tiles of 128 (a tcgen05.mma costs about the same issue time
+// for N = 64 and N = 128, so wide tiles halve the instruction count).
+// Roles (320 threads):
+//   warp 0     one thread issues TMA loads of K tiles (three-stage ring) and
+//              V tiles (two stages)
+//   warp 1     one thread issues tcgen05 MMAs. Per key tile t and query tile
+//              x: S_x(t) = Q_x K(t)^T into TMEM, then O_x += P_x(t) V(t) with
+//              P_x read from TMEM. S_x(t+1) overwrites the columns P_x(t)
+//              lives in, so it is issued only once P_x(t) V(t) has completed;
+//              the other tile's MMAs keep the tensor pipe busy meanwhile
+//   warps 2-5, 6-9   softmax of query tile 0 and 1: stage the query rows,
+//              then per key tile read S (one row per thread), apply the
+//              causal mask j <= p_i, keep a lazy running max (O and the row
+//              sum are rescaled only when the max grows by 2^8; warp-uniform,
+//              since tcgen05.ld/st are warp-collective), write P in bf16 pairs
+//              over the upper half of S, and finally write O / rowsum in bf16
+// TMEM: query tile x uses columns [256x, 256x + 128) for S (P in the upper 64
+// columns) and [256x + 128, 256x + 256) for O. When a softmax warp sees S_x(t),
+// O_x already holds P_x(t-1) V(t-1), so a rescale needs no further wait.
+// Rows are sorted by position, so a CTA needs keys up to its last row's
+// position only. Every wait is bounded by one second; a role that gives up
+// raises an abort flag the others watch, the kernel sets CONDUIT_FLAG_TIMEOUT,
+// drains its copies and MMAs, and frees TMEM.
 #include <cuda.h>
 
 #include "internal.cuh"
@@ -31,21 +37,21 @@ namespace conduit {
 namespace {
 
 constexpr int kD = 128;
-constexpr int kKT = 64;                          // keys per tile
+constexpr int kKT = 128;                         // keys per tile
 constexpr int kRows = 128;                       // rows per query tile
 constexpr int kTiles = 2;                        // query tiles per CTA
 constexpr int kSoftThreads = 128;
 constexpr int kThreads = 64 + kTiles * kSoftThreads;
-constexpr int kStages = 3;
+constexpr int kKStages = 3;
+constexpr int kVStages = 2;
 constexpr uint32_t kQHalf = kRows * 128;         // 16 KB: one 64-dim half of a query tile
 constexpr uint32_t kQBytes = 2 * kQHalf;         // 32 KB
-constexpr uint32_t kTileHalf = kKT * 128;        // 8 KB: one 64-dim half of a K or V tile
-constexpr uint32_t kTileBytes = 2 * kTileHalf;   // 16 KB
-constexpr uint32_t kPBytes = kRows * 128;        // 16 KB: 128 rows x 64 keys
-constexpr uint32_t kSmem =
-    1024 + kTiles * kQBytes + 2 * kStages * kTileBytes + kTiles * 2 * kPBytes + 512;
+constexpr uint32_t kTileHalf = kKT * 128;        // 16 KB: one 64-dim half of a K or V tile
+constexpr uint32_t kTileBytes = 2 * kTileHalf;   // 32 KB
+constexpr uint32_t kSmem = 1024 + kTiles * kQBytes + (kKStages + kVStages) * kTileBytes + 256;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kTileCols = 256;              // TMEM columns per query tile
+constexpr uint32_t kPCol = 64;                   // P (bf16 pairs) over the upper half of S
 constexpr uint32_t kOCol = 128;                  // O offset inside a tile's columns
 constexpr float kRescaleLog2 = 8.f;
 
@@ -65,12 +71,11 @@ struct RefArgs {
 
 struct Smem {
   uint8_t* q;        // [kTiles][2 halves][128 rows][128 B]
-  uint8_t* k;        // [kStages][2 halves][64 keys][128 B]
-  uint8_t* v;        // [kStages][2 halves][64 keys][128 B]
-  uint8_t* p;        // [kTiles][2][128 rows][128 B]
-  uint64_t *kfull, *kempty, *vfull, *vempty;  // [kStages] each
-  uint64_t *sfull, *pfull, *pempty;           // [kTiles][2] each
-  uint64_t *obar;                             // [kTiles]
+  uint8_t* k;        // [kKStages][2 halves][128 keys][128 B]
+  uint8_t* v;        // [kVStages][2 halves][128 keys][128 B]
+  uint64_t *kfull, *kempty;           // [kKStages]
+  uint64_t *vfull, *vempty;           // [kVStages]
+  uint64_t *sfull, *pfull, *pvdone;   // [kTiles]
   uint64_t *qready, *mdone;
   uint32_t* tmem_slot;
   volatile int* abort;
@@ -82,18 +87,16 @@ __device__ __forceinline__ Smem carve(uint8_t* raw) {
   Smem s;
   s.q = base;
   s.k = s.q + kTiles * kQBytes;
-  s.v = s.k + kStages * kTileBytes;
-  s.p = s.v + kStages * kTileBytes;
-  uint64_t* bar = reinterpret_cast<uint64_t*>(s.p + kTiles * 2 * kPBytes);
+  s.v = s.k + kKStages * kTileBytes;
+  uint64_t* bar = reinterpret_cast<uint64_t*>(s.v + kVStages * kTileBytes);
   s.kfull = bar;
-  s.kempty = bar + kStages;
-  s.vfull = bar + 2 * kStages;
-  s.vempty = bar + 3 * kStages;
-  s.sfull = bar + 4 * kStages;
-  s.pfull = s.sfull + 2 * kTiles;
-  s.pempty = s.pfull + 2 * kTiles;
-  s.obar = s.pempty + 2 * kTiles;
-  s.qready = s.obar + kTiles;
+  s.kempty = s.kfull + kKStages;
+  s.vfull = s.kempty + kKStages;
+  s.vempty = s.vfull + kVStages;
+  s.sfull = s.vempty + kVStages;
+  s.pfull = s.sfull + kTiles;
+  s.pvdone = s.pfull + kTiles;
+  s.qready = s.pvdone + kTiles;
   s.mdone = s.qready + 1;
   s.tmem_slot = reinterpret_cast<uint32_t*>(s.mdone + 1);
   s.abort = reinterpret_cast<volatile int*>(s.tmem_slot + 1);
@@ -116,7 +119,7 @@ __device__ __forceinline__ void raise_abort(const RefArgs& a, const Smem& s, int
   *s.abort = 1;
 }
 
-// TMA of the 64-key tile starting at request-local key j0 (one 64-dim half per box).
+// TMA of the 128-key tile starting at request-local key j0 (one 64-dim half per box).
 __device__ __forceinline__ void load_tile(const RefArgs& a, const CUtensorMap* map, uint8_t* dst,
                                           uint64_t* bar, int l, int g, int r, int t0, int N, int j0) {
   const KvDev& kv = a.kv;
@@ -171,18 +174,19 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int nq = cnt > a.rows_per_tile ? 2 : 1;   // query tiles in use (CTA-uniform)
 
   if (tid == 0) {
-    for (int i = 0; i < kStages; ++i) {
+    for (int i = 0; i < kKStages; ++i) {
       tc::mbar_init(&s.kfull[i], 1);
       tc::mbar_init(&s.kempty[i], 1);
+    }
+    for (int i = 0; i < kVStages; ++i) {
       tc::mbar_init(&s.vfull[i], 1);
       tc::mbar_init(&s.vempty[i], 1);
     }
-    for (int i = 0; i < 2 * kTiles; ++i) {
+    for (int i = 0; i < kTiles; ++i) {
       tc::mbar_init(&s.sfull[i], 1);
       tc::mbar_init(&s.pfull[i], kSoftThreads);
-      tc::mbar_init(&s.pempty[i], 1);
+      tc::mbar_init(&s.pvdone[i], 1);
     }
-    for (int i = 0; i < kTiles; ++i) tc::mbar_init(&s.obar[i], 1);
     tc::mbar_init(s.qready, kTiles);
     tc::mbar_init(s.mdone, 1);
     *s.abort = 0;
@@ -200,13 +204,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ---------------------------------------------------------------- loads
     uint32_t nk = 0, nv = 0;
     for (int t = 0; t < ntiles; ++t) {
-      const int st = t % kStages;
-      const uint32_t ph = ((t / kStages) & 1) ^ 1;
-      if (!wait_or_abort(&s.kempty[st], ph, s.abort)) { raise_abort(a, s, tc::kSiteLoad); break; }
-      load_tile(a, &kmap, s.k + st * kTileBytes, &s.kfull[st], l, g, r, t0, N, t * kKT);
+      const int sk = t % kKStages;
+      if (!wait_or_abort(&s.kempty[sk], ((t / kKStages) & 1) ^ 1, s.abort)) { raise_abort(a, s, tc::kSiteLoad); break; }
+      load_tile(a, &kmap, s.k + sk * kTileBytes, &s.kfull[sk], l, g, r, t0, N, t * kKT);
       ++nk;
-      if (!wait_or_abort(&s.vempty[st], ph, s.abort)) { raise_abort(a, s, tc::kSiteLoad); break; }
-      load_tile(a, &vmap, s.v + st * kTileBytes, &s.vfull[st], l, g, r, t0, N, t * kKT);
+      const int sv = t % kVStages;
+      if (!wait_or_abort(&s.vempty[sv], ((t / kVStages) & 1) ^ 1, s.abort)) { raise_abort(a, s, tc::kSiteLoad); break; }
+      load_tile(a, &vmap, s.v + sv * kTileBytes, &s.vfull[sv], l, g, r, t0, N, t * kKT);
       ++nv;
     }
     s.counters[0] = nk;
@@ -216,49 +220,54 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t ck = 0, cv = 0;
     const uint32_t idesc_s = tc::idesc_bf16(kRows, kKT);
     const uint32_t idesc_o = tc::idesc_bf16(kRows, kD, /*b_mn_major=*/true);
-    auto issue_s = [&](int t) -> bool {  // S(t) of every query tile into its S buffer t & 1
-      const int st = t % kStages;
-      if (!wait_or_abort(&s.kfull[st], (t / kStages) & 1, s.abort)) return false;
+    auto issue_s = [&](int qi, uint32_t k_addr) {  // S_qi = Q_qi K^T
+      const uint32_t q_addr = tc::smem_u32(s.q + qi * kQBytes);
+#pragma unroll
+      for (int kk = 0; kk < 8; ++kk) {
+        const uint32_t off = (kk & 3) * 32;
+        tc::mma_bf16(tmem + qi * kTileCols, tc::desc_sw128(q_addr + (kk >> 2) * kQHalf + off),
+                     tc::desc_sw128(k_addr + (kk >> 2) * kTileHalf + off), idesc_s, kk > 0);
+      }
+      tc::mma_commit(&s.sfull[qi]);
+    };
+    bool ok = wait_or_abort(s.qready, 0, s.abort) && wait_or_abort(&s.kfull[0], 0, s.abort);
+    if (ok) {
       ++ck;
       tc::tc_fence_after();
-      const uint32_t k_addr = tc::smem_u32(s.k + st * kTileBytes);
-      for (int qi = 0; qi < nq; ++qi) {
-        const uint32_t q_addr = tc::smem_u32(s.q + qi * kQBytes);
-#pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {
-          const uint32_t off = (kk & 3) * 32;
-          tc::mma_bf16(tmem + qi * kTileCols + uint32_t(t & 1) * kKT,
-                       tc::desc_sw128(q_addr + (kk >> 2) * kQHalf + off),
-                       tc::desc_sw128(k_addr + (kk >> 2) * kTileHalf + off), idesc_s, kk > 0);
-        }
-        tc::mma_commit(&s.sfull[qi * 2 + (t & 1)]);
-      }
-      tc::mma_commit(&s.kempty[st]);
-      return true;
-    };
-    bool ok = wait_or_abort(s.qready, 0, s.abort);
-    if (ok) ok = issue_s(0);
-    if (ok && ntiles > 1) ok = issue_s(1);
+      for (int qi = 0; qi < nq; ++qi) issue_s(qi, tc::smem_u32(s.k));
+      tc::mma_commit(&s.kempty[0]);
+    }
     for (int t = 0; t < ntiles && ok; ++t) {
-      const int b = t & 1, st = t % kStages;
-      if (!wait_or_abort(&s.vfull[st], (t / kStages) & 1, s.abort)) { ok = false; break; }
+      const int sv = t % kVStages;
+      if (!wait_or_abort(&s.vfull[sv], (t / kVStages) & 1, s.abort)) { ok = false; break; }
       ++cv;
-      const uint32_t v_addr = tc::smem_u32(s.v + st * kTileBytes);
-      for (int qi = 0; qi < nq && ok; ++qi) {
-        if (!wait_or_abort(&s.pfull[qi * 2 + b], (t >> 1) & 1, s.abort)) { ok = false; break; }
+      const uint32_t v_addr = tc::smem_u32(s.v + sv * kTileBytes);
+      for (int qi = 0; qi < nq && ok; ++qi) {  // O_qi += P_qi V
+        if (!wait_or_abort(&s.pfull[qi], t & 1, s.abort)) { ok = false; break; }
         tc::tc_fence_after();
-        const uint32_t p_addr = tc::smem_u32(s.p + (qi * 2 + b) * kPBytes);
+        const uint32_t tb = tmem + qi * kTileCols;
 #pragma unroll
-        for (int kk = 0; kk < kKT / 16; ++kk) {
-          tc::mma_bf16(tmem + qi * kTileCols + kOCol, tc::desc_sw128(p_addr + kk * 32),
-                       tc::desc_sw128_mn(v_addr + kk * 2048, kTileHalf), idesc_o, t > 0 || kk > 0);
-        }
-        tc::mma_commit(&s.pempty[qi * 2 + b]);
-        tc::mma_commit(&s.obar[qi]);
+        for (int kk = 0; kk < kKT / 16; ++kk)
+          tc::mma_bf16_ts(tb + kOCol, tb + kPCol + kk * 8, tc::desc_sw128_mn(v_addr + kk * 2048, kTileHalf),
+                          idesc_o, t > 0 || kk > 0);
+        tc::mma_commit(&s.pvdone[qi]);
       }
       if (!ok) break;
-      tc::mma_commit(&s.vempty[st]);
-      if (t + 2 < ntiles && !issue_s(t + 2)) { ok = false; break; }
+      tc::mma_commit(&s.vempty[sv]);
+      if (t + 1 < ntiles) {
+        const int sk = (t + 1) % kKStages;
+        if (!wait_or_abort(&s.kfull[sk], ((t + 1) / kKStages) & 1, s.abort)) { ok = false; break; }
+        ++ck;
+        const uint32_t k_addr = tc::smem_u32(s.k + sk * kTileBytes);
+        for (int qi = 0; qi < nq && ok; ++qi) {
+          // S_qi(t+1) overwrites P_qi(t): wait until P_qi(t) V(t) has completed
+          if (!wait_or_abort(&s.pvdone[qi], t & 1, s.abort)) { ok = false; break; }
+          tc::tc_fence_after();
+          issue_s(qi, k_addr);
+        }
+        if (!ok) break;
+        tc::mma_commit(&s.kempty[sk]);
+      }
     }
     if (!ok) raise_abort(a, s, tc::kSiteMma);
     s.counters[2] = ck;
@@ -272,7 +281,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int quarter = warp & 3;
     const int row = quarter * 32 + lane;                 // TMEM lane = query row of the tile
     const uint32_t lane_base = uint32_t(quarter * 32) << 16;
-    const uint32_t tcol = qi * kTileCols;
+    const uint32_t tb = tmem + lane_base + qi * kTileCols;
     const int ti0 = i0 + qi * a.rows_per_tile;           // first selected row of the tile
     const int tcnt = max(0, min(a.rows_per_tile, cnt - qi * a.rows_per_tile));
     const bool active = qi < nq;
@@ -308,111 +317,98 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (et == 0) tc::mbar_arrive(s.qready);
 
     bool ok = active;
-    float m_ref = -INFINITY, lsum = 0.f;
+    float m_ref = -INFINITY, lsum = 0.f;  // running max (scaled, log2 units) and row sum
     for (int t = 0; t < ntiles && active; ++t) {
-      const int b = t & 1;
       // the tcgen05.ld below is warp-collective: the whole warp goes on or stops
-      const bool got = __all_sync(0xffffffffu, ok && wait_or_abort(&s.sfull[qi * 2 + b], (t >> 1) & 1, s.abort));
+      const bool got = __all_sync(0xffffffffu, ok && wait_or_abort(&s.sfull[qi], t & 1, s.abort));
       if (!got) {
         if (ok) raise_abort(a, s, tc::kSiteMma);
         ok = false;
         continue;
       }
       tc::tc_fence_after();
-      float sv[2][32];
-      tc::tmem_ld32(tmem + lane_base + tcol + uint32_t(b) * kKT, sv[0]);
-      tc::tmem_ld32(tmem + lane_base + tcol + uint32_t(b) * kKT + 32, sv[1]);
+      float sv0[64], sv1[64];
+      tc::tmem_ld64(tb, sv0);
+      tc::tmem_ld64(tb + 64, sv1);
       const int j0 = t * kKT;
+      if (j0 + kKT - 1 > p_row) {  // part of the tile is past this row's position
+#pragma unroll
+        for (int i = 0; i < 64; ++i) {
+          if (j0 + i > p_row) sv0[i] = -INFINITY;
+          if (j0 + 64 + i > p_row) sv1[i] = -INFINITY;
+        }
+      }
       float tm[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-      if (j0 + kKT - 1 <= p_row) {  // the whole tile is visible to this row
 #pragma unroll
-        for (int h2 = 0; h2 < 2; ++h2)
-#pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            sv[h2][i] *= a.scale_log2;
-            tm[i & 3] = fmaxf(tm[i & 3], sv[h2][i]);
-          }
-      } else {
-#pragma unroll
-        for (int h2 = 0; h2 < 2; ++h2)
-#pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const float x = (j0 + h2 * 32 + i <= p_row) ? sv[h2][i] * a.scale_log2 : -INFINITY;
-            sv[h2][i] = x;
-            tm[i & 3] = fmaxf(tm[i & 3], x);
-          }
+      for (int i = 0; i < 64; ++i) {
+        tm[i & 3] = fmaxf(tm[i & 3], sv0[i]);
+        tm[(i + 2) & 3] = fmaxf(tm[(i + 2) & 3], sv1[i]);
       }
-      const float tmax = fmaxf(fmaxf(tm[0], tm[1]), fmaxf(tm[2], tm[3]));
+      const float tmax = fmaxf(fmaxf(tm[0], tm[1]), fmaxf(tm[2], tm[3])) * a.scale_log2;
       const bool need = tmax > m_ref + kRescaleLog2 || (m_ref == -INFINITY && tmax != -INFINITY);
-      const float alpha = need ? exp2f(m_ref - tmax) : 1.f;  // 0 when m_ref is -inf
-      if (__any_sync(0xffffffffu, need) && t > 0) {
-        // P.V(t-1) must be complete before this warp rescales its rows of O.
-        // S(t) was issued after P.V(t-2), so obar is at most one phase behind
-        // here and its parity cannot alias.
-        if (!__all_sync(0xffffffffu, wait_or_abort(&s.obar[qi], (t - 1) & 1, s.abort))) {
-          raise_abort(a, s, tc::kSiteMma);
-          ok = false;
-          continue;
-        }
-        tc::tc_fence_after();
-        for (int c = 0; c < kD; c += 32) {
-          float o[32];
-          tc::tmem_ld32(tmem + lane_base + tcol + kOCol + c, o);
-#pragma unroll
-          for (int i = 0; i < 32; ++i) o[i] *= alpha;
-          tc::tmem_st32(tmem + lane_base + tcol + kOCol + c, o);
-        }
-      }
+      const float alpha = need ? tc::ex2(m_ref - tmax) : 1.f;  // 0 when m_ref is -inf
       if (need) {
         lsum *= alpha;
         m_ref = tmax;
       }
-      // the P buffer of tile t was last read by P.V(t-2)
-      if (!wait_or_abort(&s.pempty[qi * 2 + b], ((t >> 1) & 1) ^ 1, s.abort)) {
-        raise_abort(a, s, tc::kSiteMma);
-        ok = false;
-        continue;
-      }
-      uint8_t* pb = s.p + (qi * 2 + b) * kPBytes;
+      // P = 2^(S scale - m) in bf16 pairs over the upper half of S (already read),
+      // 32 columns at a time
       float ls[4] = {0.f, 0.f, 0.f, 0.f};
+      const float nb = -m_ref;
+      const bool live = m_ref != -INFINITY;
+      {
+        uint32_t pw[32];
 #pragma unroll
-      for (int h2 = 0; h2 < 2; ++h2) {
-#pragma unroll
-        for (int c8 = 0; c8 < 4; ++c8) {
-          uint32_t w4[4];
-#pragma unroll
-          for (int u = 0; u < 4; ++u) {
-            const float p0 = (m_ref == -INFINITY) ? 0.f : tc::ex2(sv[h2][c8 * 8 + 2 * u] - m_ref);
-            const float p1 = (m_ref == -INFINITY) ? 0.f : tc::ex2(sv[h2][c8 * 8 + 2 * u + 1] - m_ref);
-            ls[u] += p0 + p1;
-            __nv_bfloat162 pr = __floats2bfloat162_rn(p0, p1);
-            w4[u] = *reinterpret_cast<uint32_t*>(&pr);
-          }
-          *reinterpret_cast<uint4*>(pb + tc::sw128_offset(row, h2 * 4 + c8)) =
-              make_uint4(w4[0], w4[1], w4[2], w4[3]);
+        for (int i = 0; i < 32; ++i) {
+          const float p0 = live ? tc::ex2(fmaf(sv0[2 * i], a.scale_log2, nb)) : 0.f;
+          const float p1 = live ? tc::ex2(fmaf(sv0[2 * i + 1], a.scale_log2, nb)) : 0.f;
+          ls[i & 1] += p0;
+          ls[(i & 1) + 2] += p1;
+          __nv_bfloat162 pr = __floats2bfloat162_rn(p0, p1);
+          pw[i] = *reinterpret_cast<uint32_t*>(&pr);
         }
+        tc::tmem_st32u(tb + kPCol, pw);
+      }
+      {
+        uint32_t pw[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          const float p0 = live ? tc::ex2(fmaf(sv1[2 * i], a.scale_log2, nb)) : 0.f;
+          const float p1 = live ? tc::ex2(fmaf(sv1[2 * i + 1], a.scale_log2, nb)) : 0.f;
+          ls[i & 1] += p0;
+          ls[(i & 1) + 2] += p1;
+          __nv_bfloat162 pr = __floats2bfloat162_rn(p0, p1);
+          pw[i] = *reinterpret_cast<uint32_t*>(&pr);
+        }
+        tc::tmem_st32u(tb + kPCol + 32, pw);
       }
       lsum += (ls[0] + ls[1]) + (ls[2] + ls[3]);
-      tc::fence_proxy_async_smem();
+      if (__any_sync(0xffffffffu, need) && t > 0) {
+        // O already holds P(t-1) V(t-1) (S(t) was issued after it completed),
+        // and P(t) V(t) waits for this warp's pfull arrival below
+        for (int c = 0; c < kD; c += 32) {
+          float o[32];
+          tc::tmem_ld32(tb + kOCol + c, o);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) o[i] *= alpha;
+          tc::tmem_st32(tb + kOCol + c, o);
+        }
+      }
       tc::tc_fence_before();
-      tc::mbar_arrive(&s.pfull[qi * 2 + b]);
+      tc::mbar_arrive(&s.pfull[qi]);
     }
     if (active) {
-      // O is complete once the MMA thread's final commit arrives. (The obar
-      // phase of the last P.V could alias: after this warp's last tile only
-      // P.V up to ntiles-3 is known to be done, two phases behind.)
-      if (ok && !wait_or_abort(s.mdone, 0, s.abort)) {
-        raise_abort(a, s, tc::kSiteFinal);
-        ok = false;
-      }
-      const bool all_ok = !__any_sync(0xffffffffu, !ok);
-      if (all_ok) {
+      // O is complete once the last P V of this tile has completed (phase
+      // ntiles-1 of pvdone; phase ntiles-2 completed before S(ntiles-1) was issued)
+      const bool fin = __all_sync(0xffffffffu, ok && wait_or_abort(&s.pvdone[qi], (ntiles - 1) & 1, s.abort));
+      if (!fin && ok) raise_abort(a, s, tc::kSiteFinal);
+      if (fin) {
         tc::tc_fence_after();
         const float inv = lsum > 0.f ? 1.f / lsum : 0.f;
         __nv_bfloat16* dst = a.out + ((int64_t(l) * a.n_sel + i_row) * Hq + h_row) * kD;
         for (int c = 0; c < kD; c += 32) {
           float o[32];
-          tc::tmem_ld32(tmem + lane_base + tcol + kOCol + c, o);
+          tc::tmem_ld32(tb + kOCol + c, o);
           if (row_ok && p_row >= 0) {
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
@@ -432,9 +428,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   if (tid == 0) {  // drain loads issued but never consumed (only after an abort)
     for (uint32_t n = s.counters[2]; n < s.counters[0]; ++n)
-      tc::mbar_wait(&s.kfull[n % kStages], (n / kStages) & 1);
+      tc::mbar_wait(&s.kfull[n % kKStages], (n / kKStages) & 1);
     for (uint32_t n = s.counters[3]; n < s.counters[1]; ++n)
-      tc::mbar_wait(&s.vfull[n % kStages], (n / kStages) & 1);
+      tc::mbar_wait(&s.vfull[n % kVStages], (n / kVStages) & 1);
   }
   tc::tc_fence_before();
   __syncthreads();
