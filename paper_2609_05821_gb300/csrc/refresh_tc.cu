@@ -237,36 +237,39 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int qi = 0; qi < nq; ++qi) issue_s(qi, tc::smem_u32(s.k));
       tc::mma_commit(&s.kempty[0]);
     }
+    // Per key tile t and query tile x in turn: O_x += P_x(t) V(t), then
+    // S_x(t+1) once that has completed. Query tile 1's softmax runs while
+    // tile 0's MMAs execute and vice versa (ping-pong).
     for (int t = 0; t < ntiles && ok; ++t) {
       const int sv = t % kVStages;
       if (!wait_or_abort(&s.vfull[sv], (t / kVStages) & 1, s.abort)) { ok = false; break; }
       ++cv;
       const uint32_t v_addr = tc::smem_u32(s.v + sv * kTileBytes);
-      for (int qi = 0; qi < nq && ok; ++qi) {  // O_qi += P_qi V
+      const bool more = t + 1 < ntiles;
+      const int sk = (t + 1) % kKStages;
+      uint32_t k_addr = 0;
+      if (more) {
+        if (!wait_or_abort(&s.kfull[sk], ((t + 1) / kKStages) & 1, s.abort)) { ok = false; break; }
+        ++ck;
+        k_addr = tc::smem_u32(s.k + sk * kTileBytes);
+      }
+      for (int qi = 0; qi < nq && ok; ++qi) {
         if (!wait_or_abort(&s.pfull[qi], t & 1, s.abort)) { ok = false; break; }
         tc::tc_fence_after();
         const uint32_t tb = tmem + qi * kTileCols;
 #pragma unroll
-        for (int kk = 0; kk < kKT / 16; ++kk)
+        for (int kk = 0; kk < kKT / 16; ++kk)  // O_qi += P_qi V
           tc::mma_bf16_ts(tb + kOCol, tb + kPCol + kk * 8, tc::desc_sw128_mn(v_addr + kk * 2048, kTileHalf),
                           idesc_o, t > 0 || kk > 0);
         tc::mma_commit(&s.pvdone[qi]);
-      }
-      if (!ok) break;
-      tc::mma_commit(&s.vempty[sv]);
-      if (t + 1 < ntiles) {
-        const int sk = (t + 1) % kKStages;
-        if (!wait_or_abort(&s.kfull[sk], ((t + 1) / kKStages) & 1, s.abort)) { ok = false; break; }
-        ++ck;
-        const uint32_t k_addr = tc::smem_u32(s.k + sk * kTileBytes);
-        for (int qi = 0; qi < nq && ok; ++qi) {
+        if (qi == nq - 1) tc::mma_commit(&s.vempty[sv]);
+        if (more) {
           // S_qi(t+1) overwrites P_qi(t): wait until P_qi(t) V(t) has completed
           if (!wait_or_abort(&s.pvdone[qi], t & 1, s.abort)) { ok = false; break; }
           tc::tc_fence_after();
           issue_s(qi, k_addr);
+          if (qi == nq - 1) tc::mma_commit(&s.kempty[sk]);
         }
-        if (!ok) break;
-        tc::mma_commit(&s.kempty[sk]);
       }
     }
     if (!ok) raise_abort(a, s, tc::kSiteMma);
