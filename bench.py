@@ -9,7 +9,7 @@ whole step per second (device time, inputs resident in HBM, L2 flushed
 between steps); ``e2e`` is the same through the public step with the cache,
 queries and fresh rows copied from pinned host memory each step and the
 selection and refresh output copied back. Under torchrun every rank runs its
-own replica on its own GPU (the path has no exchange step); the step time is
+own replica on its own GPU (the path has no collective step); the step time is
 the maximum over ranks.
 """
 
@@ -174,8 +174,7 @@ def work_model(pipe) -> dict:
     return {
         "score": {"bytes": score_bytes, "flops": score_flops},
         "select": {"bytes": sel_bytes, "flops": 0},
-        "gather": {"bytes": copy_bytes, "flops": 0},
-        "scatter": {"bytes": copy_bytes, "flops": 0},
+        "exchange": {"bytes": 2 * copy_bytes, "flops": 0},
         "refresh": {"bytes": ref_bytes, "flops": ref_flops},
     }
 
@@ -195,8 +194,7 @@ def call_kernels(pipe) -> dict:
         score = (["value_sumsq_kernel", "rowstats_kernel", "colsum_kernel"] + tail, "alu", "score_simt.cu")
         refresh = (["refresh_simt_kernel"], "alu", "refresh_simt.cu")
     return {"score": score, "select": (["select_kernel"], "hbm", "select.cu"),
-            "gather": (["kv_copy_kernel"], "hbm", "kvcopy.cu"),
-            "scatter": (["kv_copy_kernel"], "hbm", "kvcopy.cu"), "refresh": refresh}
+            "exchange": (["kv_copy_kernel"], "hbm", "kvcopy.cu"), "refresh": refresh}
 
 
 def _src_hash(src: str) -> str:
@@ -288,12 +286,12 @@ def run_conduit(args):
 
     # per-call breakdown over K eager steps (events on the launching stream)
     graph, pipe.graph = pipe.graph, None
-    calls = {"score": [], "select": [], "gather": [], "scatter": [], "refresh": []}
+    calls = {"score": [], "select": [], "exchange": [], "refresh": []}
     from paper_2609_05821_gb300 import conduit as CC
     stream = torch.cuda.current_stream()
     for _ in range(args.steps):
         flush()
-        ev = [torch.cuda.Event(enable_timing=True) for _ in range(6)]
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(5)]
         ev[0].record(stream)
         CC.conduit_score(pipe.kv, pipe.batch, pipe.q, pipe.layers, pipe.s, pipe.attn_sum, pipe.g,
                          pipe.ws_score, pipe.status)
@@ -301,16 +299,13 @@ def run_conduit(args):
         CC.conduit_select_topk(pipe.batch, pipe.s, pipe.g, pipe.lam, pipe.idx_off, pipe.idx_off_dev,
                                pipe.idx, pipe.mask, pipe.s_hat, pipe.coeff, pipe.ws_sel, pipe.status)
         ev[2].record(stream)
-        CC.conduit_kv_gather(pipe.kv, pipe.batch, pipe.idx, pipe.idx_off, pipe.idx_off_dev,
-                             pipe.k_old, pipe.v_old)
+        CC.conduit_kv_exchange(pipe.kv, pipe.batch, pipe.idx, pipe.idx_off, pipe.idx_off_dev,
+                               pipe.k_old, pipe.v_old, pipe.k_rows, pipe.v_rows)
         ev[3].record(stream)
-        CC.conduit_kv_scatter(pipe.kv, pipe.batch, pipe.idx, pipe.idx_off, pipe.idx_off_dev,
-                              pipe.k_rows, pipe.v_rows)
-        ev[4].record(stream)
         CC.conduit_refresh_attn(pipe.kv, pipe.batch, pipe.idx, pipe.idx_off, pipe.idx_off_dev,
                                 pipe.q_rows, pipe.out, pipe.ws_ref, pipe.status)
-        ev[5].record(stream)
-        ev[5].synchronize()
+        ev[4].record(stream)
+        ev[4].synchronize()
         for i, name in enumerate(calls):
             calls[name].append(ev[i].elapsed_time(ev[i + 1]))
     pipe.graph = graph
@@ -368,7 +363,7 @@ def run_conduit(args):
                    "l2": f"flushed between timed steps ({L2_FLUSH_BYTES >> 20} MB write)",
                    "cuda_graph": not args.no_graph, "parallelism": f"replicas x{world}"},
         "score_select_tokens_per_s": round(n_tok / ((call_ms["score"] + call_ms["select"]) / 1e3), 1),
-        "refresh_pass_us": round((call_ms["gather"] + call_ms["scatter"] + call_ms["refresh"]) * 1e3, 2),
+        "refresh_pass_us": round((call_ms["exchange"] + call_ms["refresh"]) * 1e3, 2),
         "breakdown": breakdown,
         "roofline": roofline,
         "e2e": {"value": round(world * n_tok / (e2e_mean / 1e3), 1), "unit": UNIT,

@@ -215,6 +215,23 @@ conduit_status conduit_kv_scatter(const conduit_kv* kv, const conduit_batch* bat
                                   const void* v_rows, void* stream);
 
 /*
+ * Gather and scatter in one launch (Sec. 3.5: the stale entries of the
+ * selected tokens are read out and replaced by their recomputed K/V): for
+ * every layer l, selected row i and KV head g,
+ *   k_old[l][i][g][:] = K[l][g][idx_i][:], then K[l][g][idx_i][:] = k_rows[l][i][g][:]
+ * (same for V). Equal to conduit_kv_gather followed by conduit_kv_scatter;
+ * the indices of a request must be distinct (conduit_select_topk's are),
+ * and k_old / v_old must not overlap k_rows / v_rows or the cache.
+ *  k_old, v_old    device [L][idx_off[R]][Hkv][d], dtype of kv (written)
+ *  k_rows, v_rows  device [L][idx_off[R]][Hkv][d], dtype of kv (read)
+ * Buffers are 16-byte aligned; errors as for conduit_kv_gather.
+ */
+conduit_status conduit_kv_exchange(const conduit_kv* kv, const conduit_batch* batch,
+                                   const int32_t* idx, const int32_t* idx_off,
+                                   const int32_t* idx_off_dev, void* k_old, void* v_old,
+                                   const void* k_rows, const void* v_rows, void* stream);
+
+/*
  * Causal attention of the refreshed rows over the patched cache (Sec. 3.1
  * and 4.3, selective recompute): for every layer l, selected row i at
  * position p_i = idx_i and query head h,

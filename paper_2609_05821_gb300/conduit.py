@@ -72,6 +72,7 @@ def _load():
         "conduit_select_topk_noalloc": (st, [P, P, P, ctypes.c_float, P, P, P, P, P, P, P, P]),
         "conduit_kv_gather": (st, [P, P, P, P, P, P, P, P]),
         "conduit_kv_scatter": (st, [P, P, P, P, P, P, P, P]),
+        "conduit_kv_exchange": (st, [P, P, P, P, P, P, P, P, P, P]),
         "conduit_refresh_workspace_size": (st, [P, P, P, ctypes.POINTER(SZ)]),
         "conduit_refresh_attn": (st, [P, P, P, P, P, P, P, P, SZ, P, P]),
         "conduit_launch_count": (ctypes.c_int64, []),
@@ -292,6 +293,14 @@ def conduit_kv_scatter(kv: KvCache, batch: Batch, idx, idx_off, idx_off_dev, k_r
                        stream=None):
     _check(_lib.conduit_kv_scatter(kv.ref(), batch.ref(), _ptr(idx), _ptr(idx_off),
                                    _ptr(idx_off_dev), _ptr(k_rows), _ptr(v_rows), _stream_ptr(stream)))
+
+
+def conduit_kv_exchange(kv: KvCache, batch: Batch, idx, idx_off, idx_off_dev, k_old, v_old,
+                        k_rows, v_rows, stream=None):
+    """Stale rows of the selected tokens into k_old / v_old, fresh rows into the cache."""
+    _check(_lib.conduit_kv_exchange(kv.ref(), batch.ref(), _ptr(idx), _ptr(idx_off),
+                                    _ptr(idx_off_dev), _ptr(k_old), _ptr(v_old), _ptr(k_rows),
+                                    _ptr(v_rows), _stream_ptr(stream)))
 
 
 def conduit_refresh_workspace_size(kv: KvCache, batch: Batch, idx_off) -> int:

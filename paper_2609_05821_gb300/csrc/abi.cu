@@ -179,6 +179,12 @@ ScoreLayout score_layout(const conduit_kv* kv, const conduit_batch* b, int n_lay
   return s;
 }
 
+int max_tokens(const conduit_batch* b) {
+  int m = 0;
+  for (int r = 0; r < b->num_requests; ++r) m = std::max(m, b->tok_off[r + 1] - b->tok_off[r]);
+  return m;
+}
+
 conduit_status check_workspace(void* ws, size_t have, size_t need) {
   if (need == 0) return CONDUIT_OK;
   if (!ws) return fail(CONDUIT_ERR_WORKSPACE, "workspace is NULL but %zu bytes are needed", need);
@@ -306,7 +312,7 @@ conduit_status conduit_select_topk(const conduit_batch* batch, const float* s, c
   size_t need = 0;
   conduit_select_workspace_size(batch, &need);
   if ((st = check_workspace(workspace, workspace_bytes, need))) return st;
-  cudaError_t err = launch_select(make_batch(batch), s, g, lambda, idx_off_dev, idx, mask, s_hat,
+  cudaError_t err = launch_select(make_batch(batch), max_tokens(batch), s, g, lambda, idx_off_dev, idx, mask, s_hat,
                                   coeff, static_cast<uint32_t*>(workspace), status,
                                   static_cast<cudaStream_t>(stream));
   if (err) return cuda_fail(err, "select");
@@ -329,7 +335,7 @@ conduit_status conduit_select_topk_noalloc(const conduit_batch* batch, const flo
     return fail(CONDUIT_ERR_UNSUPPORTED,
                 "batch has %lld tokens; the static scratch of conduit_select_topk_noalloc holds %d",
                 static_cast<long long>(n_tot), CONDUIT_NOALLOC_MAX_TOKENS);
-  cudaError_t err = launch_select_noalloc(make_batch(batch), s, g, lambda, idx_off_dev, idx, mask,
+  cudaError_t err = launch_select_noalloc(make_batch(batch), max_tokens(batch), s, g, lambda, idx_off_dev, idx, mask,
                                           s_hat, coeff, status, static_cast<cudaStream_t>(stream));
   if (err) return cuda_fail(err, "select_noalloc");
   return CONDUIT_OK;
@@ -337,20 +343,26 @@ conduit_status conduit_select_topk_noalloc(const conduit_batch* batch, const flo
 
 static conduit_status kv_copy(const conduit_kv* kv, const conduit_batch* batch,
                               const int32_t* idx, const int32_t* idx_off,
-                              const int32_t* idx_off_dev, const void* k_rows,
-                              const void* v_rows, bool scatter, void* stream) {
+                              const int32_t* idx_off_dev, void* rows_k, void* rows_v,
+                              const void* new_k, const void* new_v, int mode, void* stream) {
+  static const char* names[3] = {"kv_gather", "kv_scatter", "kv_exchange"};
   conduit_status st;
   if ((st = check_batch(batch)) || (st = check_kv(kv, batch))) return st;
   if ((st = check_selection(batch, idx_off, idx_off_dev, true, idx))) return st;
   const int n_sel = idx_off[batch->num_requests];
-  if (n_sel > 0 && (!k_rows || !v_rows))
-    return fail(CONDUIT_ERR_INVALID_ARG, "k_rows and v_rows are required");
-  if (n_sel > 0 && (!aligned16(k_rows) || !aligned16(v_rows)))
-    return fail(CONDUIT_ERR_INVALID_ARG, "k_rows and v_rows must be 16-byte aligned");
+  if (n_sel > 0 && (!rows_k || !rows_v))
+    return fail(CONDUIT_ERR_INVALID_ARG, "the K and V row buffers are required");
+  if (n_sel > 0 && (!aligned16(rows_k) || !aligned16(rows_v)))
+    return fail(CONDUIT_ERR_INVALID_ARG, "the K and V row buffers must be 16-byte aligned");
+  if (mode == 2 && n_sel > 0) {
+    if (!new_k || !new_v) return fail(CONDUIT_ERR_INVALID_ARG, "k_rows and v_rows are required");
+    if (!aligned16(new_k) || !aligned16(new_v))
+      return fail(CONDUIT_ERR_INVALID_ARG, "k_rows and v_rows must be 16-byte aligned");
+  }
   cudaError_t err = launch_kv_copy(make_kv(kv, batch), make_batch(batch), idx, idx_off_dev, n_sel,
-                                   max_budget(batch, idx_off), scatter, const_cast<void*>(k_rows),
-                                   const_cast<void*>(v_rows), static_cast<cudaStream_t>(stream));
-  if (err) return cuda_fail(err, scatter ? "kv_scatter" : "kv_gather");
+                                   max_budget(batch, idx_off), mode, rows_k, rows_v, new_k, new_v,
+                                   static_cast<cudaStream_t>(stream));
+  if (err) return cuda_fail(err, names[mode]);
   return CONDUIT_OK;
 }
 
@@ -358,14 +370,22 @@ conduit_status conduit_kv_gather(const conduit_kv* kv, const conduit_batch* batc
                                  const int32_t* idx, const int32_t* idx_off,
                                  const int32_t* idx_off_dev, void* k_rows, void* v_rows,
                                  void* stream) {
-  return kv_copy(kv, batch, idx, idx_off, idx_off_dev, k_rows, v_rows, false, stream);
+  return kv_copy(kv, batch, idx, idx_off, idx_off_dev, k_rows, v_rows, nullptr, nullptr, 0, stream);
 }
 
 conduit_status conduit_kv_scatter(const conduit_kv* kv, const conduit_batch* batch,
                                   const int32_t* idx, const int32_t* idx_off,
                                   const int32_t* idx_off_dev, const void* k_rows,
                                   const void* v_rows, void* stream) {
-  return kv_copy(kv, batch, idx, idx_off, idx_off_dev, k_rows, v_rows, true, stream);
+  return kv_copy(kv, batch, idx, idx_off, idx_off_dev, const_cast<void*>(k_rows),
+                 const_cast<void*>(v_rows), nullptr, nullptr, 1, stream);
+}
+
+conduit_status conduit_kv_exchange(const conduit_kv* kv, const conduit_batch* batch,
+                                   const int32_t* idx, const int32_t* idx_off,
+                                   const int32_t* idx_off_dev, void* k_old, void* v_old,
+                                   const void* k_rows, const void* v_rows, void* stream) {
+  return kv_copy(kv, batch, idx, idx_off, idx_off_dev, k_old, v_old, k_rows, v_rows, 2, stream);
 }
 
 conduit_status conduit_refresh_workspace_size(const conduit_kv* kv, const conduit_batch* batch,

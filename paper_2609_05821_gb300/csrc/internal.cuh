@@ -97,18 +97,24 @@ cudaError_t launch_score_tc(const KvDev& kv, const BatchDev& b, const int32_t* q
 cudaError_t launch_finalize(const float* pa, const float* ss, const BatchDev& b, int n_layers,
                             int Hkv, int Hq, int rg_max, int group_rows, int parts, int64_t n_tot, float* s,
                             float* attn_sum, float* g, int32_t* status, cudaStream_t stream);
-cudaError_t launch_select(const BatchDev& b, const float* s, const float* g, float lambda,
-                          const int32_t* idx_off_dev, int32_t* idx, uint8_t* mask, float* s_hat,
-                          float* coeff, uint32_t* keys, int32_t* status, cudaStream_t stream);
+// max_tokens: the largest request (picks how many keys a thread keeps in registers).
+cudaError_t launch_select(const BatchDev& b, int max_tokens, const float* s, const float* g,
+                          float lambda, const int32_t* idx_off_dev, int32_t* idx, uint8_t* mask,
+                          float* s_hat, float* coeff, uint32_t* keys, int32_t* status,
+                          cudaStream_t stream);
 // Same selection with the keys in the library's static device array.
 int64_t select_noalloc_max_tokens();
-cudaError_t launch_select_noalloc(const BatchDev& b, const float* s, const float* g, float lambda,
+cudaError_t launch_select_noalloc(const BatchDev& b, int max_tokens, const float* s, const float* g,
+                                  float lambda,
                                   const int32_t* idx_off_dev, int32_t* idx, uint8_t* mask,
                                   float* s_hat, float* coeff, int32_t* status,
                                   cudaStream_t stream);
+// mode 0: rows <- cache (gather); 1: cache <- rows (scatter); 2: rows <- cache,
+// then cache <- new (exchange).
 cudaError_t launch_kv_copy(const KvDev& kv, const BatchDev& b, const int32_t* idx,
-                           const int32_t* idx_off_dev, int32_t n_sel, int max_sel, bool scatter,
-                           void* k_rows, void* v_rows, cudaStream_t stream);
+                           const int32_t* idx_off_dev, int32_t n_sel, int max_sel, int mode,
+                           void* k_rows, void* v_rows, const void* k_new, const void* v_new,
+                           cudaStream_t stream);
 bool refresh_tc_supported(const KvDev& kv);
 cudaError_t launch_refresh_tc(const KvDev& kv, const BatchDev& b, const int32_t* idx,
                               const int32_t* idx_off_dev, const int32_t* idx_off_host, int32_t n_sel,

@@ -8,15 +8,17 @@
 // Keys stream in tiles of 128 (a tcgen05.mma costs about the same issue time
 // for N = 64 and N = 128, so wide tiles halve the instruction count).
 // Roles (320 threads):
-//   warp 0     one thread issues TMA loads of K tiles (three-stage ring) and
-//              V tiles (two stages)
+//   warp 0     one thread issues TMA loads of the query tiles (a 3-D box of
+//              64 dims x G heads x floor(128/G) rows lands in the tile's row
+//              order), then of K tiles (three-stage ring) and V tiles (two
+//              stages)
 //   warp 1     one thread issues tcgen05 MMAs. Per key tile t and query tile
 //              x: S_x(t) = Q_x K(t)^T into TMEM, then O_x += P_x(t) V(t) with
 //              P_x read from TMEM. S_x(t+1) overwrites the columns P_x(t)
 //              lives in, so it is issued only once P_x(t) V(t) has completed;
 //              the other tile's MMAs keep the tensor pipe busy meanwhile
-//   warps 2-5, 6-9   softmax of query tile 0 and 1: stage the query rows,
-//              then per key tile read S (one row per thread), apply the
+//   warps 2-5, 6-9   softmax of query tile 0 and 1: per key tile read S
+//              (one row per thread), apply the
 //              causal mask j <= p_i, keep a lazy running max (O and the row
 //              sum are rescaled only when the max grows by 2^8; warp-uniform,
 //              since tcgen05.ld/st are warp-collective), write P in bf16 pairs
@@ -24,8 +26,8 @@
 // TMEM: query tile x uses columns [256x, 256x + 128) for S (P in the upper 64
 // columns) and [256x + 128, 256x + 256) for O. When a softmax warp sees S_x(t),
 // O_x already holds P_x(t-1) V(t-1), so a rescale needs no further wait.
-// Rows are sorted by position, so a CTA needs keys up to its last row's
-// position only. Every wait is bounded by one second; a role that gives up
+// Rows are sorted by position, so each query tile needs keys up to its own
+// last row's position only. Every wait is bounded by one second; a role that gives up
 // raises an abort flag the others watch, the kernel sets CONDUIT_FLAG_TIMEOUT,
 // drains its copies and MMAs, and frees TMEM.
 #include <cuda.h>
@@ -143,7 +145,7 @@ __device__ __forceinline__ void load_tile(const RefArgs& a, const CUtensorMap* m
 
 __global__ void __launch_bounds__(kThreads, 1)
     refresh_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
-                      const __grid_constant__ RefArgs a) {
+                      const __grid_constant__ CUtensorMap qmap, const __grid_constant__ RefArgs a) {
   extern __shared__ uint8_t smem_raw[];
   const Smem s = carve(smem_raw);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -172,6 +174,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (p_max < 0) return;
   const int ntiles = p_max / kKT + 1;
   const int nq = cnt > a.rows_per_tile ? 2 : 1;   // query tiles in use (CTA-uniform)
+  // key tiles of each query tile (tile 0 holds the lower positions)
+  const int nt0 = nq == 1 ? ntiles : min(a.idx[i0 + a.rows_per_tile - 1], N - 1) / kKT + 1;
+  auto tiles_of = [&](int qi) { return qi == 0 ? nt0 : ntiles; };
+  const int qrows = a.rows_per_tile * G;          // rows the query box fills
 
   if (tid == 0) {
     for (int i = 0; i < kKStages; ++i) {
@@ -187,13 +193,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::mbar_init(&s.pfull[i], kSoftThreads);
       tc::mbar_init(&s.pvdone[i], 1);
     }
-    tc::mbar_init(s.qready, kTiles);
+    tc::mbar_init(s.qready, 1 + kTiles);  // the loader's expect-tx plus one per softmax group
     tc::mbar_init(s.mdone, 1);
     *s.abort = 0;
     for (int i = 0; i < 4; ++i) s.counters[i] = 0;
     tc::fence_barrier_init();
     tc::prefetch_tensormap(&kmap);
     tc::prefetch_tensormap(&vmap);
+    tc::prefetch_tensormap(&qmap);
   }
   if (warp == 1) tc::tmem_alloc(s.tmem_slot, kTmemCols);
   __syncthreads();
@@ -202,6 +209,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0 && lane == 0) {
     // ---------------------------------------------------------------- loads
+    tc::mbar_arrive_expect_tx(s.qready, uint32_t(nq) * 2u * 128u * uint32_t(qrows));
+    for (int qi = 0; qi < nq; ++qi)
+      for (int hf = 0; hf < 2; ++hf)
+        tc::tma_load_3d(s.q + qi * kQBytes + hf * kQHalf, &qmap, s.qready, hf * 64, g * G,
+                        l * a.n_sel + i0 + qi * a.rows_per_tile);
     uint32_t nk = 0, nv = 0;
     for (int t = 0; t < ntiles; ++t) {
       const int sk = t % kKStages;
@@ -254,6 +266,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         k_addr = tc::smem_u32(s.k + sk * kTileBytes);
       }
       for (int qi = 0; qi < nq && ok; ++qi) {
+        if (t >= tiles_of(qi)) continue;  // this query tile is done (tile nq-1 never is)
         if (!wait_or_abort(&s.pfull[qi], t & 1, s.abort)) { ok = false; break; }
         tc::tc_fence_after();
         const uint32_t tb = tmem + qi * kTileCols;
@@ -263,7 +276,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                           idesc_o, t > 0 || kk > 0);
         tc::mma_commit(&s.pvdone[qi]);
         if (qi == nq - 1) tc::mma_commit(&s.vempty[sv]);
-        if (more) {
+        if (more && t + 1 < tiles_of(qi)) {
           // S_qi(t+1) overwrites P_qi(t): wait until P_qi(t) V(t) has completed
           if (!wait_or_abort(&s.pvdone[qi], t & 1, s.abort)) { ok = false; break; }
           tc::tc_fence_after();
@@ -293,26 +306,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int h_row = g * G + (row_ok ? row % G : 0);
     int p_row = row_ok ? a.idx[i_row] : -1;
     if (p_row >= N) p_row = -1;
-    uint8_t* q_s = s.q + qi * kQBytes;
-    if (active) {  // query tile: row = (ti0 + row / G, head g*G + row % G), zero beyond tcnt * G
-      for (int base = 0; base < kRows * 16; base += kSoftThreads * 8) {
-        uint4 val[8];
-#pragma unroll
-        for (int u = 0; u < 8; ++u) {
-          const int x = base + u * kSoftThreads + et;
-          const int rr = x >> 4, ch = x & 15;
-          val[u] = make_uint4(0u, 0u, 0u, 0u);
-          if (rr < tcnt * G) {
-            const int ii = ti0 + rr / G, hh = g * G + rr % G;
-            val[u] = *reinterpret_cast<const uint4*>(a.q_rows + ((int64_t(l) * a.n_sel + ii) * Hq + hh) * kD + ch * 8);
-          }
-        }
-#pragma unroll
-        for (int u = 0; u < 8; ++u) {
-          const int x = base + u * kSoftThreads + et;
-          const int rr = x >> 4, ch = x & 15;
-          *reinterpret_cast<uint4*>(q_s + (ch >> 3) * kQHalf + tc::sw128_offset(rr, ch & 7)) = val[u];
-        }
+    if (active && qrows < kRows) {  // rows past the query box: zero (their S is masked anyway)
+      uint8_t* q_s = s.q + qi * kQBytes;
+      for (int x = et; x < (kRows - qrows) * 16; x += kSoftThreads) {
+        const int rr = qrows + (x >> 4), ch = x & 15;
+        *reinterpret_cast<uint4*>(q_s + (ch >> 3) * kQHalf + tc::sw128_offset(rr, ch & 7)) = make_uint4(0u, 0u, 0u, 0u);
       }
       tc::fence_proxy_async_smem();
     }
@@ -321,7 +319,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     bool ok = active;
     float m_ref = -INFINITY, lsum = 0.f;  // running max (scaled, log2 units) and row sum
-    for (int t = 0; t < ntiles && active; ++t) {
+    const int my_tiles = tiles_of(qi);
+    for (int t = 0; t < my_tiles && active; ++t) {
       // the tcgen05.ld below is warp-collective: the whole warp goes on or stops
       const bool got = __all_sync(0xffffffffu, ok && wait_or_abort(&s.sfull[qi], t & 1, s.abort));
       if (!got) {
@@ -402,8 +401,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     if (active) {
       // O is complete once the last P V of this tile has completed (phase
-      // ntiles-1 of pvdone; phase ntiles-2 completed before S(ntiles-1) was issued)
-      const bool fin = __all_sync(0xffffffffu, ok && wait_or_abort(&s.pvdone[qi], (ntiles - 1) & 1, s.abort));
+      // my_tiles-1 of pvdone; phase my_tiles-2 completed before S(my_tiles-1) was issued)
+      const bool fin = __all_sync(0xffffffffu, ok && wait_or_abort(&s.pvdone[qi], (my_tiles - 1) & 1, s.abort));
       if (!fin && ok) raise_abort(a, s, tc::kSiteFinal);
       if (fin) {
         tc::tc_fence_after();
@@ -477,6 +476,21 @@ bool make_map(CUtensorMap* m, const KvDev& kv, void* base) {
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Query rows [L * n_sel][Hq][d] as a 3-D map with box (64 dims, G heads,
+// rows_per_tile rows): one box fills one 64-dim half of a query tile in the
+// tile's row order (selected row major, head minor).
+bool make_qmap(CUtensorMap* m, const KvDev& kv, const void* q_rows, int32_t n_sel, int rows_per_tile) {
+  EncodeTiledFn enc = encode_fn();
+  if (!enc) return false;
+  cuuint64_t dims[3] = {cuuint64_t(kD), cuuint64_t(kv.Hq), cuuint64_t(kv.L) * cuuint64_t(n_sel)};
+  cuuint64_t strides[2] = {cuuint64_t(kD) * 2, cuuint64_t(kv.Hq) * kD * 2};
+  cuuint32_t box[3] = {64, cuuint32_t(kv.G), cuuint32_t(rows_per_tile)};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(q_rows), dims, strides, box,
+             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 }  // namespace
 
 bool refresh_tc_supported(const KvDev& kv) {
@@ -489,8 +503,10 @@ cudaError_t launch_refresh_tc(const KvDev& kv, const BatchDev& b, const int32_t*
                               const int32_t* idx_off_dev, const int32_t* idx_off_host, int32_t n_sel,
                               const void* q_rows, void* out, int32_t* status, cudaStream_t stream) {
   if (n_sel == 0) return cudaSuccess;
-  CUtensorMap kmap, vmap;
-  if (!make_map(&kmap, kv, kv.k) || !make_map(&vmap, kv, kv.v)) return cudaErrorInvalidValue;
+  CUtensorMap kmap, vmap, qmap;
+  if (!make_map(&kmap, kv, kv.k) || !make_map(&vmap, kv, kv.v) ||
+      !make_qmap(&qmap, kv, q_rows, n_sel, kRows / kv.G))
+    return cudaErrorInvalidValue;
   RefArgs a{};
   a.kv = kv;
   a.b = b;
@@ -513,7 +529,7 @@ cudaError_t launch_refresh_tc(const KvDev& kv, const BatchDev& b, const int32_t*
                                          int(kSmem));
   if (err) return err;
   const dim3 grid(blocks, kv.Hkv, kv.L);
-  refresh_tc_kernel<<<grid, kThreads, kSmem, stream>>>(kmap, vmap, a);
+  refresh_tc_kernel<<<grid, kThreads, kSmem, stream>>>(kmap, vmap, qmap, a);
   count_launches(1);
   return cudaGetLastError();
 }

@@ -45,6 +45,7 @@ __device__ __forceinline__ int block_exclusive_scan(int v, int* warp_s, int* tot
   return before;
 }
 
+template <int kRegKeys>  // keys a thread keeps in registers (0: keys in the workspace)
 __global__ void __launch_bounds__(kSelThreads) select_kernel(BatchDev b, const float* s,
                                                              const float* g, float lambda,
                                                              const int32_t* idx_off, int32_t* idx,
@@ -81,19 +82,39 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(BatchDev b, const f
   }
   __syncthreads();
 
-  // s_hat (Eq. 10) and its sortable key.
+  // s_hat (Eq. 10) and its sortable key. Each thread owns the contiguous
+  // tokens [lo, hi); up to kRegKeys of them stay in registers for the radix
+  // passes (requests of up to 1024 x kRegKeys tokens), otherwise the keys go
+  // through the workspace.
+  const int per = (N + kSelThreads - 1) / kSelThreads;
+  const int lo = min(N, int(threadIdx.x) * per), hi = min(N, lo + per);
+  const bool in_regs = kRegKeys > 0 && per <= kRegKeys;
+  uint32_t kr[kRegKeys > 0 ? kRegKeys : 1];
   bool bad = false;
-  for (int t = threadIdx.x; t < N; t += blockDim.x) {
-    int lo = 0, hi = K - 1;  // image of token t
-    while (lo < hi) {
-      const int mid = (lo + hi + 1) >> 1;
-      if (img_s[mid] <= t) lo = mid; else hi = mid - 1;
+  {
+    int img = 0;  // image of token lo
+    {
+      int a0 = 0, a1 = K - 1;
+      while (a0 < a1) {
+        const int mid = (a0 + a1 + 1) >> 1;
+        if (img_s[mid] <= lo) a0 = mid; else a1 = mid - 1;
+      }
+      img = a0;
     }
-    float sh = s[t0 + t] * c_s[lo];
-    if (!isfinite(sh) || sh < 0.f) bad = true;
-    if (sh == 0.f) sh = 0.f;  // -0 -> +0
-    if (s_hat) s_hat[t0 + t] = sh;
-    keys[t0 + t] = __float_as_uint(sh);
+    auto key_of = [&](int t) -> uint32_t {
+      while (img + 1 < K && img_s[img + 1] <= t) ++img;
+      float sh = s[t0 + t] * c_s[img];
+      if (!isfinite(sh) || sh < 0.f) bad = true;
+      if (sh == 0.f) sh = 0.f;  // -0 -> +0
+      if (s_hat) s_hat[t0 + t] = sh;
+      return __float_as_uint(sh);
+    };
+    if (in_regs) {
+#pragma unroll
+      for (int j = 0; j < kRegKeys; ++j) kr[j] = (lo + j < hi) ? key_of(lo + j) : 0u;
+    } else {
+      for (int t = lo; t < hi; ++t) keys[t0 + t] = key_of(t);
+    }
   }
   if (bad) flag_status(status, CONDUIT_FLAG_NONFINITE);
   __syncthreads();
@@ -114,9 +135,15 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(BatchDev b, const f
     for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0u;
     __syncthreads();
     const uint32_t prefix = prefix_s;
-    for (int t = threadIdx.x; t < N; t += blockDim.x) {
-      const uint32_t key = keys[t0 + t];
-      if ((key & pmask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+    if (in_regs) {
+#pragma unroll
+      for (int j = 0; j < kRegKeys; ++j)
+        if (lo + j < hi && (kr[j] & pmask) == prefix) atomicAdd(&hist[(kr[j] >> shift) & 255u], 1u);
+    } else {
+      for (int t = lo; t < hi; ++t) {
+        const uint32_t key = keys[t0 + t];
+        if ((key & pmask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+      }
     }
     __syncthreads();
     if (threadIdx.x < 32) {
@@ -154,20 +181,26 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(BatchDev b, const f
   const int need = remaining_s;  // keys equal to kth still to take, >= 1
 
   // Contiguous token ranges per thread keep the output in ascending order.
-  const int per = (N + kSelThreads - 1) / kSelThreads;
-  const int lo = min(N, int(threadIdx.x) * per), hi = min(N, lo + per);
   int gt = 0, eq = 0;
-  for (int t = lo; t < hi; ++t) {
-    const uint32_t key = keys[t0 + t];
-    gt += key > kth;
-    eq += key == kth;
+  if (in_regs) {
+#pragma unroll
+    for (int j = 0; j < kRegKeys; ++j)
+      if (lo + j < hi) {
+        gt += kr[j] > kth;
+        eq += kr[j] == kth;
+      }
+  } else {
+    for (int t = lo; t < hi; ++t) {
+      const uint32_t key = keys[t0 + t];
+      gt += key > kth;
+      eq += key == kth;
+    }
   }
   const int eq_base = block_exclusive_scan(eq, warp_s, nullptr);
   const int take_eq = max(0, min(eq, need - eq_base));
   const int pos0 = block_exclusive_scan(gt + take_eq, warp_s, nullptr);
   int pos = pos0, seen_eq = 0;
-  for (int t = lo; t < hi; ++t) {
-    const uint32_t key = keys[t0 + t];
+  auto emit = [&](int t, uint32_t key) {
     bool sel = key > kth;
     if (key == kth) {
       sel = seen_eq < take_eq;
@@ -175,6 +208,13 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(BatchDev b, const f
     }
     if (sel) out[pos++] = t;
     if (mask) mask[t0 + t] = sel ? 1 : 0;
+  };
+  if (in_regs) {
+#pragma unroll
+    for (int j = 0; j < kRegKeys; ++j)
+      if (lo + j < hi) emit(lo + j, kr[j]);
+  } else {
+    for (int t = lo; t < hi; ++t) emit(t, keys[t0 + t]);
   }
 }
 
@@ -193,7 +233,8 @@ std::mutex g_noalloc_mu;
 
 int64_t select_noalloc_max_tokens() { return kNoAllocMaxTokens; }
 
-cudaError_t launch_select_noalloc(const BatchDev& b, const float* s, const float* g, float lambda,
+cudaError_t launch_select_noalloc(const BatchDev& b, int max_tokens, const float* s, const float* g,
+                                  float lambda,
                                   const int32_t* idx_off_dev, int32_t* idx, uint8_t* mask,
                                   float* s_hat, float* coeff, int32_t* status,
                                   cudaStream_t stream) {
@@ -214,15 +255,24 @@ cudaError_t launch_select_noalloc(const BatchDev& b, const float* s, const float
     }
     keys = g_noalloc_ptr[dev];
   }
-  return launch_select(b, s, g, lambda, idx_off_dev, idx, mask, s_hat, coeff, keys, status,
-                       stream);
+  return launch_select(b, max_tokens, s, g, lambda, idx_off_dev, idx, mask, s_hat, coeff, keys,
+                       status, stream);
 }
 
-cudaError_t launch_select(const BatchDev& b, const float* s, const float* g, float lambda,
-                          const int32_t* idx_off_dev, int32_t* idx, uint8_t* mask, float* s_hat,
-                          float* coeff, uint32_t* keys, int32_t* status, cudaStream_t stream) {
-  select_kernel<<<b.R, kSelThreads, 0, stream>>>(b, s, g, lambda, idx_off_dev, idx, mask, s_hat,
-                                                 coeff, keys, status);
+cudaError_t launch_select(const BatchDev& b, int max_tokens, const float* s, const float* g,
+                          float lambda, const int32_t* idx_off_dev, int32_t* idx, uint8_t* mask,
+                          float* s_hat, float* coeff, uint32_t* keys, int32_t* status,
+                          cudaStream_t stream) {
+  // the smallest register budget that holds every request's keys
+  if (max_tokens <= kSelThreads)
+    select_kernel<1><<<b.R, kSelThreads, 0, stream>>>(b, s, g, lambda, idx_off_dev, idx, mask, s_hat,
+                                                      coeff, keys, status);
+  else if (max_tokens <= 8 * kSelThreads)
+    select_kernel<8><<<b.R, kSelThreads, 0, stream>>>(b, s, g, lambda, idx_off_dev, idx, mask, s_hat,
+                                                      coeff, keys, status);
+  else
+    select_kernel<0><<<b.R, kSelThreads, 0, stream>>>(b, s, g, lambda, idx_off_dev, idx, mask, s_hat,
+                                                      coeff, keys, status);
   count_launches(1);
   return cudaGetLastError();
 }

@@ -3,9 +3,9 @@
 ``RefreshPipeline.step()`` enqueues, on one CUDA stream and through the C ABI:
   1. conduit_score        scoring pass over the reused visual cache (Eqs. 6-8)
   2. conduit_select_topk  amplification + one global top-k per request (Eqs. 9-11)
-  3. conduit_kv_gather    stale K/V rows of the selected tokens
-  4. conduit_kv_scatter   fresh K/V rows written into the cache
-  5. conduit_refresh_attn causal attention of the refreshed rows over the patched cache
+  3. conduit_kv_exchange  stale K/V rows of the selected tokens out, fresh rows in
+                          (conduit_kv_gather + conduit_kv_scatter in one launch)
+  4. conduit_refresh_attn causal attention of the refreshed rows over the patched cache
 All buffers are allocated once at construction, so a step allocates nothing
 and can be captured in a CUDA graph (``capture()``). ``step_from_host()`` is
 the end-to-end form: it copies the step's inputs from pinned host memory,
@@ -77,10 +77,8 @@ class RefreshPipeline:
                               self.status, stream)
 
     def refresh(self, stream=None):
-        C.conduit_kv_gather(self.kv, self.batch, self.idx, self.idx_off, self.idx_off_dev,
-                            self.k_old, self.v_old, stream)
-        C.conduit_kv_scatter(self.kv, self.batch, self.idx, self.idx_off, self.idx_off_dev,
-                             self.k_rows, self.v_rows, stream)
+        C.conduit_kv_exchange(self.kv, self.batch, self.idx, self.idx_off, self.idx_off_dev,
+                              self.k_old, self.v_old, self.k_rows, self.v_rows, stream)
         C.conduit_refresh_attn(self.kv, self.batch, self.idx, self.idx_off, self.idx_off_dev,
                                self.q_rows, self.out, self.ws_ref, self.status, stream)
 

@@ -137,6 +137,8 @@ def test_kv_copy_and_refresh_reject_bad_arguments(C):
     bad_off = torch.tensor([1, 3, 7], dtype=torch.int32)
     _expect(C, C.ERR_INVALID_ARG, C.conduit_kv_scatter, kv, b, idx, bad_off, off_d, rows, rows)
     _expect(C, C.ERR_INVALID_ARG, C.conduit_kv_gather, kv, b, idx, off, None, rows, rows)
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_kv_exchange, kv, b, idx, off, off_d, rows, rows, None, rows)
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_kv_exchange, kv, b, idx, bad_off, off_d, rows, rows, rows, rows)
     _expect(C, C.ERR_INVALID_ARG, C.conduit_refresh_attn, kv, b, None, off, off_d, rows)
     paged = torch.zeros((2, 8, 2, 16, 64), dtype=torch.bfloat16)
     table = torch.zeros((2, 3), dtype=torch.int32)      # 3 pages x 16 < 64 tokens

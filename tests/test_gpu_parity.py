@@ -295,6 +295,27 @@ def test_index_driven_refresh_with_oracle_indices(C, P):
     _patched_equals_scatter(C, pipe, inputs)
 
 
+@pytest.mark.parametrize("paged", [False, True])
+def test_exchange_equals_gather_then_scatter(C, P, paged):
+    """conduit_kv_exchange (the pipeline's call) against conduit_kv_gather
+    followed by conduit_kv_scatter on a copy of the cache: bitwise."""
+    inputs = synth.make_inputs(synth.workload("batched" if paged else "multi",
+                                              **({"num_requests": 3} if paged else {})), device="cuda")
+    a = P.from_inputs({**inputs, "k": inputs["k"].clone(), "v": inputs["v"].clone()})
+    b = P.from_inputs({**inputs, "k": inputs["k"].clone(), "v": inputs["v"].clone()})
+    a.score_select()
+    b.score_select()
+    C.conduit_kv_exchange(a.kv, a.batch, a.idx, a.idx_off, a.idx_off_dev, a.k_old, a.v_old,
+                          a.k_rows, a.v_rows)
+    C.conduit_kv_gather(b.kv, b.batch, b.idx, b.idx_off, b.idx_off_dev, b.k_old, b.v_old)
+    C.conduit_kv_scatter(b.kv, b.batch, b.idx, b.idx_off, b.idx_off_dev, b.k_rows, b.v_rows)
+    torch.cuda.synchronize()
+    assert torch.equal(a.idx, b.idx)
+    for x, y in ((a.k_old, b.k_old), (a.v_old, b.v_old), (a.kv.k, b.kv.k), (a.kv.v, b.kv.v)):
+        assert torch.equal(x, y)
+    assert not torch.equal(a.k_old, a.k_rows)  # the stale rows differ from the fresh ones
+
+
 def test_refresh_late_max_jump_in_some_heads(C, P):
     """Rows whose running max jumps far (> 2^8) at a late key tile while other
     rows of the same warp do not: the lazy O rescale must stay correct."""
