@@ -230,6 +230,12 @@ __device__ __forceinline__ void stage_rows(const TcArgs& a, const Unit& w, uint8
   }
 }
 
+// 2^(s scale + b) for a pair of accumulator values (one packed FMA, two MUFU ops).
+__device__ __forceinline__ float2 exp2_pair(float s0, float s1, float2 sc2, float2 b2, int) {
+  const float2 y = tc::ffma2(make_float2(s0, s1), sc2, b2);
+  return make_float2(tc::ex2(y.x), tc::ex2(y.y));
+}
+
 // Online row statistics over NC accumulator columns of which the first
 // `valid` are tokens of the slab: running max m (raw logit) and
 // z = sum 2^((S - m) scale). Only a ragged last tile takes the masked path.
@@ -246,29 +252,29 @@ __device__ __forceinline__ void row_stats(float (&v)[NC], int valid, float scale
   for (int x = 0; x < NC; ++x) cm[x & 3] = fmaxf(cm[x & 3], v[x]);
   const float mn = fmaxf(m, fmaxf(fmaxf(cm[0], cm[1]), fmaxf(cm[2], cm[3])));
   if (mn == -INFINITY) return;
-  const float nb = -mn * scale;
-  float ac[4] = {0.f, 0.f, 0.f, 0.f};
+  const float2 sc2 = make_float2(scale, scale), nb2 = make_float2(-mn * scale, -mn * scale);
+  float2 ac[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
 #pragma unroll
-  for (int x = 0; x < NC; ++x) ac[x & 3] += tc::ex2(fmaf(v[x], scale, nb));
-  z = z * tc::ex2((m - mn) * scale) + ((ac[0] + ac[1]) + (ac[2] + ac[3]));
+  for (int x = 0; x < NC / 2; ++x) ac[x & 1] = tc::fadd2(ac[x & 1], exp2_pair(v[2 * x], v[2 * x + 1], sc2, nb2, x));
+  z = z * tc::ex2((m - mn) * scale) + ((ac[0].x + ac[0].y) + (ac[1].x + ac[1].y));
   m = mn;
 }
 
-// Sum over NC accumulator columns (scoring rows c0 ...) of 2^(S scale - lse_row).
-// Columns past the row group carry lse = +inf and add exactly zero (the
-// accumulator columns there hold finite values: TMEM is zeroed at start).
+// Sum over NC accumulator columns (scoring rows c0 ...) of 2^(S scale - lse_row),
+// given nlse = -lse. Columns past the row group carry nlse = -inf and add
+// exactly zero (the accumulator columns there hold finite values: TMEM is
+// zeroed at start).
 template <int NC>
-__device__ __forceinline__ float col_sum(const float (&v)[NC], const float* lse, float scale) {
-  float ac[4] = {0.f, 0.f, 0.f, 0.f};
+__device__ __forceinline__ float col_sum(const float (&v)[NC], const float* nlse, float scale) {
+  const float2 sc2 = make_float2(scale, scale);
+  float2 ac[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
 #pragma unroll
   for (int x4 = 0; x4 < NC / 4; ++x4) {
-    const float4 lv = reinterpret_cast<const float4*>(lse)[x4];
-    ac[0] += tc::ex2(fmaf(v[4 * x4 + 0], scale, -lv.x));
-    ac[1] += tc::ex2(fmaf(v[4 * x4 + 1], scale, -lv.y));
-    ac[2] += tc::ex2(fmaf(v[4 * x4 + 2], scale, -lv.z));
-    ac[3] += tc::ex2(fmaf(v[4 * x4 + 3], scale, -lv.w));
+    const float4 lv = reinterpret_cast<const float4*>(nlse)[x4];
+    ac[0] = tc::fadd2(ac[0], exp2_pair(v[4 * x4 + 0], v[4 * x4 + 1], sc2, make_float2(lv.x, lv.y), 2 * x4));
+    ac[1] = tc::fadd2(ac[1], exp2_pair(v[4 * x4 + 2], v[4 * x4 + 3], sc2, make_float2(lv.z, lv.w), 2 * x4 + 1));
   }
-  return (ac[0] + ac[1]) + (ac[2] + ac[3]);
+  return (ac[0].x + ac[0].y) + (ac[1].x + ac[1].y);
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
@@ -478,11 +484,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (tok < w.N) ss_out[tok] = (sq[0] + sq[1]) + (sq[2] + sq[3]);
         }
       }
-      // log2-sum-exp of each row, shared with the token-owning threads of pass B
-      // (+inf past the row group: those columns then add zero)
+      // minus the log2-sum-exp of each row, shared with the token-owning
+      // threads of pass B (-inf past the row group: those columns add nothing)
       {
         const int row = (do_rows ? rb : 1) * 128 + lrow;
-        s.lse[row] = (do_rows && row < w.rows) ? m * a.scale_log2 + log2f(z) : INFINITY;
+        s.lse[row] = (do_rows && row < w.rows) ? -(m * a.scale_log2 + log2f(z)) : -INFINITY;
       }
       epi_barrier();
       // pass B share: 32-row chunks [cb0, cb1)
