@@ -17,9 +17,9 @@
 //
 // Pass B walks the tiles in reverse so the most recent K tiles of pass A are
 // still in L2. Roles (320 threads):
-//   warp 0       one thread issues TMA loads of K tiles (128 tokens x 128
-//                dims, 128-byte swizzle) into a three-stage ring, and of the
-//                matching V tiles into two buffers during pass A
+//   warp 0       lane 0 issues TMA loads of K tiles (128 tokens x 128 dims,
+//                128-byte swizzle) into a three-stage ring; lane 1 loads the
+//                matching V tiles of pass A into two buffers
 //   warp 1       one thread issues tcgen05 MMAs into two 256-column TMEM
 //                accumulator slots (it also owns the TMEM allocation)
 //   warps 2-9    epilogue, two warps per TMEM lane quarter (warp group h
@@ -310,8 +310,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = *s.tmem_slot;
 
   if (warp == 0 && lane == 0) {
-    // ------------------------------------------------------------ producer
-    uint32_t seq = 0, vseq = 0;
+    // ---------------------------------------------------------- producer: K
+    uint32_t seq = 0;
     bool ok = true;
     for (int u = blockIdx.x; u < a.n_units && ok; u += gridDim.x) {
       Unit w;
@@ -324,20 +324,28 @@ __global__ void __launch_bounds__(kThreads, 1)
           break;
         }
         load_k_tile(a, &kmap, w, s.k + st * kStageBytes, &s.kfull[st], tile_of(w, i));
-        if (i < w.tiles && w.rg == 0) {  // V tile for the value norms, read by the epilogue in pass A
-          const int vb = vseq % kVBufs;
-          if (!wait_or_abort(&s.vempty[vb], ((vseq / kVBufs) & 1) ^ 1, s.abort)) {
-            if (!*s.abort) raise_abort(a, s, tc::kSiteLoad);
-            ok = false;
-            ++seq;
-            break;
-          }
-          load_k_tile(a, &vmap, w, s.v + vb * kStageBytes, &s.vfull[vb], i);
-          ++vseq;
-        }
       }
     }
     s.counters[0] = seq;
+  } else if (warp == 0 && lane == 1) {
+    // ---------------------------------------------------------- producer: V
+    // V tiles of pass 1 for the value norms, on a thread of their own so that
+    // a V tile waiting for its buffer never holds back the K ring
+    uint32_t vseq = 0;
+    bool ok = true;
+    for (int u = blockIdx.x; u < a.n_units && ok; u += gridDim.x) {
+      Unit w;
+      if (!decode_unit(a, u, w) || w.rg != 0) continue;
+      for (int i = 0; i < w.tiles; ++i, ++vseq) {
+        const int vb = vseq % kVBufs;
+        if (!wait_or_abort(&s.vempty[vb], ((vseq / kVBufs) & 1) ^ 1, s.abort)) {
+          if (!*s.abort) raise_abort(a, s, tc::kSiteLoad);
+          ok = false;
+          break;
+        }
+        load_k_tile(a, &vmap, w, s.v + vb * kStageBytes, &s.vfull[vb], i);
+      }
+    }
     s.counters[2] = vseq;
   } else if (warp == 1 && lane == 0) {
     // ----------------------------------------------------------------- MMA
