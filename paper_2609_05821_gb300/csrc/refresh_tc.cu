@@ -2,34 +2,31 @@
 // (selective recompute, Conduit Sec. 3.1 / 4.3):
 //   out[l][i][h] = sum_{j <= p_i} softmax_j(<q[l][i][h], K'[l][h/G][j]> / sqrt(d)) V'[l][h/G][j]
 //
-// One CTA owns up to two query tiles of 128 rows of one (layer, KV head,
-// request); a tile holds floor(128/G) consecutive selected rows times the G
-// query heads that share the KV head, and both tiles share every K/V tile.
-// Keys stream in tiles of 128 (a tcgen05.mma costs about the same issue time
-// for N = 64 and N = 128, so wide tiles halve the instruction count).
-// Roles (320 threads):
-//   warp 0     one thread issues TMA loads of the query tiles (a 3-D box of
-//              64 dims x G heads x floor(128/G) rows lands in the tile's row
-//              order), then of K tiles (three-stage ring) and V tiles (two
-//              stages)
-//   warp 1     one thread issues tcgen05 MMAs. Per key tile t and query tile
-//              x: S_x(t) = Q_x K(t)^T into TMEM, then O_x += P_x(t) V(t) with
-//              P_x read from TMEM. S_x(t+1) overwrites the columns P_x(t)
-//              lives in, so it is issued only once P_x(t) V(t) has completed;
-//              the other tile's MMAs keep the tensor pipe busy meanwhile
-//   warps 2-5, 6-9   softmax of query tile 0 and 1: per key tile read S
-//              (one row per thread), apply the
-//              causal mask j <= p_i, keep a lazy running max (O and the row
-//              sum are rescaled only when the max grows by 2^8; warp-uniform,
-//              since tcgen05.ld/st are warp-collective), write P in bf16 pairs
-//              over the upper half of S, and finally write O / rowsum in bf16
-// TMEM: query tile x uses columns [256x, 256x + 128) for S (P in the upper 64
-// columns) and [256x + 128, 256x + 256) for O. When a softmax warp sees S_x(t),
-// O_x already holds P_x(t-1) V(t-1), so a rescale needs no further wait.
-// Rows are sorted by position, so each query tile needs keys up to its own
-// last row's position only. Every wait is bounded by one second; a role that gives up
-// raises an abort flag the others watch, the kernel sets CONDUIT_FLAG_TIMEOUT,
-// drains its copies and MMAs, and frees TMEM.
+// One CTA owns one query tile of 128 rows of one (layer, KV head, request):
+// floor(128/G) consecutive selected rows times the G query heads that share
+// the KV head. Keys stream in tiles of 128 (a tcgen05.mma costs about the same
+// issue time for N = 64 and N = 128, so wide tiles halve the instruction
+// count). Roles (320 threads):
+//   warp 0     one thread issues TMA loads: the query tile (a 3-D box of 64
+//              dims x G heads x floor(128/G) rows lands in the tile's row
+//              order), then K tiles (three-stage ring) and V tiles (two stages)
+//   warp 1     one thread issues tcgen05 MMAs: S(t) = Q K(t)^T into one of two
+//              TMEM buffers, O += P(t) V(t) with P read from TMEM
+//   warps 2-9  softmax, two warps per TMEM lane quarter: each thread owns one
+//              row and one half (64 keys) of every key tile. Per tile it reads
+//              its half of S(t), applies the causal mask j <= p_i, exchanges
+//              the half-row max with its partner through shared memory, keeps
+//              a lazy running max (O and the row sum are rescaled only when
+//              the max grows by 2^8; warp-uniform, since tcgen05.ld/st are
+//              warp-collective), writes its half of P as bf16 pairs over the
+//              upper half of S(t), and finally writes its half of O / rowsum
+// TMEM: S buffers at columns [0, 128) and [128, 256) (P in the upper 64 of
+// each), O at [256, 384). S(t+1) is computed while the softmax works on
+// S(t); S(t+2) reuses the buffer of P(t), so it is issued once P(t) V(t) has
+// completed. Rows are sorted by position, so the tile needs keys up to its
+// last row's position only. Every wait is bounded by one second; a role that
+// gives up raises an abort flag the others watch, the kernel sets
+// CONDUIT_FLAG_TIMEOUT, drains its copies and MMAs, and frees TMEM.
 #include <cuda.h>
 
 #include "internal.cuh"
@@ -41,20 +38,19 @@ namespace {
 constexpr int kD = 128;
 constexpr int kKT = 128;                         // keys per tile
 constexpr int kRows = 128;                       // rows per query tile
-constexpr int kTiles = 2;                        // query tiles per CTA
-constexpr int kSoftThreads = 128;
-constexpr int kThreads = 64 + kTiles * kSoftThreads;
+constexpr int kSoftThreads = 256;
+constexpr int kThreads = 64 + kSoftThreads;
 constexpr int kKStages = 3;
 constexpr int kVStages = 2;
-constexpr uint32_t kQHalf = kRows * 128;         // 16 KB: one 64-dim half of a query tile
+constexpr uint32_t kQHalf = kRows * 128;         // 16 KB: one 64-dim half of the query tile
 constexpr uint32_t kQBytes = 2 * kQHalf;         // 32 KB
 constexpr uint32_t kTileHalf = kKT * 128;        // 16 KB: one 64-dim half of a K or V tile
 constexpr uint32_t kTileBytes = 2 * kTileHalf;   // 32 KB
-constexpr uint32_t kSmem = 1024 + kTiles * kQBytes + (kKStages + kVStages) * kTileBytes + 256;
-constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kTileCols = 256;              // TMEM columns per query tile
+constexpr uint32_t kSmem = 1024 + kQBytes + (kKStages + kVStages) * kTileBytes + 256 + 2 * 2 * 128 * 4 + 2 * 128 * 4;
+constexpr uint32_t kTmemCols = 512;              // 384 used; allocations are powers of two
+constexpr uint32_t kSCols = 128;                 // one S buffer
 constexpr uint32_t kPCol = 64;                   // P (bf16 pairs) over the upper half of S
-constexpr uint32_t kOCol = 128;                  // O offset inside a tile's columns
+constexpr uint32_t kOCol = 256;                  // O
 constexpr float kRescaleLog2 = 8.f;
 
 struct RefArgs {
@@ -72,23 +68,26 @@ struct RefArgs {
 };
 
 struct Smem {
-  uint8_t* q;        // [kTiles][2 halves][128 rows][128 B]
+  uint8_t* q;        // [2 halves][128 rows][128 B]
   uint8_t* k;        // [kKStages][2 halves][128 keys][128 B]
   uint8_t* v;        // [kVStages][2 halves][128 keys][128 B]
-  uint64_t *kfull, *kempty;           // [kKStages]
-  uint64_t *vfull, *vempty;           // [kVStages]
-  uint64_t *sfull, *pfull, *pvdone;   // [kTiles]
+  uint64_t *kfull, *kempty;   // [kKStages]
+  uint64_t *vfull, *vempty;   // [kVStages]
+  uint64_t *sfull, *pfull;    // [2] per S buffer
+  uint64_t *pvdone;           // once per key tile
   uint64_t *qready, *mdone;
   uint32_t* tmem_slot;
   volatile int* abort;
   uint32_t* counters;  // [0] K loads, [1] V loads, [2] K consumed, [3] V consumed
+  float* xmax;         // [2 tile parities][2 halves][128 rows] half-row maxima
+  float* xsum;         // [2 halves][128 rows] half-row sums at the end
 };
 
 __device__ __forceinline__ Smem carve(uint8_t* raw) {
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(raw) + 1023) & ~uintptr_t(1023));
   Smem s;
   s.q = base;
-  s.k = s.q + kTiles * kQBytes;
+  s.k = s.q + kQBytes;
   s.v = s.k + kKStages * kTileBytes;
   uint64_t* bar = reinterpret_cast<uint64_t*>(s.v + kVStages * kTileBytes);
   s.kfull = bar;
@@ -96,13 +95,15 @@ __device__ __forceinline__ Smem carve(uint8_t* raw) {
   s.vfull = s.kempty + kKStages;
   s.vempty = s.vfull + kVStages;
   s.sfull = s.vempty + kVStages;
-  s.pfull = s.sfull + kTiles;
-  s.pvdone = s.pfull + kTiles;
-  s.qready = s.pvdone + kTiles;
+  s.pfull = s.sfull + 2;
+  s.pvdone = s.pfull + 2;
+  s.qready = s.pvdone + 1;
   s.mdone = s.qready + 1;
   s.tmem_slot = reinterpret_cast<uint32_t*>(s.mdone + 1);
   s.abort = reinterpret_cast<volatile int*>(s.tmem_slot + 1);
   s.counters = reinterpret_cast<uint32_t*>(s.tmem_slot + 2);
+  s.xmax = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bar) + 256);
+  s.xsum = s.xmax + 2 * 2 * 128;
   return s;
 }
 
@@ -154,7 +155,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int G = kv.G, Hq = kv.Hq;
 
   // CTA -> (request, first selected row, row count); larger positions first
-  const int span = kTiles * a.rows_per_tile;
+  const int span = a.rows_per_tile;
   int blk = a.n_blocks - 1 - int(blockIdx.x);
   int r = 0, i0 = -1, cnt = 0;
   for (int rr = 0; rr < a.b.R; ++rr) {
@@ -173,10 +174,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int p_max = min(a.idx[i0 + cnt - 1], N - 1);
   if (p_max < 0) return;
   const int ntiles = p_max / kKT + 1;
-  const int nq = cnt > a.rows_per_tile ? 2 : 1;   // query tiles in use (CTA-uniform)
-  // key tiles of each query tile (tile 0 holds the lower positions)
-  const int nt0 = nq == 1 ? ntiles : min(a.idx[i0 + a.rows_per_tile - 1], N - 1) / kKT + 1;
-  auto tiles_of = [&](int qi) { return qi == 0 ? nt0 : ntiles; };
   const int qrows = a.rows_per_tile * G;          // rows the query box fills
 
   if (tid == 0) {
@@ -188,12 +185,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::mbar_init(&s.vfull[i], 1);
       tc::mbar_init(&s.vempty[i], 1);
     }
-    for (int i = 0; i < kTiles; ++i) {
+    for (int i = 0; i < 2; ++i) {
       tc::mbar_init(&s.sfull[i], 1);
+      // per buffer, so the softmax can never be two phases ahead of the MMA's
+      // wait: P(t+2) needs S(t+2), issued only after the wait for P(t)
       tc::mbar_init(&s.pfull[i], kSoftThreads);
-      tc::mbar_init(&s.pvdone[i], 1);
     }
-    tc::mbar_init(s.qready, 1 + kTiles);  // the loader's expect-tx plus one per softmax group
+    tc::mbar_init(s.pvdone, 1);
+    tc::mbar_init(s.qready, 2);  // the loader's expect-tx plus the softmax warps
     tc::mbar_init(s.mdone, 1);
     *s.abort = 0;
     for (int i = 0; i < 4; ++i) s.counters[i] = 0;
@@ -209,11 +208,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0 && lane == 0) {
     // ---------------------------------------------------------------- loads
-    tc::mbar_arrive_expect_tx(s.qready, uint32_t(nq) * 2u * 128u * uint32_t(qrows));
-    for (int qi = 0; qi < nq; ++qi)
-      for (int hf = 0; hf < 2; ++hf)
-        tc::tma_load_3d(s.q + qi * kQBytes + hf * kQHalf, &qmap, s.qready, hf * 64, g * G,
-                        l * a.n_sel + i0 + qi * a.rows_per_tile);
+    tc::mbar_arrive_expect_tx(s.qready, 2u * 128u * uint32_t(qrows));
+    for (int hf = 0; hf < 2; ++hf)
+      tc::tma_load_3d(s.q + hf * kQHalf, &qmap, s.qready, hf * 64, g * G, l * a.n_sel + i0);
     uint32_t nk = 0, nv = 0;
     for (int t = 0; t < ntiles; ++t) {
       const int sk = t % kKStages;
@@ -232,57 +229,45 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t ck = 0, cv = 0;
     const uint32_t idesc_s = tc::idesc_bf16(kRows, kKT);
     const uint32_t idesc_o = tc::idesc_bf16(kRows, kD, /*b_mn_major=*/true);
-    auto issue_s = [&](int qi, uint32_t k_addr) {  // S_qi = Q_qi K^T
-      const uint32_t q_addr = tc::smem_u32(s.q + qi * kQBytes);
+    const uint32_t q_addr = tc::smem_u32(s.q);
+    // S(t) = Q K(t)^T into S buffer t & 1
+    auto issue_s = [&](int t) -> bool {
+      const int sk = t % kKStages;
+      if (!wait_or_abort(&s.kfull[sk], (t / kKStages) & 1, s.abort)) return false;
+      ++ck;
+      tc::tc_fence_after();
+      const uint32_t k_addr = tc::smem_u32(s.k + sk * kTileBytes);
 #pragma unroll
       for (int kk = 0; kk < 8; ++kk) {
         const uint32_t off = (kk & 3) * 32;
-        tc::mma_bf16(tmem + qi * kTileCols, tc::desc_sw128(q_addr + (kk >> 2) * kQHalf + off),
+        tc::mma_bf16(tmem + uint32_t(t & 1) * kSCols, tc::desc_sw128(q_addr + (kk >> 2) * kQHalf + off),
                      tc::desc_sw128(k_addr + (kk >> 2) * kTileHalf + off), idesc_s, kk > 0);
       }
-      tc::mma_commit(&s.sfull[qi]);
+      tc::mma_commit(&s.sfull[t & 1]);
+      tc::mma_commit(&s.kempty[sk]);
+      return true;
     };
-    bool ok = wait_or_abort(s.qready, 0, s.abort) && wait_or_abort(&s.kfull[0], 0, s.abort);
-    if (ok) {
-      ++ck;
-      tc::tc_fence_after();
-      for (int qi = 0; qi < nq; ++qi) issue_s(qi, tc::smem_u32(s.k));
-      tc::mma_commit(&s.kempty[0]);
-    }
-    // Per key tile t and query tile x in turn: O_x += P_x(t) V(t), then
-    // S_x(t+1) once that has completed. Query tile 1's softmax runs while
-    // tile 0's MMAs execute and vice versa (ping-pong).
+    bool ok = wait_or_abort(s.qready, 0, s.abort);
+    if (ok) ok = issue_s(0);
+    if (ok && ntiles > 1) ok = issue_s(1);
     for (int t = 0; t < ntiles && ok; ++t) {
       const int sv = t % kVStages;
       if (!wait_or_abort(&s.vfull[sv], (t / kVStages) & 1, s.abort)) { ok = false; break; }
       ++cv;
+      if (!wait_or_abort(&s.pfull[t & 1], (t >> 1) & 1, s.abort)) { ok = false; break; }
+      tc::tc_fence_after();
       const uint32_t v_addr = tc::smem_u32(s.v + sv * kTileBytes);
-      const bool more = t + 1 < ntiles;
-      const int sk = (t + 1) % kKStages;
-      uint32_t k_addr = 0;
-      if (more) {
-        if (!wait_or_abort(&s.kfull[sk], ((t + 1) / kKStages) & 1, s.abort)) { ok = false; break; }
-        ++ck;
-        k_addr = tc::smem_u32(s.k + sk * kTileBytes);
-      }
-      for (int qi = 0; qi < nq && ok; ++qi) {
-        if (t >= tiles_of(qi)) continue;  // this query tile is done (tile nq-1 never is)
-        if (!wait_or_abort(&s.pfull[qi], t & 1, s.abort)) { ok = false; break; }
-        tc::tc_fence_after();
-        const uint32_t tb = tmem + qi * kTileCols;
+      const uint32_t pb = tmem + uint32_t(t & 1) * kSCols + kPCol;
 #pragma unroll
-        for (int kk = 0; kk < kKT / 16; ++kk)  // O_qi += P_qi V
-          tc::mma_bf16_ts(tb + kOCol, tb + kPCol + kk * 8, tc::desc_sw128_mn(v_addr + kk * 2048, kTileHalf),
-                          idesc_o, t > 0 || kk > 0);
-        tc::mma_commit(&s.pvdone[qi]);
-        if (qi == nq - 1) tc::mma_commit(&s.vempty[sv]);
-        if (more && t + 1 < tiles_of(qi)) {
-          // S_qi(t+1) overwrites P_qi(t): wait until P_qi(t) V(t) has completed
-          if (!wait_or_abort(&s.pvdone[qi], t & 1, s.abort)) { ok = false; break; }
-          tc::tc_fence_after();
-          issue_s(qi, k_addr);
-          if (qi == nq - 1) tc::mma_commit(&s.kempty[sk]);
-        }
+      for (int kk = 0; kk < kKT / 16; ++kk)  // O += P(t) V(t)
+        tc::mma_bf16_ts(tmem + kOCol, pb + kk * 8, tc::desc_sw128_mn(v_addr + kk * 2048, kTileHalf),
+                        idesc_o, t > 0 || kk > 0);
+      tc::mma_commit(s.pvdone);
+      tc::mma_commit(&s.vempty[sv]);
+      if (t + 2 < ntiles) {
+        // S(t+2) overwrites P(t): wait until P(t) V(t) has completed
+        if (!wait_or_abort(s.pvdone, t & 1, s.abort)) { ok = false; break; }
+        if (!issue_s(t + 2)) { ok = false; break; }
       }
     }
     if (!ok) raise_abort(a, s, tc::kSiteMma);
@@ -292,69 +277,67 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc::mbar_wait(s.mdone, 0);
   } else if (warp >= 2) {
     // -------------------------------------------------------------- softmax
-    const int qi = (warp - 2) >> 2;                      // query tile of this warp
-    const int et = tid - 64 - qi * kSoftThreads;         // 0..127 within the tile
+    const int et = tid - 64;                             // 0..255
+    const int hh = et >> 7;                              // half of the key tile / of O
     const int quarter = warp & 3;
     const int row = quarter * 32 + lane;                 // TMEM lane = query row of the tile
     const uint32_t lane_base = uint32_t(quarter * 32) << 16;
-    const uint32_t tb = tmem + lane_base + qi * kTileCols;
-    const int ti0 = i0 + qi * a.rows_per_tile;           // first selected row of the tile
-    const int tcnt = max(0, min(a.rows_per_tile, cnt - qi * a.rows_per_tile));
-    const bool active = qi < nq;
-    const bool row_ok = row < tcnt * G;
-    const int i_row = ti0 + (row_ok ? row / G : 0);
+    const uint32_t tl = tmem + lane_base;
+    const bool row_ok = row < cnt * G;
+    const int i_row = i0 + (row_ok ? row / G : 0);
     const int h_row = g * G + (row_ok ? row % G : 0);
     int p_row = row_ok ? a.idx[i_row] : -1;
     if (p_row >= N) p_row = -1;
-    if (active && qrows < kRows) {  // rows past the query box: zero (their S is masked anyway)
-      uint8_t* q_s = s.q + qi * kQBytes;
+    if (qrows < kRows) {  // rows past the query box: zero (their S is masked anyway)
       for (int x = et; x < (kRows - qrows) * 16; x += kSoftThreads) {
         const int rr = qrows + (x >> 4), ch = x & 15;
-        *reinterpret_cast<uint4*>(q_s + (ch >> 3) * kQHalf + tc::sw128_offset(rr, ch & 7)) = make_uint4(0u, 0u, 0u, 0u);
+        *reinterpret_cast<uint4*>(s.q + (ch >> 3) * kQHalf + tc::sw128_offset(rr, ch & 7)) = make_uint4(0u, 0u, 0u, 0u);
       }
       tc::fence_proxy_async_smem();
     }
-    asm volatile("bar.sync %0, %1;" ::"r"(1 + qi), "n"(kSoftThreads) : "memory");
+    asm volatile("bar.sync 1, %0;" ::"n"(kSoftThreads) : "memory");
     if (et == 0) tc::mbar_arrive(s.qready);
 
-    bool ok = active;
-    float m_ref = -INFINITY, lsum = 0.f;  // running max (scaled, log2 units) and row sum
-    const int my_tiles = tiles_of(qi);
-    for (int t = 0; t < my_tiles && active; ++t) {
+    bool ok = true;
+    float m_ref = -INFINITY, lsum = 0.f;  // running max (scaled, log2 units, same in both halves) and half-row sum
+    for (int t = 0; t < ntiles; ++t) {
+      const uint32_t sb = tl + uint32_t(t & 1) * kSCols;
       // the tcgen05.ld below is warp-collective: the whole warp goes on or stops
-      const bool got = __all_sync(0xffffffffu, ok && wait_or_abort(&s.sfull[qi], t & 1, s.abort));
+      const bool got = __all_sync(0xffffffffu, ok && wait_or_abort(&s.sfull[t & 1], (t >> 1) & 1, s.abort));
       if (!got) {
         if (ok) raise_abort(a, s, tc::kSiteMma);
         ok = false;
-        continue;
       }
-      tc::tc_fence_after();
-      float sv0[64], sv1[64];
-      tc::tmem_ld64(tb, sv0);
-      tc::tmem_ld64(tb + 64, sv1);
-      const int j0 = t * kKT;
-      if (j0 + kKT - 1 > p_row) {  // part of the tile is past this row's position
+      float sv[64];
+      float hmax = -INFINITY;
+      const int j0 = t * kKT + hh * 64;
+      if (got) {
+        tc::tc_fence_after();
+        tc::tmem_ld64(sb + hh * 64, sv);
+        if (j0 + 63 > p_row) {  // part of this half is past this row's position
 #pragma unroll
-        for (int i = 0; i < 64; ++i) {
-          if (j0 + i > p_row) sv0[i] = -INFINITY;
-          if (j0 + 64 + i > p_row) sv1[i] = -INFINITY;
+          for (int i = 0; i < 64; ++i)
+            if (j0 + i > p_row) sv[i] = -INFINITY;
         }
-      }
-      float tm[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+        float tm[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-      for (int i = 0; i < 64; ++i) {
-        tm[i & 3] = fmaxf(tm[i & 3], sv0[i]);
-        tm[(i + 2) & 3] = fmaxf(tm[(i + 2) & 3], sv1[i]);
+        for (int i = 0; i < 64; ++i) tm[i & 3] = fmaxf(tm[i & 3], sv[i]);
+        hmax = fmaxf(fmaxf(tm[0], tm[1]), fmaxf(tm[2], tm[3]));
       }
-      const float tmax = fmaxf(fmaxf(tm[0], tm[1]), fmaxf(tm[2], tm[3])) * a.scale_log2;
+      // exchange the half-row maxima (buffers alternate with the tile, so a
+      // half that runs ahead never overwrites a value its partner still reads)
+      float* xm = s.xmax + (t & 1) * 256;
+      xm[hh * 128 + row] = hmax;
+      asm volatile("bar.sync 1, %0;" ::"n"(kSoftThreads) : "memory");
+      if (!ok) continue;
+      const float tmax = fmaxf(hmax, xm[(hh ^ 1) * 128 + row]) * a.scale_log2;
       const bool need = tmax > m_ref + kRescaleLog2 || (m_ref == -INFINITY && tmax != -INFINITY);
       const float alpha = need ? tc::ex2(m_ref - tmax) : 1.f;  // 0 when m_ref is -inf
       if (need) {
         lsum *= alpha;
         m_ref = tmax;
       }
-      // P = 2^(S scale - m) in bf16 pairs over the upper half of S (already read),
-      // 32 columns at a time
+      // this half of P = 2^(S scale - m) in bf16 pairs over the upper half of S
       float ls[4] = {0.f, 0.f, 0.f, 0.f};
       const float nb = -m_ref;
       const bool live = m_ref != -INFINITY;
@@ -362,66 +345,63 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint32_t pw[32];
 #pragma unroll
         for (int i = 0; i < 32; ++i) {
-          const float p0 = live ? tc::ex2(fmaf(sv0[2 * i], a.scale_log2, nb)) : 0.f;
-          const float p1 = live ? tc::ex2(fmaf(sv0[2 * i + 1], a.scale_log2, nb)) : 0.f;
+          const float p0 = live ? tc::ex2(fmaf(sv[2 * i], a.scale_log2, nb)) : 0.f;
+          const float p1 = live ? tc::ex2(fmaf(sv[2 * i + 1], a.scale_log2, nb)) : 0.f;
           ls[i & 1] += p0;
           ls[(i & 1) + 2] += p1;
           __nv_bfloat162 pr = __floats2bfloat162_rn(p0, p1);
           pw[i] = *reinterpret_cast<uint32_t*>(&pr);
         }
-        tc::tmem_st32u(tb + kPCol, pw);
-      }
-      {
-        uint32_t pw[32];
-#pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          const float p0 = live ? tc::ex2(fmaf(sv1[2 * i], a.scale_log2, nb)) : 0.f;
-          const float p1 = live ? tc::ex2(fmaf(sv1[2 * i + 1], a.scale_log2, nb)) : 0.f;
-          ls[i & 1] += p0;
-          ls[(i & 1) + 2] += p1;
-          __nv_bfloat162 pr = __floats2bfloat162_rn(p0, p1);
-          pw[i] = *reinterpret_cast<uint32_t*>(&pr);
-        }
-        tc::tmem_st32u(tb + kPCol + 32, pw);
+        tc::tmem_st32u(sb + kPCol + hh * 32, pw);
       }
       lsum += (ls[0] + ls[1]) + (ls[2] + ls[3]);
       if (__any_sync(0xffffffffu, need) && t > 0) {
-        // O already holds P(t-1) V(t-1) (S(t) was issued after it completed),
-        // and P(t) V(t) waits for this warp's pfull arrival below
-        for (int c = 0; c < kD; c += 32) {
+        // P(t-1) V(t-1) must have completed before this warp rescales its half
+        // of O. S(t) was issued after P(t-2) V(t-2) completed, so pvdone is at
+        // most one phase behind here and its parity cannot alias; P(t) V(t)
+        // waits for this warp's pfull arrival below.
+        if (!__all_sync(0xffffffffu, wait_or_abort(s.pvdone, (t - 1) & 1, s.abort))) {
+          raise_abort(a, s, tc::kSiteMma);
+          ok = false;
+          continue;
+        }
+        tc::tc_fence_after();
+        for (int c = hh * 64; c < hh * 64 + 64; c += 32) {
           float o[32];
-          tc::tmem_ld32(tb + kOCol + c, o);
+          tc::tmem_ld32(tl + kOCol + c, o);
 #pragma unroll
           for (int i = 0; i < 32; ++i) o[i] *= alpha;
-          tc::tmem_st32(tb + kOCol + c, o);
+          tc::tmem_st32(tl + kOCol + c, o);
         }
       }
       tc::tc_fence_before();
-      tc::mbar_arrive(&s.pfull[qi]);
+      tc::mbar_arrive(&s.pfull[t & 1]);
     }
-    if (active) {
-      // O is complete once the last P V of this tile has completed (phase
-      // my_tiles-1 of pvdone; phase my_tiles-2 completed before S(my_tiles-1) was issued)
-      const bool fin = __all_sync(0xffffffffu, ok && wait_or_abort(&s.pvdone[qi], (my_tiles - 1) & 1, s.abort));
-      if (!fin && ok) raise_abort(a, s, tc::kSiteFinal);
-      if (fin) {
-        tc::tc_fence_after();
-        const float inv = lsum > 0.f ? 1.f / lsum : 0.f;
-        __nv_bfloat16* dst = a.out + ((int64_t(l) * a.n_sel + i_row) * Hq + h_row) * kD;
-        for (int c = 0; c < kD; c += 32) {
-          float o[32];
-          tc::tmem_ld32(tb + kOCol + c, o);
-          if (row_ok && p_row >= 0) {
+    // row sum = the two halves' sums (same running max in both)
+    s.xsum[hh * 128 + row] = lsum;
+    asm volatile("bar.sync 1, %0;" ::"n"(kSoftThreads) : "memory");
+    const float total = s.xsum[row] + s.xsum[128 + row];
+    // O is complete once every MMA has: wait on the MMA thread's single-use
+    // final commit (pvdone could be two phases behind here and alias)
+    const bool fin = __all_sync(0xffffffffu, ok && wait_or_abort(s.mdone, 0, s.abort));
+    if (!fin && ok) raise_abort(a, s, tc::kSiteFinal);
+    if (fin) {
+      tc::tc_fence_after();
+      const float inv = total > 0.f ? 1.f / total : 0.f;
+      __nv_bfloat16* dst = a.out + ((int64_t(l) * a.n_sel + i_row) * Hq + h_row) * kD;
+      for (int c = hh * 64; c < hh * 64 + 64; c += 32) {
+        float o[32];
+        tc::tmem_ld32(tl + kOCol + c, o);
+        if (row_ok && p_row >= 0) {
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-              uint32_t w4[4];
+          for (int u = 0; u < 4; ++u) {
+            uint32_t w4[4];
 #pragma unroll
-              for (int k2 = 0; k2 < 4; ++k2) {
-                __nv_bfloat162 pr = __floats2bfloat162_rn(o[u * 8 + 2 * k2] * inv, o[u * 8 + 2 * k2 + 1] * inv);
-                w4[k2] = *reinterpret_cast<uint32_t*>(&pr);
-              }
-              *reinterpret_cast<uint4*>(dst + c + u * 8) = make_uint4(w4[0], w4[1], w4[2], w4[3]);
+            for (int k2 = 0; k2 < 4; ++k2) {
+              __nv_bfloat162 pr = __floats2bfloat162_rn(o[u * 8 + 2 * k2] * inv, o[u * 8 + 2 * k2 + 1] * inv);
+              w4[k2] = *reinterpret_cast<uint32_t*>(&pr);
             }
+            *reinterpret_cast<uint4*>(dst + c + u * 8) = make_uint4(w4[0], w4[1], w4[2], w4[3]);
           }
         }
       }
@@ -519,7 +499,7 @@ cudaError_t launch_refresh_tc(const KvDev& kv, const BatchDev& b, const int32_t*
   int blocks = 0;
   for (int r = 0; r < b.R; ++r) {
     const int kr = idx_off_host[r + 1] - idx_off_host[r];
-    blocks += (kr + kTiles * a.rows_per_tile - 1) / (kTiles * a.rows_per_tile);
+    blocks += (kr + a.rows_per_tile - 1) / a.rows_per_tile;
   }
   a.n_blocks = blocks;
   a.scale_log2 = kLog2e / sqrtf(float(kD));
