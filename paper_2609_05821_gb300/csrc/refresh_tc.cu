@@ -338,22 +338,25 @@ __global__ void __launch_bounds__(kThreads, 1)
         m_ref = tmax;
       }
       // this half of P = 2^(S scale - m) in bf16 pairs over the upper half of S
-      float ls[4] = {0.f, 0.f, 0.f, 0.f};
-      const float nb = -m_ref;
-      const bool live = m_ref != -INFINITY;
+      // (one packed FMA per pair for scale and bias, packed adds for the sum).
+      // A row with no visible key yet (m = -inf) uses bias 0: its logits are
+      // all -inf and its P is 0.
+      const float2 sc2 = make_float2(a.scale_log2, a.scale_log2);
+      const float2 nb2 = m_ref == -INFINITY ? make_float2(0.f, 0.f) : make_float2(-m_ref, -m_ref);
+      float2 ls2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
       {
         uint32_t pw[32];
 #pragma unroll
         for (int i = 0; i < 32; ++i) {
-          const float p0 = live ? tc::ex2(fmaf(sv[2 * i], a.scale_log2, nb)) : 0.f;
-          const float p1 = live ? tc::ex2(fmaf(sv[2 * i + 1], a.scale_log2, nb)) : 0.f;
-          ls[i & 1] += p0;
-          ls[(i & 1) + 2] += p1;
-          __nv_bfloat162 pr = __floats2bfloat162_rn(p0, p1);
+          const float2 y = tc::ffma2(make_float2(sv[2 * i], sv[2 * i + 1]), sc2, nb2);
+          const float2 pp = make_float2(tc::ex2(y.x), tc::ex2(y.y));
+          ls2[i & 1] = tc::fadd2(ls2[i & 1], pp);
+          __nv_bfloat162 pr = __floats2bfloat162_rn(pp.x, pp.y);
           pw[i] = *reinterpret_cast<uint32_t*>(&pr);
         }
         tc::tmem_st32u(sb + kPCol + hh * 32, pw);
       }
+      const float ls[4] = {ls2[0].x, ls2[0].y, ls2[1].x, ls2[1].y};
       lsum += (ls[0] + ls[1]) + (ls[2] + ls[3]);
       if (__any_sync(0xffffffffu, need) && t > 0) {
         // P(t-1) V(t-1) must have completed before this warp rescales its half
