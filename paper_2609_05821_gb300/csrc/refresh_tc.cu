@@ -155,6 +155,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int G = kv.G, Hq = kv.Hq;
 
   // CTA -> (request, first selected row, row count); larger positions first
+  // within each (layer, KV head), whose CTAs run together and share K/V in L2
   const int span = a.rows_per_tile;
   int blk = a.n_blocks - 1 - int(blockIdx.x);
   int r = 0, i0 = -1, cnt = 0;
@@ -321,7 +322,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         float tm[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-        for (int i = 0; i < 64; ++i) tm[i & 3] = fmaxf(tm[i & 3], sv[i]);
+        for (int i = 0; i < 32; ++i) tm[i & 3] = tc::fmax3(tm[i & 3], sv[2 * i], sv[2 * i + 1]);
         hmax = fmaxf(fmaxf(tm[0], tm[1]), fmaxf(tm[2], tm[3]));
       }
       // exchange the half-row maxima (buffers alternate with the tile, so a

@@ -249,7 +249,7 @@ __device__ __forceinline__ void row_stats(float (&v)[NC], int valid, float scale
   }
   float cm[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-  for (int x = 0; x < NC; ++x) cm[x & 3] = fmaxf(cm[x & 3], v[x]);
+  for (int x = 0; x < NC / 2; ++x) cm[x & 3] = tc::fmax3(cm[x & 3], v[2 * x], v[2 * x + 1]);
   const float mn = fmaxf(m, fmaxf(fmaxf(cm[0], cm[1]), fmaxf(cm[2], cm[3])));
   if (mn == -INFINITY) return;
   const float2 sc2 = make_float2(scale, scale), nb2 = make_float2(-mn * scale, -mn * scale);
