@@ -7,9 +7,10 @@
 // the KV head. Keys stream in tiles of 128 (a tcgen05.mma costs about the same
 // issue time for N = 64 and N = 128, so wide tiles halve the instruction
 // count). Roles (320 threads):
-//   warp 0     one thread issues TMA loads: the query tile (a 3-D box of 64
-//              dims x G heads x floor(128/G) rows lands in the tile's row
-//              order), then K tiles (three-stage ring) and V tiles (two stages)
+//   warp 0     TMA loads: the query tile (a 3-D box of 64 dims x G heads x
+//              floor(128/G) rows lands in the tile's row order), then K tiles
+//              (three-stage ring) and V tiles (two stages); the lanes issue
+//              the copies of a tile together (one per page half when paged)
 //   warp 1     one thread issues tcgen05 MMAs: S(t) = Q K(t)^T into one of two
 //              TMEM buffers, O += P(t) V(t) with P read from TMEM
 //   warps 2-9  softmax, two warps per TMEM lane quarter: each thread owns one
@@ -122,24 +123,31 @@ __device__ __forceinline__ void raise_abort(const RefArgs& a, const Smem& s, int
   *s.abort = 1;
 }
 
-// TMA of the 128-key tile starting at request-local key j0 (one 64-dim half per box).
+// Warp-cooperative TMA of the 128-key tile starting at request-local key j0:
+// lane 0 posts the byte count, then copy c is issued by lane c. A copy is one
+// 64-dim half of the whole tile (contiguous cache: 2 copies) or of one page
+// (paged cache: 2 x 128/page copies, up to 32), so a paged tile costs one
+// round of parallel page-index loads and copy issues instead of a serial loop.
 __device__ __forceinline__ void load_tile(const RefArgs& a, const CUtensorMap* map, uint8_t* dst,
-                                          uint64_t* bar, int l, int g, int r, int t0, int N, int j0) {
+                                          uint64_t* bar, int l, int g, int r, int t0, int N, int j0,
+                                          int lane) {
   const KvDev& kv = a.kv;
-  tc::mbar_arrive_expect_tx(bar, kTileBytes);
+  if (lane == 0) tc::mbar_arrive_expect_tx(bar, kTileBytes);
+  __syncwarp();
+  const int hf = lane & 1;
   if (kv.page_size == 0) {
-    const int32_t y = int32_t((int64_t(l) * kv.Hkv + g) * kv.n_tot + t0 + j0);
-    tc::tma_load_2d(dst, map, bar, 0, y);
-    tc::tma_load_2d(dst + kTileHalf, map, bar, 64, y);
+    if (lane < 2) {
+      const int32_t y = int32_t((int64_t(l) * kv.Hkv + g) * kv.n_tot + t0 + j0);
+      tc::tma_load_2d(dst + hf * kTileHalf, map, bar, hf * 64, y);
+    }
   } else {
     const int ps = kv.page_size;
-    const int last_page = (N - 1) / ps;
-    for (int i = 0; i < kKT / ps; ++i) {
-      const int lp = min((j0 + i * ps) / ps, last_page);
+    const int i = lane >> 1;  // page of the tile
+    if (i < kKT / ps) {
+      const int lp = min((j0 + i * ps) / ps, (N - 1) / ps);  // tail pages repeat the last one (masked)
       const int page = kv.page_table[int64_t(r) * kv.max_pages + lp];
       const int32_t y = int32_t(((int64_t(l) * kv.num_pages + page) * kv.Hkv + g) * ps);
-      tc::tma_load_2d(dst + i * ps * 128, map, bar, 0, y);
-      tc::tma_load_2d(dst + kTileHalf + i * ps * 128, map, bar, 64, y);
+      tc::tma_load_2d(dst + hf * kTileHalf + i * ps * 128, map, bar, hf * 64, y);
     }
   }
 }
@@ -207,24 +215,34 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc::tc_fence_after();
   const uint32_t tmem = *s.tmem_slot;
 
-  if (warp == 0 && lane == 0) {
-    // ---------------------------------------------------------------- loads
-    tc::mbar_arrive_expect_tx(s.qready, 2u * 128u * uint32_t(qrows));
-    for (int hf = 0; hf < 2; ++hf)
-      tc::tma_load_3d(s.q + hf * kQHalf, &qmap, s.qready, hf * 64, g * G, l * a.n_sel + i0);
+  if (warp == 0) {
+    // ------------------------------------------------------- loads (warp 0)
+    if (lane == 0) {
+      tc::mbar_arrive_expect_tx(s.qready, 2u * 128u * uint32_t(qrows));
+      for (int hf = 0; hf < 2; ++hf)
+        tc::tma_load_3d(s.q + hf * kQHalf, &qmap, s.qready, hf * 64, g * G, l * a.n_sel + i0);
+    }
     uint32_t nk = 0, nv = 0;
     for (int t = 0; t < ntiles; ++t) {
       const int sk = t % kKStages;
-      if (!wait_or_abort(&s.kempty[sk], ((t / kKStages) & 1) ^ 1, s.abort)) { raise_abort(a, s, tc::kSiteLoad); break; }
-      load_tile(a, &kmap, s.k + sk * kTileBytes, &s.kfull[sk], l, g, r, t0, N, t * kKT);
+      if (!__all_sync(0xffffffffu, wait_or_abort(&s.kempty[sk], ((t / kKStages) & 1) ^ 1, s.abort))) {
+        if (lane == 0) raise_abort(a, s, tc::kSiteLoad);
+        break;
+      }
+      load_tile(a, &kmap, s.k + sk * kTileBytes, &s.kfull[sk], l, g, r, t0, N, t * kKT, lane);
       ++nk;
       const int sv = t % kVStages;
-      if (!wait_or_abort(&s.vempty[sv], ((t / kVStages) & 1) ^ 1, s.abort)) { raise_abort(a, s, tc::kSiteLoad); break; }
-      load_tile(a, &vmap, s.v + sv * kTileBytes, &s.vfull[sv], l, g, r, t0, N, t * kKT);
+      if (!__all_sync(0xffffffffu, wait_or_abort(&s.vempty[sv], ((t / kVStages) & 1) ^ 1, s.abort))) {
+        if (lane == 0) raise_abort(a, s, tc::kSiteLoad);
+        break;
+      }
+      load_tile(a, &vmap, s.v + sv * kTileBytes, &s.vfull[sv], l, g, r, t0, N, t * kKT, lane);
       ++nv;
     }
-    s.counters[0] = nk;
-    s.counters[1] = nv;
+    if (lane == 0) {
+      s.counters[0] = nk;
+      s.counters[1] = nv;
+    }
   } else if (warp == 1 && lane == 0) {
     // ------------------------------------------------------------------ MMA
     uint32_t ck = 0, cv = 0;

@@ -186,10 +186,16 @@ __device__ __forceinline__ void load_k_tile(const TcArgs& a, const CUtensorMap* 
   } else {
     const int ps = kv.page_size;
     const int last_page = (w.N - 1) / ps;
-    for (int i = 0; i < kTile / ps; ++i) {
-      const int lp = min((tok + i * ps) / ps, last_page);  // tail pages repeat the last one (masked)
-      const int page = kv.page_table[int64_t(w.r) * kv.max_pages + lp];
-      const int32_t y = int32_t(((int64_t(w.l) * kv.num_pages + page) * kv.Hkv + w.g) * ps);
+    const int np = kTile / ps;  // 1..16 pages per tile (page sizes 8..128)
+    int page[16];
+    const int32_t* pt = kv.page_table + int64_t(w.r) * kv.max_pages;
+#pragma unroll
+    for (int i = 0; i < 16; ++i)  // all page indices first: their loads overlap
+      if (i < np) page[i] = pt[min((tok + i * ps) / ps, last_page)];  // tail pages repeat the last one (masked)
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      if (i >= np) break;
+      const int32_t y = int32_t(((int64_t(w.l) * kv.num_pages + page[i]) * kv.Hkv + w.g) * ps);
       tc::tma_load_2d(dst + i * ps * 128, kmap, bar, 0, y);
       tc::tma_load_2d(dst + kHalfK + i * ps * 128, kmap, bar, 64, y);
     }
