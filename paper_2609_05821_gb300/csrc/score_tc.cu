@@ -16,10 +16,11 @@
 //            sum_q sum_h alpha
 //
 // Pass B walks the tiles in reverse so the most recent K tiles of pass A are
-// still in L2. Roles (320 threads):
-//   warp 0       lane 0 issues TMA loads of K tiles (128 tokens x 128 dims,
-//                128-byte swizzle) into a three-stage ring; lane 1 loads the
-//                matching V tiles of pass A into two buffers
+// still in L2. Roles (352 threads):
+//   warp 0       TMA loads of K tiles (128 tokens x 128 dims, 128-byte
+//                swizzle) into a three-stage ring, the lanes issuing a tile's
+//                copies together (one per page half when paged)
+//   warp 10      the same for the matching V tiles of pass A (two buffers)
 //   warp 1       one thread issues tcgen05 MMAs into two 256-column TMEM
 //                accumulator slots (it also owns the TMEM allocation)
 //   warps 2-9    epilogue, two warps per TMEM lane quarter (warp group h
@@ -43,8 +44,9 @@ constexpr int kTile = 128;
 constexpr int kStages = 3;                     // K ring
 constexpr int kVBufs = 2;                      // V tiles (value norms, pass A)
 constexpr int kGroupRows = 256;
-constexpr int kThreads = 320;
+constexpr int kThreads = 352;
 constexpr int kEpiThreads = 256;
+constexpr int kVWarp = 10;                     // warps 2-9 are the epilogue
 constexpr uint32_t kHalfQ = kGroupRows * 128;  // 32 KB: one 64-dim half of the row tile
 constexpr uint32_t kHalfK = kTile * 128;       // 16 KB
 constexpr uint32_t kStageBytes = 2 * kHalfK;   // 32 KB per K tile
@@ -173,31 +175,31 @@ __device__ __forceinline__ void epi_barrier() {
   asm volatile("bar.sync 1, %0;" ::"n"(kEpiThreads) : "memory");
 }
 
-// Issue the TMA loads of K (or V) tile `tile` of unit w into `dst`.
+// Warp-cooperative TMA of K (or V) tile `tile` of unit w into `dst`: lane 0
+// posts the byte count, then copy c is issued by lane c. A copy is one 64-dim
+// half of the whole tile (contiguous cache: 2 copies) or of one page (paged
+// cache: 2 x 128/page copies, up to 32), so a paged tile costs one round of
+// parallel page-index loads and copy issues.
 __device__ __forceinline__ void load_k_tile(const TcArgs& a, const CUtensorMap* kmap, const Unit& w,
-                                            uint8_t* dst, uint64_t* bar, int tile) {
-  tc::mbar_arrive_expect_tx(bar, kStageBytes);
+                                            uint8_t* dst, uint64_t* bar, int tile, int lane) {
+  if (lane == 0) tc::mbar_arrive_expect_tx(bar, kStageBytes);
+  __syncwarp();
   const int tok = tile * kTile;
   const KvDev& kv = a.kv;
+  const int hf = lane & 1;
   if (kv.page_size == 0) {
-    const int32_t y = int32_t((int64_t(w.l) * kv.Hkv + w.g) * kv.n_tot + w.t0 + tok);
-    tc::tma_load_2d(dst, kmap, bar, 0, y);
-    tc::tma_load_2d(dst + kHalfK, kmap, bar, 64, y);
+    if (lane < 2) {
+      const int32_t y = int32_t((int64_t(w.l) * kv.Hkv + w.g) * kv.n_tot + w.t0 + tok);
+      tc::tma_load_2d(dst + hf * kHalfK, kmap, bar, hf * 64, y);
+    }
   } else {
     const int ps = kv.page_size;
-    const int last_page = (w.N - 1) / ps;
-    const int np = kTile / ps;  // 1..16 pages per tile (page sizes 8..128)
-    int page[16];
-    const int32_t* pt = kv.page_table + int64_t(w.r) * kv.max_pages;
-#pragma unroll
-    for (int i = 0; i < 16; ++i)  // all page indices first: their loads overlap
-      if (i < np) page[i] = pt[min((tok + i * ps) / ps, last_page)];  // tail pages repeat the last one (masked)
-#pragma unroll
-    for (int i = 0; i < 16; ++i) {
-      if (i >= np) break;
-      const int32_t y = int32_t(((int64_t(w.l) * kv.num_pages + page[i]) * kv.Hkv + w.g) * ps);
-      tc::tma_load_2d(dst + i * ps * 128, kmap, bar, 0, y);
-      tc::tma_load_2d(dst + kHalfK + i * ps * 128, kmap, bar, 64, y);
+    const int i = lane >> 1;  // page of the tile
+    if (i < kTile / ps) {
+      const int lp = min((tok + i * ps) / ps, (w.N - 1) / ps);  // tail pages repeat the last one (masked)
+      const int page = kv.page_table[int64_t(w.r) * kv.max_pages + lp];
+      const int32_t y = int32_t(((int64_t(w.l) * kv.num_pages + page) * kv.Hkv + w.g) * ps);
+      tc::tma_load_2d(dst + hf * kHalfK + i * ps * 128, kmap, bar, hf * 64, y);
     }
   }
 }
@@ -315,8 +317,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc::tc_fence_after();
   const uint32_t tmem = *s.tmem_slot;
 
-  if (warp == 0 && lane == 0) {
-    // ---------------------------------------------------------- producer: K
+  if (warp == 0) {
+    // ------------------------------------------------- producer: K (warp 0)
     uint32_t seq = 0;
     bool ok = true;
     for (int u = blockIdx.x; u < a.n_units && ok; u += gridDim.x) {
@@ -324,19 +326,19 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!decode_unit(a, u, w)) continue;
       for (int i = 0; i < 2 * w.tiles; ++i, ++seq) {
         const int st = seq % kStages;
-        if (!wait_or_abort(&s.kempty[st], ((seq / kStages) & 1) ^ 1, s.abort)) {
-          if (!*s.abort) raise_abort(a, s, tc::kSiteLoad);
+        if (!__all_sync(0xffffffffu, wait_or_abort(&s.kempty[st], ((seq / kStages) & 1) ^ 1, s.abort))) {
+          if (lane == 0 && !*s.abort) raise_abort(a, s, tc::kSiteLoad);
           ok = false;
           break;
         }
-        load_k_tile(a, &kmap, w, s.k + st * kStageBytes, &s.kfull[st], tile_of(w, i));
+        load_k_tile(a, &kmap, w, s.k + st * kStageBytes, &s.kfull[st], tile_of(w, i), lane);
       }
     }
-    s.counters[0] = seq;
-  } else if (warp == 0 && lane == 1) {
-    // ---------------------------------------------------------- producer: V
-    // V tiles of pass 1 for the value norms, on a thread of their own so that
-    // a V tile waiting for its buffer never holds back the K ring
+    if (lane == 0) s.counters[0] = seq;
+  } else if (warp == kVWarp) {
+    // ------------------------------------------------ producer: V (warp 10)
+    // V tiles of pass 1 for the value norms, on a warp of their own so that a
+    // V tile waiting for its buffer never holds back the K ring
     uint32_t vseq = 0;
     bool ok = true;
     for (int u = blockIdx.x; u < a.n_units && ok; u += gridDim.x) {
@@ -344,15 +346,15 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!decode_unit(a, u, w) || w.rg != 0) continue;
       for (int i = 0; i < w.tiles; ++i, ++vseq) {
         const int vb = vseq % kVBufs;
-        if (!wait_or_abort(&s.vempty[vb], ((vseq / kVBufs) & 1) ^ 1, s.abort)) {
-          if (!*s.abort) raise_abort(a, s, tc::kSiteLoad);
+        if (!__all_sync(0xffffffffu, wait_or_abort(&s.vempty[vb], ((vseq / kVBufs) & 1) ^ 1, s.abort))) {
+          if (lane == 0 && !*s.abort) raise_abort(a, s, tc::kSiteLoad);
           ok = false;
           break;
         }
-        load_k_tile(a, &vmap, w, s.v + vb * kStageBytes, &s.vfull[vb], i);
+        load_k_tile(a, &vmap, w, s.v + vb * kStageBytes, &s.vfull[vb], i, lane);
       }
     }
-    s.counters[2] = vseq;
+    if (lane == 0) s.counters[2] = vseq;
   } else if (warp == 1 && lane == 0) {
     // ----------------------------------------------------------------- MMA
     uint32_t kseq = 0, tseq = 0, useq = 0;
@@ -413,7 +415,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     s.counters[1] = kseq;
     tc::mma_commit(s.mdone);  // every MMA issued above has completed once this arrives
     tc::mbar_wait(s.mdone, 0);
-  } else if (warp >= 2) {
+  } else if (warp >= 2 && warp < kVWarp) {
     // ------------------------------------------------------------ epilogue
     // After an abort the epilogue keeps walking its units (skipping the work)
     // so that every thread reaches every named barrier.
