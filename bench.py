@@ -158,7 +158,12 @@ def work_model(pipe) -> dict:
     tok, qo = b.tok_off.tolist(), b.q_off.tolist()
     R, K = b.num_requests, b.num_images
     n_tot = tok[-1]
-    score_bytes = 2 * L * Hkv * n_tot * d * esz + L * Hq * qo[-1] * d * esz + 8 * n_tot + 4 * K
+    # K read once, the queries, s and attn_sum written, g; then the value-norm source:
+    # V read once, or one stored fp32 per token and scored layer, or nothing
+    score_bytes = L * Hkv * n_tot * d * esz + L * Hq * qo[-1] * d * esz + 8 * n_tot + 4 * K
+    score_bytes += {"v": L * Hkv * n_tot * d * esz, "side_cache": 4 * L * n_tot, "none": 0}[pipe.value_norm]
+    if pipe.extra_lse is not None:  # one fp32 per scoring row
+        score_bytes += 4 * L * Hq * qo[-1]
     score_flops = sum(2 * L * Hq * (qo[r + 1] - qo[r]) * (tok[r + 1] - tok[r]) * d for r in range(R))
     k_sel = pipe.n_sel
     sel_bytes = 4 * n_tot + 4 * K + 4 * n_tot + n_tot + 4 * k_sel + 4 * K
@@ -171,12 +176,22 @@ def work_model(pipe) -> dict:
         ref_flops += sum(4 * Hq * d * (p + 1) for p in ps) * Lall
         if ps:
             ref_bytes += 2 * Lall * Hkv * (max(ps) + 1) * d * esz
-    return {
+    out = {
         "score": {"bytes": score_bytes, "flops": score_flops},
         "select": {"bytes": sel_bytes, "flops": 0},
         "exchange": {"bytes": 2 * copy_bytes, "flops": 0},
         "refresh": {"bytes": ref_bytes, "flops": ref_flops},
     }
+    if pipe.vnorm is not None:  # re-read the rewritten value rows, write their norms
+        out["norm_update"] = {"bytes": Lall * k_sel * Hkv * d * esz + 4 * Lall * k_sel, "flops": 0}
+    return out
+
+
+def side_cache_bytes(pipe) -> int:
+    """conduit_value_norms: every value row read once, one fp32 per token and layer written."""
+    kv = pipe.kv
+    n_tot = pipe.batch.n_tot
+    return kv.num_layers * n_tot * (kv.num_kv_heads * kv.head_dim * kv.k.element_size() + 4)
 
 
 def call_kernels(pipe) -> dict:
@@ -193,8 +208,12 @@ def call_kernels(pipe) -> dict:
     else:
         score = (["value_sumsq_kernel", "rowstats_kernel", "colsum_kernel"] + tail, "alu", "score_simt.cu")
         refresh = (["refresh_simt_kernel"], "alu", "refresh_simt.cu")
+    norms = (["vnorm_halves_kernel" if tc else "vnorm_rows_kernel"], "hbm", "vnorm.cu")
+    if pipe.value_norm != "v" and not tc:  # no separate value pass
+        score = (["rowstats_kernel", "colsum_kernel"] + tail, "alu", "score_simt.cu")
     return {"score": score, "select": (["select_kernel"], "hbm", "select.cu"),
-            "exchange": (["kv_copy_kernel"], "hbm", "kvcopy.cu"), "refresh": refresh}
+            "exchange": (["kv_copy_kernel"], "hbm", "kvcopy.cu"), "refresh": refresh,
+            "norm_update": norms, "side_cache": norms}
 
 
 def _src_hash(src: str) -> str:
@@ -218,12 +237,15 @@ def _traffic(call: str, workload: str, src: str):
 
 
 # -------------------------------------------------------------- our arm
-def build_pipeline(cfg: str, device, ratio=None):
+def build_pipeline(cfg: str, device, ratio=None, statistic="mean", value_norm="v",
+                   full_context=False):
     from paper_2609_05821_gb300 import pipeline, synth
     w = synth.workload(cfg)
     inputs = synth.make_inputs(w, device=device)
     _with_ratio(inputs, ratio)  # one refresh ratio for every request (e.g. the long-document budgets)
-    return pipeline.from_inputs(inputs), w
+    extra = synth.make_extra_lse(inputs) if full_context else None
+    return pipeline.from_inputs(inputs, statistic=statistic, value_norm=value_norm,
+                                extra_lse=extra), w
 
 
 def time_steps(fn, steps: int, flush=None):
@@ -252,7 +274,8 @@ def run_conduit(args):
     dev = torch.device("cuda", local)
     from paper_2609_05821_gb300 import conduit as C
 
-    pipe, w = build_pipeline(args.config, dev, args.ratio)
+    pipe, w = build_pipeline(args.config, dev, args.ratio, args.statistic, args.value_norm,
+                             args.full_context)
     n_tok = pipe.batch.n_tot
     flush_buf = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
     flush = lambda: flush_buf.zero_()
@@ -286,28 +309,41 @@ def run_conduit(args):
 
     # per-call breakdown over K eager steps (events on the launching stream)
     graph, pipe.graph = pipe.graph, None
-    calls = {"score": [], "select": [], "exchange": [], "refresh": []}
     from paper_2609_05821_gb300 import conduit as CC
+    seq = [("score", pipe.score), ("select", pipe.select), ("exchange", pipe.exchange)]
+    if pipe.vnorm is not None:
+        seq.append(("norm_update", pipe.norm_update))
+    seq.append(("refresh", pipe.refresh_attn))
+    calls = {name: [] for name, _ in seq}
     stream = torch.cuda.current_stream()
     for _ in range(args.steps):
         flush()
-        ev = [torch.cuda.Event(enable_timing=True) for _ in range(5)]
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(len(seq) + 1)]
         ev[0].record(stream)
-        CC.conduit_score(pipe.kv, pipe.batch, pipe.q, pipe.layers, pipe.s, pipe.attn_sum, pipe.g,
-                         pipe.ws_score, pipe.status)
-        ev[1].record(stream)
-        CC.conduit_select_topk(pipe.batch, pipe.s, pipe.g, pipe.lam, pipe.idx_off, pipe.idx_off_dev,
-                               pipe.idx, pipe.mask, pipe.s_hat, pipe.coeff, pipe.ws_sel, pipe.status)
-        ev[2].record(stream)
-        CC.conduit_kv_exchange(pipe.kv, pipe.batch, pipe.idx, pipe.idx_off, pipe.idx_off_dev,
-                               pipe.k_old, pipe.v_old, pipe.k_rows, pipe.v_rows)
-        ev[3].record(stream)
-        CC.conduit_refresh_attn(pipe.kv, pipe.batch, pipe.idx, pipe.idx_off, pipe.idx_off_dev,
-                                pipe.q_rows, pipe.out, pipe.ws_ref, pipe.status)
-        ev[4].record(stream)
-        ev[4].synchronize()
-        for i, name in enumerate(calls):
+        for i, (_, fn) in enumerate(seq):
+            fn()
+            ev[i + 1].record(stream)
+        ev[-1].synchronize()
+        for i, (name, _) in enumerate(seq):
             calls[name].append(ev[i].elapsed_time(ev[i + 1]))
+    side_cache = None
+    if pipe.vnorm is not None:  # built once per cache (outside the step): timed on its own
+        scratch = torch.empty_like(pipe.vnorm)
+        ts = []
+        for _ in range(max(3, args.steps)):
+            flush()
+            ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+            ev[0].record(stream)
+            CC.conduit_value_norms(pipe.kv, pipe.batch, scratch)
+            ev[1].record(stream)
+            ev[1].synchronize()
+            ts.append(ev[0].elapsed_time(ev[1]))
+        sc_ms = sum(ts) / len(ts)
+        sc_bytes = side_cache_bytes(pipe)
+        side_cache = {"us": round(sc_ms * 1e3, 2), "bytes": sc_bytes,
+                      "GB_per_s": round(sc_bytes / (sc_ms / 1e3) / 1e9, 1),
+                      "hbm_frac": round(sc_bytes / (sc_ms / 1e3) / 1e9 / hbm, 4),
+                      "kernels": call_kernels(pipe)["side_cache"][0]}
     pipe.graph = graph
     call_ms = {k: sum(v) / len(v) for k, v in calls.items()}
     status = C.conduit_read_status(pipe.status)
@@ -329,7 +365,8 @@ def run_conduit(args):
     else:
         achieved, peak, unit = model[dom]["flops"] / sec / 1e12, ALU_FP32_TFLOPS, "TFLOP/s"
         peak_note = "fp32 FMA: 152 SMs x 128 lanes x 2 FLOP x 2.07 GHz"
-    traffic = _traffic(dom, args.config, src)
+    # committed ncu traffic covers the default scoring pass only
+    traffic = _traffic(dom, args.config, src) if pipe.plain else None
     roofline = {"bound": bound, "achieved": round(achieved, 3), "peak": round(peak, 1), "unit": unit,
                 "frac": round(achieved / peak, 4), "traffic": traffic, "kernel": dom,
                 "kernels": kernels, "peak_source": peak_note,
@@ -361,10 +398,19 @@ def run_conduit(args):
                    "budget_total": pipe.n_sel, "layers": pipe.kv.num_layers,
                    "ratio_override": args.ratio,
                    "l2": f"flushed between timed steps ({L2_FLUSH_BYTES >> 20} MB write)",
-                   "cuda_graph": not args.no_graph, "parallelism": f"replicas x{world}"},
+                   "cuda_graph": not args.no_graph, "parallelism": f"replicas x{world}",
+                   "statistic": args.statistic,
+                   "value_norms": {"v": "read from V inside the scoring pass",
+                                   "side_cache": "side cache: built once per cache outside the step, "
+                                                 "updated for the rewritten rows inside it",
+                                   "none": "not used (attention alone)"}[args.value_norm],
+                   "softmax": ("full context (seeded outside-key log-sum-exps)" if args.full_context
+                               else "visual keys")},
         "score_select_tokens_per_s": round(n_tok / ((call_ms["score"] + call_ms["select"]) / 1e3), 1),
-        "refresh_pass_us": round((call_ms["exchange"] + call_ms["refresh"]) * 1e3, 2),
+        "refresh_pass_us": round((call_ms["exchange"] + call_ms.get("norm_update", 0.0)
+                                  + call_ms["refresh"]) * 1e3, 2),
         "breakdown": breakdown,
+        **({"side_cache_build": side_cache} if side_cache else {}),
         "roofline": roofline,
         "e2e": {"value": round(world * n_tok / (e2e_mean / 1e3), 1), "unit": UNIT,
                 "h2d_bytes_per_step": pipe.h2d_bytes(), "d2h_bytes_per_step": pipe.d2h_bytes()},
@@ -373,7 +419,7 @@ def run_conduit(args):
         "status": status,
         "wall_s_timed": round(wall, 3),
     }
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and pipe.plain:  # the oracle arm times the default pass
         out["cpu_baseline"] = cpu_baseline(args.config, args.cpu_seconds, args.ratio)
     if world > 1:
         import torch.distributed as dist
@@ -507,6 +553,12 @@ def main():
     ap.add_argument("--no-graph", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--value-norm", default="v", choices=["v", "side_cache", "none"],
+                    help="value norms from V (default), the side cache (Sec. 4.3), or none")
+    ap.add_argument("--statistic", default="mean", choices=["mean", "rms"],
+                    help="attention statistic in s: mean (Eq. 6, default) or RMS (Eq. 4)")
+    ap.add_argument("--full-context", action="store_true",
+                    help="softmax denominators include outside keys (seeded log-sum-exps)")
     ap.add_argument("--ratio", type=float, default=None,
                     help="refresh ratio r for every request (default: the workload's own)")
     args = ap.parse_args()

@@ -143,6 +143,100 @@ conduit_status conduit_score(const conduit_kv* kv, const conduit_batch* batch, c
                              void* stream);
 
 /*
+ * Scoring variants (conduit_score_ex). The defaults (all fields zero, or a
+ * NULL options pointer) are conduit_score.
+ *  statistic   CONDUIT_STAT_MEAN: s uses a_t^(l) of Eq. 6 (the deployed policy).
+ *              CONDUIT_STAT_RMS: s uses the RMS attention of Eq. 4,
+ *                abar_t^(l) = sqrt( sum_q sum_h alpha^2 / (|Q| Hq) ),
+ *              over the same query rows and heads. attn_sum and g (Eq. 8) keep
+ *              the mean of Eq. 6 in both cases.
+ *  value_norm  CONDUIT_VNORM_FROM_V: v_t^(l) from V (Sec. 3.3).
+ *              CONDUIT_VNORM_SIDE_CACHE: v_t^(l) = vnorm[l][t], the side cache
+ *                of conduit_value_norms (V is not read).
+ *              CONDUIT_VNORM_NONE: v_t^(l) = 1, the score is attention alone
+ *                (the factor ablation that drops the value norm, Sec. 4.4).
+ *  vnorm       device fp32 [L][tok_off[R]]; required with SIDE_CACHE, else NULL.
+ *  extra_lse   device fp32 [L][Hq][Q_tot] (layout of q without d), or NULL.
+ *              When given, alpha_{q,t} is normalised over the whole context
+ *              rather than the visual keys alone: extra_lse[l][h][q] is the
+ *              natural-log log-sum-exp of <q_{l,h,q}, k_j> / sqrt(d) over the
+ *              keys j outside the request's visual span (text, query span),
+ *              -inf where there are none, as a flash-attention pass over those
+ *              keys returns it. The softmax denominator of row (l, h, q)
+ *              becomes sum_{t visual} exp(x_t) + exp(extra_lse), so the alphas
+ *              of a row sum to less than 1.
+ */
+enum { CONDUIT_STAT_MEAN = 0, CONDUIT_STAT_RMS = 1 };
+enum { CONDUIT_VNORM_FROM_V = 0, CONDUIT_VNORM_SIDE_CACHE = 1, CONDUIT_VNORM_NONE = 2 };
+
+typedef struct conduit_score_opts {
+  int32_t statistic;     /* CONDUIT_STAT_* */
+  int32_t value_norm;    /* CONDUIT_VNORM_* */
+  const float* vnorm;    /* side cache (value_norm == CONDUIT_VNORM_SIDE_CACHE) or NULL */
+  const float* extra_lse; /* full-context softmax denominators or NULL */
+} conduit_score_opts;
+
+/*
+ * conduit_score with the variants of `opts` (NULL: the defaults). Arguments,
+ * results and errors are otherwise those of conduit_score; INVALID_ARG also
+ * for an unknown statistic or value_norm, a vnorm that does not match
+ * value_norm, or a misaligned extra_lse. The workspace depends on opts (RMS
+ * adds one partial-sum array, any value_norm but FROM_V drops one).
+ */
+conduit_status conduit_score_ex_workspace_size(const conduit_kv* kv, const conduit_batch* batch,
+                                               int32_t n_layers, const conduit_score_opts* opts,
+                                               size_t* bytes);
+conduit_status conduit_score_ex(const conduit_kv* kv, const conduit_batch* batch, const void* q,
+                                const int32_t* layers, int32_t n_layers,
+                                const conduit_score_opts* opts, float* s, float* attn_sum,
+                                float* g, void* workspace, size_t workspace_bytes,
+                                int32_t* status, void* stream);
+
+/*
+ * Value-norm side cache (Sec. 4.3 and App. C.2: v_t^(l) depends only on the
+ * cached content, so one scalar per token and layer stored when the cache is
+ * built keeps the scores exact and takes the value rows off the scoring
+ * pass).
+ *   vnorm[l][t] = || concat_g V_{l,g,t} ||_2   for every layer l < L and
+ *                 global token row t < tok_off[R]
+ * The norm is computed with the operations, in the order, that conduit_score
+ * uses for this cache, so conduit_score_with_norms over this side cache
+ * returns bitwise the s, attn_sum and g of conduit_score.
+ *  vnorm  device fp32 [L][tok_off[R]], 4-byte aligned (written); caller-owned
+ * Errors: INVALID_ARG for a NULL or misaligned vnorm, UNSUPPORTED for more
+ * than 65535 layers, otherwise as for conduit_score.
+ */
+conduit_status conduit_value_norms(const conduit_kv* kv, const conduit_batch* batch, float* vnorm,
+                                   void* stream);
+
+/*
+ * Keep the side cache exact after conduit_kv_scatter or conduit_kv_exchange
+ * rewrote rows: recompute vnorm[l][tok_off[r] + idx_i] for every layer l and
+ * every selected row i (idx, idx_off, idx_off_dev as for conduit_kv_scatter).
+ * The other entries are left as they are.
+ */
+conduit_status conduit_value_norms_update(const conduit_kv* kv, const conduit_batch* batch,
+                                          const int32_t* idx, const int32_t* idx_off,
+                                          const int32_t* idx_off_dev, float* vnorm, void* stream);
+
+/*
+ * conduit_score with v_t^(l) read from the side cache at vnorm[l][t] (l the
+ * scored layer id) instead of from V: the scoring pass reads K, Q and 4 bytes
+ * per token and layer. All other arguments, results and errors are those of
+ * conduit_score; the workspace is smaller (no value partial sums). Same as
+ * conduit_score_ex with value_norm = CONDUIT_VNORM_SIDE_CACHE.
+ *  vnorm  device fp32 [L][tok_off[R]] from conduit_value_norms (read)
+ */
+conduit_status conduit_score_with_norms_workspace_size(const conduit_kv* kv,
+                                                       const conduit_batch* batch,
+                                                       int32_t n_layers, size_t* bytes);
+conduit_status conduit_score_with_norms(const conduit_kv* kv, const conduit_batch* batch,
+                                        const void* q, const int32_t* layers, int32_t n_layers,
+                                        const float* vnorm, float* s, float* attn_sum, float* g,
+                                        void* workspace, size_t workspace_bytes, int32_t* status,
+                                        void* stream);
+
+/*
  * Image-level amplification and one global top-k per request (Sec. 3.4-3.5,
  * Eqs. 9-11; Algorithm 1 last loops).
  *   c_j    = (1 - lambda) + lambda g_j / g_bar, g_bar = mean of the request's g_j;

@@ -52,6 +52,8 @@ __all__ = [
     "cached_key_logits",
     "softmax_over_visual_keys",
     "head_query_mean_attention",
+    "softmax_with_outside_keys",
+    "head_query_rms_attention",
     "value_norms",
     "throughput_score",
     "image_mean_attention",
@@ -102,22 +104,60 @@ def softmax_over_visual_keys(x: np.ndarray) -> np.ndarray:
     return e / e.sum(axis=1, keepdims=True)
 
 
-def head_query_mean_attention(q_l: np.ndarray, k_l: np.ndarray) -> np.ndarray:
-    """a_t^{(l)} = (1 / (|Q| H)) sum_q sum_h alpha_{q,t,l,h}, Eq. 6.
+def softmax_with_outside_keys(x: np.ndarray, extra_lse: np.ndarray) -> np.ndarray:
+    """alpha[q, t] = exp(x[q,t]) / (sum_u exp(x[q,u]) + exp(extra_lse[q])).
 
-    q_l: [Hq, n_q, d] scoring queries of one layer; k_l: [Hkv, N, d] cached keys.
-    Query head h reads KV head h // G.
+    The full-context reading of the softmax: the keys outside the visual span
+    (text, query span) stay in the denominator, entering through the natural
+    log of their summed exponentials, extra_lse[q] (-inf: no such keys, which
+    gives softmax_over_visual_keys). Shifted by c_q = max(max_u x[q,u], extra_lse[q]).
     """
-    hq, n_q, _ = q_l.shape
-    hkv, n, _ = k_l.shape
+    c = np.maximum(x.max(axis=1), extra_lse)[:, None]
+    e = np.exp(x - c)
+    return e / (e.sum(axis=1, keepdims=True) + np.exp(extra_lse[:, None] - c))
+
+
+def _attention_rows(q_l, k_l, extra_lse_l=None):
+    """alpha of every query head of one layer, [Hq, n_q, N] (head h reads KV head h // G)."""
+    hq = q_l.shape[0]
+    hkv = k_l.shape[0]
     if hq % hkv != 0:
         raise ValueError("Hq must be a multiple of Hkv")
     group = hq // hkv
-    total = np.zeros(n, dtype=np.float64)
+    out = []
     for h in range(hq):
-        alpha = softmax_over_visual_keys(cached_key_logits(q_l[h], k_l[h // group]))
-        total += alpha.sum(axis=0)
-    return total / (n_q * hq)
+        x = cached_key_logits(q_l[h], k_l[h // group])
+        if extra_lse_l is None:
+            out.append(softmax_over_visual_keys(x))
+        else:
+            out.append(softmax_with_outside_keys(x, np.asarray(extra_lse_l[h], dtype=np.float64)))
+    return np.stack(out)
+
+
+def head_query_mean_attention(q_l: np.ndarray, k_l: np.ndarray,
+                              extra_lse_l: Optional[np.ndarray] = None) -> np.ndarray:
+    """a_t^{(l)} = (1 / (|Q| H)) sum_q sum_h alpha_{q,t,l,h}, Eq. 6.
+
+    q_l: [Hq, n_q, d] scoring queries of one layer; k_l: [Hkv, N, d] cached keys.
+    Query head h reads KV head h // G. extra_lse_l: optional [Hq, n_q]
+    outside-key log-sum-exps (full-context softmax).
+    """
+    hq, n_q, _ = q_l.shape
+    alpha = _attention_rows(q_l, k_l, extra_lse_l)
+    return alpha.sum(axis=(0, 1)) / (n_q * hq)
+
+
+def head_query_rms_attention(q_l: np.ndarray, k_l: np.ndarray,
+                             extra_lse_l: Optional[np.ndarray] = None) -> np.ndarray:
+    """abar_t^{(l)} = sqrt((1 / (|Q| H)) sum_q sum_h alpha_{q,t,l,h}^2), Eq. 4.
+
+    The RMS of the cached-key attention over the same query rows and heads
+    that Eq. 6 averages over (Eq. 4 states it for one head; the heads enter
+    as Eq. 6 takes them).
+    """
+    hq, n_q, _ = q_l.shape
+    alpha = _attention_rows(q_l, k_l, extra_lse_l)
+    return np.sqrt((alpha * alpha).sum(axis=(0, 1)) / (n_q * hq))
 
 
 def value_norms(v_l: np.ndarray) -> np.ndarray:
@@ -198,23 +238,47 @@ def topk_select(s_hat: np.ndarray, k: int) -> np.ndarray:
     return np.array(sorted(order[:k]), dtype=np.int64)
 
 
-def score_request(q: np.ndarray, k: np.ndarray, v: np.ndarray,
-                  img_off: Sequence[int], layers: Optional[Sequence[int]] = None) -> dict:
+def score_request(q: np.ndarray, k: np.ndarray, v: Optional[np.ndarray],
+                  img_off: Sequence[int], layers: Optional[Sequence[int]] = None,
+                  vnorm: Optional[np.ndarray] = None, statistic: str = "mean",
+                  use_value_norm: bool = True, extra_lse: Optional[np.ndarray] = None) -> dict:
     """The query-conditioned scoring pass for one request (Algorithm 1, scoring loop).
 
     q: [L, Hq, n_q, d]; k, v: [L, Hkv, N, d] (anything whose [l] gives one
     layer's array); layers: the scored layer set (default all layers, App. A.2).
-    Returns a, vn ([|L|, N]), s, A ([N]) and g ([K]).
+    vnorm: optional stored norms [L, N] (Sec. 4.3 and App. C.2: the value norm
+    depends only on the cached content, so it may be kept per token and layer
+    from cache construction); when given, v_t^{(l)} = vnorm[l, t] and v is not
+    read (it may be None).
+    statistic: "mean" (Eq. 6, the deployed policy) or "rms" (Eq. 4) for the
+    attention factor of s; A and g always use the mean.
+    use_value_norm: False drops the value norm from s (the factor ablation of
+    Sec. 4.4: s ranks by attention alone; v may be None).
+    extra_lse: optional [L, Hq, n_q] outside-key log-sum-exps (full-context
+    softmax, see softmax_with_outside_keys).
+    Returns a, vn ([|L|, N]), stat (the factor used in s), s, A ([N]) and g ([K]).
     """
     f64 = lambda x: np.asarray(x, dtype=np.float64)
+    if statistic not in ("mean", "rms"):
+        raise ValueError("statistic must be 'mean' or 'rms'")
     if layers is None:
         layers = list(range(len(k)))
-    a = np.stack([head_query_mean_attention(f64(q[l]), f64(k[l])) for l in layers])
-    vn = np.stack([value_norms(f64(v[l])) for l in layers])
-    s = throughput_score(a, vn)
+    ex = (lambda l: None) if extra_lse is None else (lambda l: f64(extra_lse[l]))
+    a = np.stack([head_query_mean_attention(f64(q[l]), f64(k[l]), ex(l)) for l in layers])
+    if statistic == "rms":
+        stat = np.stack([head_query_rms_attention(f64(q[l]), f64(k[l]), ex(l)) for l in layers])
+    else:
+        stat = a
+    if not use_value_norm:
+        vn = np.ones_like(a)
+    elif vnorm is None:
+        vn = np.stack([value_norms(f64(v[l])) for l in layers])
+    else:
+        vn = np.stack([f64(vnorm[l]) for l in layers])
+    s = throughput_score(stat, vn)
     attn_sum = a.sum(axis=0)
     g = image_mean_attention(a, img_off)
-    return {"a": a, "vn": vn, "s": s, "A": attn_sum, "g": g}
+    return {"a": a, "vn": vn, "stat": stat, "s": s, "A": attn_sum, "g": g}
 
 
 def refresh_mask(q: np.ndarray, k: np.ndarray, v: np.ndarray, img_off: Sequence[int],

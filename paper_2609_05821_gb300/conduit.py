@@ -22,6 +22,10 @@ OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_CUDA, ERR_NONFINITE, ERR_TIMEOUT, ERR_
 FLAG_NONFINITE, FLAG_TIMEOUT = 1, 2
 F32, BF16 = 0, 1
 MAX_LAYERS = 512
+STAT_MEAN, STAT_RMS = 0, 1
+VNORM_FROM_V, VNORM_SIDE_CACHE, VNORM_NONE = 0, 1, 2
+_STATS = {"mean": STAT_MEAN, "rms": STAT_RMS}
+_VNORMS = {"v": VNORM_FROM_V, "side_cache": VNORM_SIDE_CACHE, "none": VNORM_NONE}
 
 _STATUS_NAMES = {0: "OK", 1: "INVALID_ARG", 2: "UNSUPPORTED", 3: "CUDA", 4: "NONFINITE",
                  5: "TIMEOUT", 6: "WORKSPACE"}
@@ -40,6 +44,13 @@ class ConduitKV(ctypes.Structure):
         ("dtype", ctypes.c_int32), ("page_size", ctypes.c_int32),
         ("num_pages", ctypes.c_int32), ("max_pages_per_req", ctypes.c_int32),
         ("k", ctypes.c_void_p), ("v", ctypes.c_void_p), ("page_table", ctypes.c_void_p),
+    ]
+
+
+class ConduitScoreOpts(ctypes.Structure):
+    _fields_ = [
+        ("statistic", ctypes.c_int32), ("value_norm", ctypes.c_int32),
+        ("vnorm", ctypes.c_void_p), ("extra_lse", ctypes.c_void_p),
     ]
 
 
@@ -67,6 +78,12 @@ def _load():
         "conduit_budget": (I32, [ctypes.c_double, ctypes.c_int64]),
         "conduit_score_workspace_size": (st, [P, P, I32, ctypes.POINTER(SZ)]),
         "conduit_score": (st, [P, P, P, P, I32, P, P, P, P, SZ, P, P]),
+        "conduit_score_ex_workspace_size": (st, [P, P, I32, P, ctypes.POINTER(SZ)]),
+        "conduit_score_ex": (st, [P, P, P, P, I32, P, P, P, P, P, SZ, P, P]),
+        "conduit_value_norms": (st, [P, P, P, P]),
+        "conduit_value_norms_update": (st, [P, P, P, P, P, P, P]),
+        "conduit_score_with_norms_workspace_size": (st, [P, P, I32, ctypes.POINTER(SZ)]),
+        "conduit_score_with_norms": (st, [P, P, P, P, I32, P, P, P, P, P, SZ, P, P]),
         "conduit_select_workspace_size": (st, [P, ctypes.POINTER(SZ)]),
         "conduit_select_topk": (st, [P, P, P, ctypes.c_float, P, P, P, P, P, P, P, SZ, P, P]),
         "conduit_select_topk_noalloc": (st, [P, P, P, ctypes.c_float, P, P, P, P, P, P, P, P]),
@@ -226,6 +243,81 @@ def conduit_score(kv: KvCache, batch: Batch, q: torch.Tensor, layers=None, s=Non
     ws = _workspace(need, dev, workspace)
     _check(_lib.conduit_score(kv.ref(), batch.ref(), _ptr(q), larr, nl, _ptr(s), _ptr(attn_sum),
                               _ptr(g), _ptr(ws), ws.numel(), _ptr(status), _stream_ptr(stream)))
+    return s, attn_sum, g
+
+
+def score_opts(statistic: str = "mean", value_norm: str = "v", vnorm=None, extra_lse=None):
+    """conduit_score_opts: statistic "mean" | "rms", value_norm "v" | "side_cache" | "none"."""
+    o = ConduitScoreOpts()
+    o.statistic = _STATS[statistic]
+    o.value_norm = _VNORMS[value_norm]
+    o.vnorm = None if vnorm is None else vnorm.data_ptr()
+    o.extra_lse = None if extra_lse is None else extra_lse.data_ptr()
+    return o
+
+
+def conduit_score_ex_workspace_size(kv: KvCache, batch: Batch, n_layers: int = 0,
+                                    opts: Optional[ConduitScoreOpts] = None) -> int:
+    n = ctypes.c_size_t(0)
+    _check(_lib.conduit_score_ex_workspace_size(kv.ref(), batch.ref(), int(n_layers),
+                                                None if opts is None else ctypes.byref(opts),
+                                                ctypes.byref(n)))
+    return int(n.value)
+
+
+def conduit_score_ex(kv: KvCache, batch: Batch, q: torch.Tensor, layers=None, statistic="mean",
+                     value_norm="v", vnorm=None, extra_lse=None, s=None, attn_sum=None, g=None,
+                     workspace=None, status=None, stream=None):
+    """Scoring pass with the variants of conduit_score_opts. Returns (s, attn_sum, g)."""
+    dev = kv.k.device
+    larr, nl = _layer_array(layers)
+    opts = score_opts(statistic, value_norm, vnorm, extra_lse)
+    s = torch.empty(batch.n_tot, dtype=torch.float32, device=dev) if s is None else s
+    attn_sum = torch.empty(batch.n_tot, dtype=torch.float32, device=dev) if attn_sum is None else attn_sum
+    g = torch.empty(batch.num_images, dtype=torch.float32, device=dev) if g is None else g
+    ws = _workspace(conduit_score_ex_workspace_size(kv, batch, nl, opts), dev, workspace)
+    _check(_lib.conduit_score_ex(kv.ref(), batch.ref(), _ptr(q), larr, nl, ctypes.byref(opts),
+                                 _ptr(s), _ptr(attn_sum), _ptr(g), _ptr(ws), ws.numel(),
+                                 _ptr(status), _stream_ptr(stream)))
+    return s, attn_sum, g
+
+
+def conduit_value_norms(kv: KvCache, batch: Batch, vnorm=None, stream=None) -> torch.Tensor:
+    """Value-norm side cache vnorm[l][t] = ||concat_g V[l][g][t]|| (fp32 [L, N_tot])."""
+    if vnorm is None:
+        vnorm = torch.empty((kv.num_layers, batch.n_tot), dtype=torch.float32, device=kv.k.device)
+    _check(_lib.conduit_value_norms(kv.ref(), batch.ref(), _ptr(vnorm), _stream_ptr(stream)))
+    return vnorm
+
+
+def conduit_value_norms_update(kv: KvCache, batch: Batch, idx, idx_off, idx_off_dev, vnorm,
+                               stream=None):
+    """Recompute the side-cache entries of the selected rows (after a scatter or exchange)."""
+    _check(_lib.conduit_value_norms_update(kv.ref(), batch.ref(), _ptr(idx), _ptr(idx_off),
+                                           _ptr(idx_off_dev), _ptr(vnorm), _stream_ptr(stream)))
+
+
+def conduit_score_with_norms_workspace_size(kv: KvCache, batch: Batch, n_layers: int = 0) -> int:
+    n = ctypes.c_size_t(0)
+    _check(_lib.conduit_score_with_norms_workspace_size(kv.ref(), batch.ref(), int(n_layers),
+                                                        ctypes.byref(n)))
+    return int(n.value)
+
+
+def conduit_score_with_norms(kv: KvCache, batch: Batch, q: torch.Tensor, vnorm: torch.Tensor,
+                             layers=None, s=None, attn_sum=None, g=None, workspace=None,
+                             status=None, stream=None):
+    """Scoring pass with the value norms from the side cache; V is not read."""
+    dev = kv.k.device
+    larr, nl = _layer_array(layers)
+    s = torch.empty(batch.n_tot, dtype=torch.float32, device=dev) if s is None else s
+    attn_sum = torch.empty(batch.n_tot, dtype=torch.float32, device=dev) if attn_sum is None else attn_sum
+    g = torch.empty(batch.num_images, dtype=torch.float32, device=dev) if g is None else g
+    need = conduit_score_with_norms_workspace_size(kv, batch, nl)
+    ws = _workspace(need, dev, workspace)
+    _check(_lib.conduit_score_with_norms(kv.ref(), batch.ref(), _ptr(q), larr, nl, _ptr(vnorm),
+                                         _ptr(s), _ptr(attn_sum), _ptr(g), _ptr(ws), ws.numel(),
+                                         _ptr(status), _stream_ptr(stream)))
     return s, attn_sum, g
 
 

@@ -148,10 +148,38 @@ struct ScoreLayout {
   int rg_max;  // row groups per slab (column-sum partials per KV head)
   int group_rows;
   int parts;   // partials per row group and per value norm (2 for the tensor-core kernel)
-  size_t stats, pa, ss, attn, total;
+  size_t stats, pa, pa2, ss, attn, total;
 };
 
-ScoreLayout score_layout(const conduit_kv* kv, const conduit_batch* b, int n_layers) {
+// What a scoring call computes (conduit_score_opts with its defaults filled in).
+struct ScoreMode {
+  bool rms;                // RMS statistic in s (Eq. 4) instead of the mean (Eq. 6)
+  int vmode;               // 0 value norms from V, 1 from the side cache, 2 none
+  const float* vnorm;
+  const float* extra_lse;  // full-context softmax denominators, or NULL
+};
+
+conduit_status read_opts(const conduit_score_opts* o, ScoreMode* m) {
+  *m = ScoreMode{false, 0, nullptr, nullptr};
+  if (!o) return CONDUIT_OK;
+  if (o->statistic != CONDUIT_STAT_MEAN && o->statistic != CONDUIT_STAT_RMS)
+    return fail(CONDUIT_ERR_INVALID_ARG, "opts->statistic must be CONDUIT_STAT_MEAN or _RMS");
+  if (o->value_norm < CONDUIT_VNORM_FROM_V || o->value_norm > CONDUIT_VNORM_NONE)
+    return fail(CONDUIT_ERR_INVALID_ARG, "opts->value_norm must be a CONDUIT_VNORM_* value");
+  if ((o->value_norm == CONDUIT_VNORM_SIDE_CACHE) != (o->vnorm != nullptr))
+    return fail(CONDUIT_ERR_INVALID_ARG,
+                "opts->vnorm is required with CONDUIT_VNORM_SIDE_CACHE and must be NULL otherwise");
+  if (o->extra_lse && reinterpret_cast<uintptr_t>(o->extra_lse) % 4)
+    return fail(CONDUIT_ERR_INVALID_ARG, "opts->extra_lse must be 4-byte aligned");
+  *m = ScoreMode{o->statistic == CONDUIT_STAT_RMS, o->value_norm, o->vnorm, o->extra_lse};
+  return CONDUIT_OK;
+}
+
+// Without value partials (vmode != 0) there is no ss region; the RMS
+// statistic adds a pa2 region of the size of pa.
+ScoreLayout score_layout(const conduit_kv* kv, const conduit_batch* b, int n_layers,
+                         const ScoreMode& mode) {
+  const bool normed = mode.vmode != 0;
   const int R = b->num_requests;
   const size_t n_tot = size_t(b->tok_off[R]);
   const size_t q_tot = size_t(b->q_off[R]);
@@ -169,10 +197,14 @@ ScoreLayout score_layout(const conduit_kv* kv, const conduit_batch* b, int n_lay
   size_t off = 0;
   s.stats = off;
   if (!s.tc) off += align_up(size_t(total_rows) * sizeof(float2));  // (max, sum) per row
+  const size_t pa_bytes =
+      align_up(size_t(n_layers) * kv->num_kv_heads * s.rg_max * s.parts * n_tot * sizeof(float));
   s.pa = off;
-  off += align_up(size_t(n_layers) * kv->num_kv_heads * s.rg_max * s.parts * n_tot * sizeof(float));
+  off += pa_bytes;
+  s.pa2 = off;
+  if (mode.rms) off += pa_bytes;
   s.ss = off;
-  off += align_up(size_t(n_layers) * kv->num_kv_heads * s.parts * n_tot * sizeof(float));
+  if (!normed) off += align_up(size_t(n_layers) * kv->num_kv_heads * s.parts * n_tot * sizeof(float));
   s.attn = off;
   off += align_up(n_tot * sizeof(float));
   s.total = off;
@@ -216,6 +248,66 @@ int max_budget(const conduit_batch* b, const int32_t* idx_off) {
   return m;
 }
 
+conduit_status check_norm_cache(const conduit_kv* kv, const float* vnorm) {
+  if (!vnorm) return fail(CONDUIT_ERR_INVALID_ARG, "vnorm is NULL");
+  if (reinterpret_cast<uintptr_t>(vnorm) % 4)
+    return fail(CONDUIT_ERR_INVALID_ARG, "vnorm must be 4-byte aligned");
+  if (kv->num_layers > 65535)
+    return fail(CONDUIT_ERR_UNSUPPORTED, "the norm cache takes at most 65535 layers");
+  return CONDUIT_OK;
+}
+
+// Every scoring entry point: conduit_score_ex with the options read into `mode`.
+conduit_status score_impl(const conduit_kv* kv, const conduit_batch* batch, const void* q,
+                          const int32_t* layers, int32_t n_layers, const ScoreMode& mode, float* s,
+                          float* attn_sum, float* g, void* workspace, size_t workspace_bytes,
+                          int32_t* status, void* stream) {
+  conduit_status st;
+  if ((st = check_batch(batch)) || (st = check_kv(kv, batch))) return st;
+  if (!q || !s || !g) return fail(CONDUIT_ERR_INVALID_ARG, "q, s and g are required");
+  if (!aligned16(q)) return fail(CONDUIT_ERR_INVALID_ARG, "q must be 16-byte aligned");
+  for (int r = 0; r < batch->num_requests; ++r)
+    if (batch->q_off[r + 1] == batch->q_off[r])
+      return fail(CONDUIT_ERR_INVALID_ARG, "request %d has an empty scoring span", r);
+  static thread_local LayerList ll;
+  if ((st = make_layers(kv, layers, n_layers, &ll))) return st;
+  const bool normed = mode.vmode != 0;
+  if (mode.vmode == 1 && (st = check_norm_cache(kv, mode.vnorm))) return st;
+  const ScoreLayout lay = score_layout(kv, batch, ll.n, mode);
+  if ((st = check_workspace(workspace, workspace_bytes, lay.total))) return st;
+
+  const KvDev kd = make_kv(kv, batch);
+  const BatchDev bd = make_batch(batch);
+  const int R = batch->num_requests;
+  int max_tok = 0, max_rows = 0;
+  for (int r = 0; r < R; ++r) {
+    max_tok = std::max(max_tok, batch->tok_off[r + 1] - batch->tok_off[r]);
+    max_rows = std::max(max_rows, kd.G * (batch->q_off[r + 1] - batch->q_off[r]));
+  }
+  char* ws = static_cast<char*>(workspace);
+  float2* stats = reinterpret_cast<float2*>(ws + lay.stats);
+  float* pa = reinterpret_cast<float*>(ws + lay.pa);
+  float* ss = normed ? nullptr : reinterpret_cast<float*>(ws + lay.ss);
+  float* pa2 = mode.rms ? reinterpret_cast<float*>(ws + lay.pa2) : nullptr;
+  float* attn = attn_sum ? attn_sum : reinterpret_cast<float*>(ws + lay.attn);
+  cudaStream_t cs = static_cast<cudaStream_t>(stream);
+  cudaError_t err;
+  if (lay.tc) {  // the tensor-core kernel also streams V for the value norms (unless normed)
+    err = launch_score_tc(kd, bd, batch->q_off, q, batch->q_off[R], ll, lay.rg_max, pa, ss, pa2,
+                          mode.extra_lse, status, cs);
+  } else {
+    if (!normed && (err = launch_value_sumsq(kd, bd, ll, max_tok, ss, cs)))
+      return cuda_fail(err, "value_sumsq");
+    err = launch_score_simt(kd, bd, q, batch->q_off[R], ll, max_rows, max_tok, stats, pa, pa2,
+                            mode.extra_lse, cs);
+  }
+  if (err) return cuda_fail(err, "score");
+  if ((err = launch_finalize(pa, pa2, ss, mode.vnorm, mode.vmode, ll, bd, ll.n, kd.Hkv, kd.Hq,
+                             lay.rg_max, lay.group_rows, lay.parts, kd.n_tot, s, attn, g, status, cs)))
+    return cuda_fail(err, "finalize");
+  return CONDUIT_OK;
+}
+
 }  // namespace
 
 namespace conduit {
@@ -242,7 +334,7 @@ conduit_status conduit_score_workspace_size(const conduit_kv* kv, const conduit_
   if (!bytes) return fail(CONDUIT_ERR_INVALID_ARG, "bytes is NULL");
   if ((st = check_batch(batch)) || (st = check_kv(kv, batch))) return st;
   const int nl = n_layers > 0 ? n_layers : kv->num_layers;
-  *bytes = score_layout(kv, batch, nl).total;
+  *bytes = score_layout(kv, batch, nl, ScoreMode{false, 0, nullptr, nullptr}).total;
   return CONDUIT_OK;
 }
 
@@ -250,44 +342,82 @@ conduit_status conduit_score(const conduit_kv* kv, const conduit_batch* batch, c
                              const int32_t* layers, int32_t n_layers, float* s, float* attn_sum,
                              float* g, void* workspace, size_t workspace_bytes, int32_t* status,
                              void* stream) {
+  return score_impl(kv, batch, q, layers, n_layers, ScoreMode{false, 0, nullptr, nullptr}, s,
+                    attn_sum, g, workspace, workspace_bytes, status, stream);
+}
+
+conduit_status conduit_score_ex_workspace_size(const conduit_kv* kv, const conduit_batch* batch,
+                                               int32_t n_layers, const conduit_score_opts* opts,
+                                               size_t* bytes) {
+  conduit_status st;
+  if (!bytes) return fail(CONDUIT_ERR_INVALID_ARG, "bytes is NULL");
+  if ((st = check_batch(batch)) || (st = check_kv(kv, batch))) return st;
+  ScoreMode mode;
+  if ((st = read_opts(opts, &mode))) return st;
+  const int nl = n_layers > 0 ? n_layers : kv->num_layers;
+  *bytes = score_layout(kv, batch, nl, mode).total;
+  return CONDUIT_OK;
+}
+
+conduit_status conduit_score_ex(const conduit_kv* kv, const conduit_batch* batch, const void* q,
+                                const int32_t* layers, int32_t n_layers,
+                                const conduit_score_opts* opts, float* s, float* attn_sum,
+                                float* g, void* workspace, size_t workspace_bytes,
+                                int32_t* status, void* stream) {
+  conduit_status st;
+  ScoreMode mode;
+  if ((st = read_opts(opts, &mode))) return st;
+  return score_impl(kv, batch, q, layers, n_layers, mode, s, attn_sum, g, workspace,
+                    workspace_bytes, status, stream);
+}
+
+conduit_status conduit_value_norms(const conduit_kv* kv, const conduit_batch* batch, float* vnorm,
+                                   void* stream) {
   conduit_status st;
   if ((st = check_batch(batch)) || (st = check_kv(kv, batch))) return st;
-  if (!q || !s || !g) return fail(CONDUIT_ERR_INVALID_ARG, "q, s and g are required");
-  if (!aligned16(q)) return fail(CONDUIT_ERR_INVALID_ARG, "q must be 16-byte aligned");
-  for (int r = 0; r < batch->num_requests; ++r)
-    if (batch->q_off[r + 1] == batch->q_off[r])
-      return fail(CONDUIT_ERR_INVALID_ARG, "request %d has an empty scoring span", r);
-  static thread_local LayerList ll;
-  if ((st = make_layers(kv, layers, n_layers, &ll))) return st;
-  const ScoreLayout lay = score_layout(kv, batch, ll.n);
-  if ((st = check_workspace(workspace, workspace_bytes, lay.total))) return st;
-
-  const KvDev kd = make_kv(kv, batch);
-  const BatchDev bd = make_batch(batch);
-  const int R = batch->num_requests;
-  int max_tok = 0, max_rows = 0;
-  for (int r = 0; r < R; ++r) {
-    max_tok = std::max(max_tok, batch->tok_off[r + 1] - batch->tok_off[r]);
-    max_rows = std::max(max_rows, kd.G * (batch->q_off[r + 1] - batch->q_off[r]));
-  }
-  char* ws = static_cast<char*>(workspace);
-  float2* stats = reinterpret_cast<float2*>(ws + lay.stats);
-  float* pa = reinterpret_cast<float*>(ws + lay.pa);
-  float* ss = reinterpret_cast<float*>(ws + lay.ss);
-  float* attn = attn_sum ? attn_sum : reinterpret_cast<float*>(ws + lay.attn);
-  cudaStream_t cs = static_cast<cudaStream_t>(stream);
-  cudaError_t err;
-  if (lay.tc) {  // the tensor-core kernel also streams V for the value norms
-    err = launch_score_tc(kd, bd, batch->q_off, q, batch->q_off[R], ll, lay.rg_max, pa, ss, status, cs);
-  } else {
-    if ((err = launch_value_sumsq(kd, bd, ll, max_tok, ss, cs))) return cuda_fail(err, "value_sumsq");
-    err = launch_score_simt(kd, bd, q, batch->q_off[R], ll, max_rows, max_tok, stats, pa, cs);
-  }
-  if (err) return cuda_fail(err, "score");
-  if ((err = launch_finalize(pa, ss, bd, ll.n, kd.Hkv, kd.Hq, lay.rg_max, lay.group_rows, lay.parts, kd.n_tot,
-                             s, attn, g, status, cs)))
-    return cuda_fail(err, "finalize");
+  if ((st = check_norm_cache(kv, vnorm))) return st;
+  cudaError_t err = launch_value_norms(make_kv(kv, batch), make_batch(batch), nullptr, nullptr,
+                                       batch->tok_off[batch->num_requests], vnorm,
+                                       static_cast<cudaStream_t>(stream));
+  if (err) return cuda_fail(err, "value_norms");
   return CONDUIT_OK;
+}
+
+conduit_status conduit_value_norms_update(const conduit_kv* kv, const conduit_batch* batch,
+                                          const int32_t* idx, const int32_t* idx_off,
+                                          const int32_t* idx_off_dev, float* vnorm, void* stream) {
+  conduit_status st;
+  if ((st = check_batch(batch)) || (st = check_kv(kv, batch))) return st;
+  if ((st = check_selection(batch, idx_off, idx_off_dev, true, idx))) return st;
+  if ((st = check_norm_cache(kv, vnorm))) return st;
+  cudaError_t err = launch_value_norms(make_kv(kv, batch), make_batch(batch), idx, idx_off_dev,
+                                       idx_off[batch->num_requests], vnorm,
+                                       static_cast<cudaStream_t>(stream));
+  if (err) return cuda_fail(err, "value_norms_update");
+  return CONDUIT_OK;
+}
+
+conduit_status conduit_score_with_norms_workspace_size(const conduit_kv* kv,
+                                                       const conduit_batch* batch,
+                                                       int32_t n_layers, size_t* bytes) {
+  conduit_status st;
+  if (!bytes) return fail(CONDUIT_ERR_INVALID_ARG, "bytes is NULL");
+  if ((st = check_batch(batch)) || (st = check_kv(kv, batch))) return st;
+  const int nl = n_layers > 0 ? n_layers : kv->num_layers;
+  *bytes = score_layout(kv, batch, nl, ScoreMode{false, 1, nullptr, nullptr}).total;
+  return CONDUIT_OK;
+}
+
+conduit_status conduit_score_with_norms(const conduit_kv* kv, const conduit_batch* batch,
+                                        const void* q, const int32_t* layers, int32_t n_layers,
+                                        const float* vnorm, float* s, float* attn_sum, float* g,
+                                        void* workspace, size_t workspace_bytes, int32_t* status,
+                                        void* stream) {
+  conduit_status st;
+  if ((st = check_batch(batch)) || (st = check_kv(kv, batch))) return st;
+  if ((st = check_norm_cache(kv, vnorm))) return st;
+  return score_impl(kv, batch, q, layers, n_layers, ScoreMode{false, 1, vnorm, nullptr}, s,
+                    attn_sum, g, workspace, workspace_bytes, status, stream);
 }
 
 conduit_status conduit_select_workspace_size(const conduit_batch* batch, size_t* bytes) {

@@ -115,7 +115,8 @@ __global__ void __launch_bounds__(kThreads) rowstats_kernel(KvDev kv, BatchDev b
 template <typename T>
 __global__ void __launch_bounds__(kThreads) colsum_kernel(KvDev kv, BatchDev b, const T* q,
                                                           int32_t q_tot, LayerList layers,
-                                                          const float2* stats, float* pa) {
+                                                          const float2* stats, float* pa,
+                                                          float* pa2, const float* extra_lse) {
   extern __shared__ float smem[];
   const int d = kv.d, ld = d + 1;
   float* q_s = smem;
@@ -123,6 +124,7 @@ __global__ void __launch_bounds__(kThreads) colsum_kernel(KvDev kv, BatchDev b, 
   __shared__ int64_t q_off_s[kRowBlock], k_off_s[kTokTile];
   __shared__ float lse_s[kRowBlock];
   __shared__ float red_s[kThreads / 32][kTokTile];
+  __shared__ float red2_s[kThreads / 32][kTokTile];
 
   const int r = blockIdx.z;
   const int li = blockIdx.y / kv.Hkv, g = blockIdx.y % kv.Hkv;
@@ -144,6 +146,7 @@ __global__ void __launch_bounds__(kThreads) colsum_kernel(KvDev kv, BatchDev b, 
   const int i = threadIdx.x / 8, j = threadIdx.x % 8;
   const float scale = kLog2e * rsqrtf(float(d));
   float acc[4] = {0.f, 0.f, 0.f, 0.f};
+  float acc2[4] = {0.f, 0.f, 0.f, 0.f};
 
   for (int row0 = 0; row0 < R; row0 += kRowBlock) {
     __syncthreads();
@@ -156,6 +159,8 @@ __global__ void __launch_bounds__(kThreads) colsum_kernel(KvDev kv, BatchDev b, 
         off = ((int64_t(l) * kv.Hq + h) * q_tot + q0 + qi) * d;
         const float2 st = stats[sbase + rr];
         lse = st.x + log2f(st.y);
+        if (extra_lse)  // full-context softmax: keys outside the visual span join the denominator
+          lse = log2_add(lse, extra_lse[(int64_t(l) * kv.Hq + h) * q_tot + q0 + qi] * kLog2e);
       }
       q_off_s[threadIdx.x] = off;
       lse_s[threadIdx.x] = lse;
@@ -174,16 +179,25 @@ __global__ void __launch_bounds__(kThreads) colsum_kernel(KvDev kv, BatchDev b, 
 #pragma unroll
     for (int m = 0; m < 4; ++m) {
       float p = (row_ok && tt + j + 8 * m < N) ? exp2f(x[m] * scale - lse) : 0.f;
+      float p2 = p * p;
       // sum over the 4 rows of this warp that share token lane j
       p += __shfl_xor_sync(0xffffffffu, p, 8);
       p += __shfl_xor_sync(0xffffffffu, p, 16);
       acc[m] += p;
+      if (pa2) {
+        p2 += __shfl_xor_sync(0xffffffffu, p2, 8);
+        p2 += __shfl_xor_sync(0xffffffffu, p2, 16);
+        acc2[m] += p2;
+      }
     }
   }
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   if (lane < 8) {
 #pragma unroll
-    for (int m = 0; m < 4; ++m) red_s[warp][lane + 8 * m] = acc[m];
+    for (int m = 0; m < 4; ++m) {
+      red_s[warp][lane + 8 * m] = acc[m];
+      red2_s[warp][lane + 8 * m] = acc2[m];
+    }
   }
   __syncthreads();
   if (threadIdx.x < kTokTile && tt + threadIdx.x < N) {
@@ -191,6 +205,12 @@ __global__ void __launch_bounds__(kThreads) colsum_kernel(KvDev kv, BatchDev b, 
 #pragma unroll
     for (int w = 0; w < kThreads / 32; ++w) sum += red_s[w][threadIdx.x];
     pa[int64_t(blockIdx.y) * kv.n_tot + t0 + tt + threadIdx.x] = sum;
+    if (pa2) {
+      float sum2 = 0.f;
+#pragma unroll
+      for (int w = 0; w < kThreads / 32; ++w) sum2 += red2_s[w][threadIdx.x];
+      pa2[int64_t(blockIdx.y) * kv.n_tot + t0 + tt + threadIdx.x] = sum2;
+    }
   }
 }
 
@@ -198,27 +218,13 @@ __global__ void __launch_bounds__(kThreads) colsum_kernel(KvDev kv, BatchDev b, 
 template <typename T>
 __global__ void __launch_bounds__(256) value_sumsq_kernel(KvDev kv, BatchDev b, LayerList layers,
                                                           float* ss) {
-  constexpr int VEC = 16 / sizeof(T);
   const int r = blockIdx.y, li = blockIdx.z, l = layers.ids[li];
   const int t0 = b.tok_off[r], N = b.tok_off[r + 1] - t0;
   const int t = blockIdx.x * 8 + threadIdx.x / 32, lane = threadIdx.x % 32;
   if (t >= N) return;
-  const int cpr = kv.d / VEC;            // 16-byte chunks per head row
   const T* vb = static_cast<const T*>(kv.v);
   for (int g = 0; g < kv.Hkv; ++g) {
-    const int64_t base = kv.row(l, g, r, int64_t(t0) + t, t);
-    float acc = 0.f;
-    for (int c = lane; c < cpr; c += 32) {
-      const uint4 raw = *reinterpret_cast<const uint4*>(vb + base + c * VEC);
-      const T* vals = reinterpret_cast<const T*>(&raw);
-#pragma unroll
-      for (int u = 0; u < VEC; ++u) {
-        const float x = to_float(vals[u]);
-        acc = fmaf(x, x, acc);
-      }
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    const float acc = warp_row_sumsq(vb + kv.row(l, g, r, int64_t(t0) + t, t), kv.d, lane);
     if (lane == 0) ss[(int64_t(li) * kv.Hkv + g) * kv.n_tot + t0 + t] = acc;
   }
 }
@@ -239,7 +245,8 @@ cudaError_t launch_value_sumsq(const KvDev& kv, const BatchDev& b, const LayerLi
 
 cudaError_t launch_score_simt(const KvDev& kv, const BatchDev& b, const void* q, int32_t q_tot,
                               const LayerList& layers, int max_rows, int max_tokens,
-                              float2* stats, float* pa, cudaStream_t stream) {
+                              float2* stats, float* pa, float* pa2, const float* extra_lse,
+                              cudaStream_t stream) {
   if (layers.n == 0 || max_rows == 0 || max_tokens == 0) return cudaSuccess;
   const size_t smem = size_t(kRowBlock + kTokTile) * (kv.d + 1) * sizeof(float);
   const dim3 g1((max_rows + kRowBlock - 1) / kRowBlock, layers.n * kv.Hkv, b.R);
@@ -253,7 +260,7 @@ cudaError_t launch_score_simt(const KvDev& kv, const BatchDev& b, const void* q,
     const auto* qq = static_cast<const __nv_bfloat16*>(q);
     f1<<<g1, kThreads, smem, stream>>>(kv, b, qq, q_tot, layers, stats);
     if ((err = cudaGetLastError())) return err;
-    f2<<<g2, kThreads, smem, stream>>>(kv, b, qq, q_tot, layers, stats, pa);
+    f2<<<g2, kThreads, smem, stream>>>(kv, b, qq, q_tot, layers, stats, pa, pa2, extra_lse);
   } else {
     auto* f1 = rowstats_kernel<float>;
     auto* f2 = colsum_kernel<float>;
@@ -262,7 +269,7 @@ cudaError_t launch_score_simt(const KvDev& kv, const BatchDev& b, const void* q,
     const auto* qq = static_cast<const float*>(q);
     f1<<<g1, kThreads, smem, stream>>>(kv, b, qq, q_tot, layers, stats);
     if ((err = cudaGetLastError())) return err;
-    f2<<<g2, kThreads, smem, stream>>>(kv, b, qq, q_tot, layers, stats, pa);
+    f2<<<g2, kThreads, smem, stream>>>(kv, b, qq, q_tot, layers, stats, pa, pa2, extra_lse);
   }
   count_launches(2);
   return cudaGetLastError();

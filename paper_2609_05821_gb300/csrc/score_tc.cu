@@ -20,7 +20,8 @@
 //   warp 0       TMA loads of K tiles (128 tokens x 128 dims, 128-byte
 //                swizzle) into a three-stage ring, the lanes issuing a tile's
 //                copies together (one per page half when paged)
-//   warp 10      the same for the matching V tiles of pass A (two buffers)
+//   warp 10      the same for the matching V tiles of pass A (two buffers);
+//                idle when the value norms come from the side cache
 //   warp 1       one thread issues tcgen05 MMAs into two 256-column TMEM
 //                accumulator slots (it also owns the TMEM allocation)
 //   warps 2-9    epilogue, two warps per TMEM lane quarter (warp group h
@@ -62,7 +63,10 @@ struct TcArgs {
   int32_t rg_max;      // row groups per slab, maximum over requests (pa stride)
   float scale_log2;    // log2(e) / sqrt(d)
   float* pa;           // [n_layers][Hkv][rg_max][2][n_tot]
-  float* ss;           // [n_layers][Hkv][2][n_tot] sum of squares of V, per half of the head
+  float* ss;           // [n_layers][Hkv][2][n_tot] sum of squares of V, per half of the head;
+                       // NULL when the norms come from the side cache (V is not read)
+  float* pa2;          // like pa, sums of alpha^2 (RMS statistic, Eq. 4), or NULL
+  const float* extra_lse;  // [L][Hq][q_tot] natural-log LSE of keys outside the visual span, or NULL
   int32_t* status;
   LayerList layers;
 };
@@ -285,6 +289,28 @@ __device__ __forceinline__ float col_sum(const float (&v)[NC], const float* nlse
   return (ac[0].x + ac[0].y) + (ac[1].x + ac[1].y);
 }
 
+// col_sum that also returns the sum of the squared terms (alpha^2, for the
+// RMS statistic); the plain sum is computed exactly as col_sum computes it.
+template <int NC>
+__device__ __forceinline__ float col_sum_sq(const float (&v)[NC], const float* nlse, float scale,
+                                            float& sq) {
+  const float2 sc2 = make_float2(scale, scale);
+  float2 ac[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+  float2 aq[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+#pragma unroll
+  for (int x4 = 0; x4 < NC / 4; ++x4) {
+    const float4 lv = reinterpret_cast<const float4*>(nlse)[x4];
+    const float2 p0 = exp2_pair(v[4 * x4 + 0], v[4 * x4 + 1], sc2, make_float2(lv.x, lv.y), 2 * x4);
+    const float2 p1 = exp2_pair(v[4 * x4 + 2], v[4 * x4 + 3], sc2, make_float2(lv.z, lv.w), 2 * x4 + 1);
+    ac[0] = tc::fadd2(ac[0], p0);
+    ac[1] = tc::fadd2(ac[1], p1);
+    aq[0] = tc::ffma2(p0, p0, aq[0]);
+    aq[1] = tc::ffma2(p1, p1, aq[1]);
+  }
+  sq = (aq[0].x + aq[0].y) + (aq[1].x + aq[1].y);
+  return (ac[0].x + ac[0].y) + (ac[1].x + ac[1].y);
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
     score_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
                     const __grid_constant__ TcArgs a) {
@@ -340,7 +366,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // V tiles of pass 1 for the value norms, on a warp of their own so that a
     // V tile waiting for its buffer never holds back the K ring
     uint32_t vseq = 0;
-    bool ok = true;
+    bool ok = a.ss != nullptr;  // no V traffic when the norms come from the side cache
     for (int u = blockIdx.x; u < a.n_units && ok; u += gridDim.x) {
       Unit w;
       if (!decode_unit(a, u, w) || w.rg != 0) continue;
@@ -446,9 +472,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       // only does value norms) and this thread's half of each V row
       const bool do_rows = nrb == 2 || h == 0;
       const int rb = nrb == 2 ? h : 0;
-      const bool do_norm = w.rg == 0;  // one row group of each slab also streams V
+      const bool do_norm = w.rg == 0 && a.ss != nullptr;  // one row group of each slab also streams V
       const int64_t lg = int64_t(w.li) * a.kv.Hkv + w.g;
-      float* ss_out = a.ss + (lg * 2 + h) * n_tot + w.t0;
+      float* ss_out = do_norm ? a.ss + (lg * 2 + h) * n_tot + w.t0 : nullptr;
       float m = -INFINITY, z = 0.f;
       for (int i = 0; i < w.tiles; ++i) {            // pass A
         const int slot = tseq & 1;
@@ -486,25 +512,25 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint8_t* vh = s.v + vb * kStageBytes + h * kHalfK;
           float sq[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-          for (int c = 0; c < 8; ++c) {
-            const uint4 x = *reinterpret_cast<const uint4*>(vh + tc::sw128_offset(lrow, c));
-            const __nv_bfloat162* hv = reinterpret_cast<const __nv_bfloat162*>(&x);
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const float2 f = __bfloat1622float2(hv[e]);
-              sq[e] = fmaf(f.x, f.x, fmaf(f.y, f.y, sq[e]));
-            }
-          }
+          for (int c = 0; c < 8; ++c)
+            sumsq_bf16_chunk(*reinterpret_cast<const uint4*>(vh + tc::sw128_offset(lrow, c)), sq);
           tc::mbar_arrive(&s.vempty[vb]);
           const int tok = i * kTile + lrow;
-          if (tok < w.N) ss_out[tok] = (sq[0] + sq[1]) + (sq[2] + sq[3]);
+          if (tok < w.N) ss_out[tok] = sumsq_combine(sq);
         }
       }
       // minus the log2-sum-exp of each row, shared with the token-owning
       // threads of pass B (-inf past the row group: those columns add nothing)
       {
         const int row = (do_rows ? rb : 1) * 128 + lrow;
-        s.lse[row] = (do_rows && row < w.rows) ? -(m * a.scale_log2 + log2f(z)) : -INFINITY;
+        float lse = (do_rows && row < w.rows) ? m * a.scale_log2 + log2f(z) : INFINITY;
+        if (a.extra_lse != nullptr && do_rows && row < w.rows) {
+          // full-context softmax: the keys outside the visual span join the denominator
+          const int j = w.row0 + row, hq = w.g * a.kv.G + j / w.nq, qi = j % w.nq;
+          const float e = a.extra_lse[(int64_t(w.l) * a.kv.Hq + hq) * a.q_tot + w.q0 + qi];
+          lse = log2_add(lse, e * kLog2e);
+        }
+        s.lse[row] = -lse;
       }
       epi_barrier();
       // pass B share: 32-row chunks [cb0, cb1)
@@ -512,6 +538,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int hc = (nchunk + 1) / 2;
       const int cb0 = h * hc, cb1 = min(nchunk, cb0 + hc);
       float* pa_out = a.pa + ((lg * a.rg_max + w.rg) * 2 + h) * n_tot + w.t0;
+      float* pa2_out = a.pa2 ? a.pa2 + ((lg * a.rg_max + w.rg) * 2 + h) * n_tot + w.t0 : nullptr;
       for (int i = w.tiles; i < 2 * w.tiles; ++i) {  // pass B
         const int slot = tseq & 1;
         const int tok = tile_of(w, i) * kTile + lrow;
@@ -529,7 +556,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t col0 = uint32_t(slot) * kSlotCols + cb0 * 32;
         const int ncol = (cb1 - cb0) * 32;
         const float* lse = s.lse + cb0 * 32;
-        float acc = 0.f;
+        float acc = 0.f, acc2 = 0.f;
         int c = 0;
         for (; c + 64 <= ncol; c += 64) {
           float v[64];
@@ -538,19 +565,34 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc::tc_fence_before();
             tc::mbar_arrive(&s.tempty[slot]);
           }
-          acc += col_sum<64>(v, lse + c, a.scale_log2);
+          if (pa2_out) {
+            float q2;
+            acc += col_sum_sq<64>(v, lse + c, a.scale_log2, q2);
+            acc2 += q2;
+          } else {
+            acc += col_sum<64>(v, lse + c, a.scale_log2);
+          }
         }
         if (c < ncol) {
           float v[32];
           tc::tmem_ld32(tmem + lane_base + col0 + c, v);
           tc::tc_fence_before();
           tc::mbar_arrive(&s.tempty[slot]);
-          acc += col_sum<32>(v, lse + c, a.scale_log2);
+          if (pa2_out) {
+            float q2;
+            acc += col_sum_sq<32>(v, lse + c, a.scale_log2, q2);
+            acc2 += q2;
+          } else {
+            acc += col_sum<32>(v, lse + c, a.scale_log2);
+          }
         } else if (ncol == 0) {
           tc::tc_fence_before();
           tc::mbar_arrive(&s.tempty[slot]);
         }
-        if (tok < w.N) pa_out[tok] = acc;
+        if (tok < w.N) {
+          pa_out[tok] = acc;
+          if (pa2_out) pa2_out[tok] = acc2;
+        }
       }
       epi_barrier();  // every thread is done with this unit's rows and lse
     }
@@ -598,7 +640,8 @@ int score_tc_groups(int rows) { return n_groups(rows); }
 
 cudaError_t launch_score_tc(const KvDev& kv, const BatchDev& b, const int32_t* q_off_host,
                             const void* q, int32_t q_tot, const LayerList& layers, int rg_max,
-                            float* pa, float* ss, int32_t* status, cudaStream_t stream) {
+                            float* pa, float* ss, float* pa2, const float* extra_lse,
+                            int32_t* status, cudaStream_t stream) {
   EncodeTiledFn enc = encode_fn();
   if (!enc) return cudaErrorNotSupported;
   CUtensorMap kmap, vmap;
@@ -617,7 +660,7 @@ cudaError_t launch_score_tc(const KvDev& kv, const BatchDev& b, const int32_t* q
           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
     return cudaErrorInvalidValue;
-  if (enc(&vmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, kv.v, dims, strides, box, estr,
+  if (enc(&vmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, ss ? kv.v : kv.k, dims, strides, box, estr,
           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
     return cudaErrorInvalidValue;
@@ -635,6 +678,8 @@ cudaError_t launch_score_tc(const KvDev& kv, const BatchDev& b, const int32_t* q
   a.scale_log2 = kLog2e / sqrtf(float(kD));
   a.pa = pa;
   a.ss = ss;
+  a.pa2 = pa2;
+  a.extra_lse = extra_lse;
   a.status = status;
   a.layers = layers;
   if (units == 0) return cudaSuccess;

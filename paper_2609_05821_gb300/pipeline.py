@@ -6,6 +6,13 @@
   3. conduit_kv_exchange  stale K/V rows of the selected tokens out, fresh rows in
                           (conduit_kv_gather + conduit_kv_scatter in one launch)
   4. conduit_refresh_attn causal attention of the refreshed rows over the patched cache
+Scoring variants (conduit_score_ex): ``statistic="rms"`` (Eq. 4),
+``value_norm="none"`` (attention alone) and ``extra_lse`` (full-context
+softmax). With ``value_norm="side_cache"`` the pipeline keeps the value-norm
+side cache (Sec. 4.3, App. C.2): it is built once at construction
+(conduit_value_norms), step 1 reads it instead of V, and step 3 is followed by
+conduit_value_norms_update for the rewritten rows, so every step's scores are
+bitwise those of the pass that reads V.
 All buffers are allocated once at construction, so a step allocates nothing
 and can be captured in a CUDA graph (``capture()``). ``step_from_host()`` is
 the end-to-end form: it copies the step's inputs from pinned host memory,
@@ -26,7 +33,8 @@ class RefreshPipeline:
                  tok_off, img_off, req_img_off, q_off, ratios: Sequence[float],
                  fresh: dict, lam: float = 1.0, layers: Optional[Sequence[int]] = None,
                  page_size: int = 0, page_table: Optional[torch.Tensor] = None,
-                 budgets: Optional[Sequence[int]] = None):
+                 budgets: Optional[Sequence[int]] = None, statistic: str = "mean",
+                 value_norm: str = "v", extra_lse: Optional[torch.Tensor] = None):
         dev = k.device
         self.device = dev
         self.kv = C.KvCache(k, v, num_q_heads, page_size, page_table)
@@ -52,7 +60,11 @@ class RefreshPipeline:
         self.idx = torch.empty(max(self.n_sel, 1), dtype=torch.int32, device=dev)
         self.status = torch.zeros(1, dtype=torch.int32, device=dev)
         nl = 0 if self.layers is None else len(self.layers)
-        self.ws_score = torch.empty(max(C.conduit_score_workspace_size(self.kv, self.batch, nl), 1),
+        self.statistic, self.value_norm, self.extra_lse = statistic, value_norm, extra_lse
+        self.vnorm = C.conduit_value_norms(self.kv, self.batch) if value_norm == "side_cache" else None
+        self.plain = statistic == "mean" and value_norm == "v" and extra_lse is None
+        opts = C.score_opts(statistic, value_norm, self.vnorm, extra_lse)
+        self.ws_score = torch.empty(max(C.conduit_score_ex_workspace_size(self.kv, self.batch, nl, opts), 1),
                                     dtype=torch.uint8, device=dev)
         self.ws_sel = torch.empty(max(C.conduit_select_workspace_size(self.batch), 1),
                                   dtype=torch.uint8, device=dev)
@@ -69,18 +81,41 @@ class RefreshPipeline:
         self.graph = None
 
     # ----------------------------------------------------------------- steps
-    def score_select(self, stream=None):
-        C.conduit_score(self.kv, self.batch, self.q, self.layers, self.s, self.attn_sum, self.g,
-                        self.ws_score, self.status, stream)
+    def score(self, stream=None):
+        if self.plain:
+            C.conduit_score(self.kv, self.batch, self.q, self.layers, self.s, self.attn_sum, self.g,
+                            self.ws_score, self.status, stream)
+        else:
+            C.conduit_score_ex(self.kv, self.batch, self.q, self.layers, self.statistic,
+                               self.value_norm, self.vnorm, self.extra_lse, self.s, self.attn_sum,
+                               self.g, self.ws_score, self.status, stream)
+
+    def select(self, stream=None):
         C.conduit_select_topk(self.batch, self.s, self.g, self.lam, self.idx_off, self.idx_off_dev,
                               self.idx, self.mask, self.s_hat, self.coeff, self.ws_sel,
                               self.status, stream)
 
-    def refresh(self, stream=None):
+    def exchange(self, stream=None):
         C.conduit_kv_exchange(self.kv, self.batch, self.idx, self.idx_off, self.idx_off_dev,
                               self.k_old, self.v_old, self.k_rows, self.v_rows, stream)
+
+    def norm_update(self, stream=None):
+        if self.vnorm is not None:
+            C.conduit_value_norms_update(self.kv, self.batch, self.idx, self.idx_off, self.idx_off_dev,
+                                         self.vnorm, stream)
+
+    def refresh_attn(self, stream=None):
         C.conduit_refresh_attn(self.kv, self.batch, self.idx, self.idx_off, self.idx_off_dev,
                                self.q_rows, self.out, self.ws_ref, self.status, stream)
+
+    def score_select(self, stream=None):
+        self.score(stream)
+        self.select(stream)
+
+    def refresh(self, stream=None):
+        self.exchange(stream)
+        self.norm_update(stream)
+        self.refresh_attn(stream)
 
     def step(self, stream=None):
         """One pass of the whole hot path (launches only; asynchronous)."""
@@ -134,7 +169,8 @@ class RefreshPipeline:
 
 
 def from_inputs(inputs: dict, lam: float = 1.0, paged: Optional[bool] = None,
-                layers=None, budgets=None, fresh: Optional[dict] = None) -> RefreshPipeline:
+                layers=None, budgets=None, fresh: Optional[dict] = None,
+                **score_variant) -> RefreshPipeline:
     """A pipeline over a batch drawn by ``synth.make_inputs``."""
     from . import synth
     w = inputs["workload"]
@@ -153,4 +189,5 @@ def from_inputs(inputs: dict, lam: float = 1.0, paged: Optional[bool] = None,
         v, _ = synth.to_paged(inputs["v"], tok, ps, w.seed)
     return RefreshPipeline(k, v, inputs["q"], w.num_q_heads, inputs["tok_off"], inputs["img_off"],
                            inputs["req_img_off"], inputs["q_off"], inputs["ratios"], fresh, lam=lam,
-                           layers=layers, page_size=ps, page_table=table, budgets=budgets)
+                           layers=layers, page_size=ps, page_table=table, budgets=budgets,
+                           **score_variant)

@@ -33,7 +33,7 @@ from typing import List, Optional, Sequence
 import torch
 
 __all__ = ["Workload", "WORKLOADS", "workload", "make_inputs", "make_fresh_rows",
-           "to_paged", "request_view"]
+           "make_extra_lse", "to_paged", "request_view"]
 
 
 @dataclasses.dataclass(frozen=True)
@@ -206,6 +206,24 @@ def make_fresh_rows(w: Workload, n_sel_total: int, device="cpu", seed: Optional[
         "k_rows": torch.randn(shape_kv, generator=gen, device=dev, dtype=torch.float32).to(dt),
         "v_rows": torch.randn(shape_kv, generator=gen, device=dev, dtype=torch.float32).to(dt),
     }
+
+
+def make_extra_lse(inputs: dict, seed: int = 7) -> torch.Tensor:
+    """Outside-key log-sum-exps for the full-context softmax, fp32 [L, Hq, Q_tot].
+
+    A stand-in for what a prefill over the text and query-span keys would
+    return per scoring row: the request's own visual scale log(N_r) plus a
+    N(0, 4) spread, and one row in ten with no outside keys (-inf). Seeded.
+    """
+    L, Hq, q_tot, _ = inputs["q"].shape
+    tok = inputs["tok_off"].tolist()
+    q_off = inputs["q_off"].tolist()
+    gen = torch.Generator(device="cpu").manual_seed(seed)
+    e = torch.randn((L, Hq, q_tot), generator=gen, dtype=torch.float32) * 2.0
+    for r in range(len(tok) - 1):
+        e[:, :, q_off[r]:q_off[r + 1]] += float(math.log(max(tok[r + 1] - tok[r], 2)))
+    e[torch.rand((L, Hq, q_tot), generator=gen) < 0.1] = -float("inf")
+    return e.to(inputs["q"].device)
 
 
 def to_paged(k: torch.Tensor, tok_off: Sequence[int], page_size: int, seed: int) -> tuple:

@@ -34,7 +34,9 @@ def test_header_declares_the_boundary():
     names = _declared()
     for want in ("conduit_score", "conduit_select_topk", "conduit_refresh_attn", "conduit_kv_scatter",
                  "conduit_kv_gather", "conduit_budget", "conduit_score_workspace_size",
-                 "conduit_read_status"):
+                 "conduit_read_status", "conduit_value_norms", "conduit_value_norms_update",
+                 "conduit_score_with_norms", "conduit_score_with_norms_workspace_size",
+                 "conduit_score_ex", "conduit_score_ex_workspace_size"):
         assert want in names
 
 
@@ -145,6 +147,79 @@ def test_kv_copy_and_refresh_reject_bad_arguments(C):
     kvp = C.KvCache(paged, torch.zeros_like(paged), 4, 16, table)
     _expect(C, C.ERR_INVALID_ARG, C.conduit_kv_scatter, kvp, b, idx, off, off_d, rows, rows,
             match="page-table")
+
+
+def test_norm_side_cache_rejects_bad_arguments(C):
+    kv, b = _kv(C), _batch(C)
+    lib = C._lib
+    q = torch.zeros((2, 4, 8, 64), dtype=torch.bfloat16)
+    vn = torch.zeros((2, 128))
+    # a NULL or misaligned side cache
+    assert lib.conduit_value_norms(kv.ref(), b.ref(), None, None) == C.ERR_INVALID_ARG
+    assert "vnorm" in lib.conduit_last_error_string().decode()
+    odd = ctypes.c_void_p(vn.data_ptr() + 2)
+    assert lib.conduit_value_norms(kv.ref(), b.ref(), odd, None) == C.ERR_INVALID_ARG
+    # the batch and cache checks of the scoring pass apply
+    bad = _batch(C, img=(0, 70, 64, 128))
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_value_norms, kv, bad, vn, match="empty or out of order")
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_score_with_norms, kv, bad, q, vn)
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_score_with_norms, kv, b, q, vn, [1, 0], match="increasing")
+    # the update takes a selection like the scatter
+    off, off_d = C.idx_offsets([3, 4], "cpu")
+    bad_off = torch.tensor([1, 3, 7], dtype=torch.int32)
+    idx = torch.zeros(7, dtype=torch.int32)
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_value_norms_update, kv, b, idx, bad_off, off_d, vn)
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_value_norms_update, kv, b, None, off, off_d, vn)
+    assert lib.conduit_value_norms_update(kv.ref(), b.ref(), C._ptr(idx), C._ptr(off), C._ptr(off_d),
+                                          None, None) == C.ERR_INVALID_ARG
+    # workspace: the normed pass has no value partials, so it needs less
+    full = C.conduit_score_workspace_size(kv, b)
+    normed = C.conduit_score_with_norms_workspace_size(kv, b)
+    assert 0 < normed < full
+    ws = torch.zeros(normed - 256, dtype=torch.uint8)
+    _expect(C, C.ERR_WORKSPACE, C.conduit_score_with_norms, kv, b, q, vn, None, None, None, None, ws)
+    assert lib.conduit_score_with_norms(kv.ref(), b.ref(), C._ptr(q), None, 0, None, C._ptr(vn),
+                                        C._ptr(vn), C._ptr(vn), None, 0, None, None) == C.ERR_INVALID_ARG
+
+
+def test_score_options_are_checked(C):
+    kv, b = _kv(C), _batch(C)
+    lib = C._lib
+    q = torch.zeros((2, 4, 8, 64), dtype=torch.bfloat16)
+    vn = torch.zeros((2, 128))
+    out = torch.zeros(128)
+
+    def call(opts, ws=None):
+        n = ctypes.c_size_t(0)
+        rc = lib.conduit_score_ex_workspace_size(kv.ref(), b.ref(), 0, ctypes.byref(opts), ctypes.byref(n))
+        if ws is None:
+            return rc
+        return lib.conduit_score_ex(kv.ref(), b.ref(), C._ptr(q), None, 0, ctypes.byref(opts), C._ptr(out),
+                                    C._ptr(out), C._ptr(out), C._ptr(ws), ws.numel(), None, None)
+
+    bad = C.score_opts()
+    bad.statistic = 7
+    assert call(bad) == C.ERR_INVALID_ARG and "statistic" in lib.conduit_last_error_string().decode()
+    bad = C.score_opts()
+    bad.value_norm = 3
+    assert call(bad) == C.ERR_INVALID_ARG
+    assert call(C.score_opts(value_norm="side_cache")) == C.ERR_INVALID_ARG      # no vnorm
+    assert call(C.score_opts(value_norm="v", vnorm=vn)) == C.ERR_INVALID_ARG     # vnorm not used
+    odd = C.score_opts()
+    odd.extra_lse = vn.data_ptr() + 2
+    assert call(odd) == C.ERR_INVALID_ARG
+    # workspace sizes: NULL options = conduit_score; RMS adds, dropping V's partials removes
+    n = ctypes.c_size_t(0)
+    assert lib.conduit_score_ex_workspace_size(kv.ref(), b.ref(), 0, None, ctypes.byref(n)) == C.OK
+    base = C.conduit_score_workspace_size(kv, b)
+    assert n.value == base
+    rms = C.conduit_score_ex_workspace_size(kv, b, 0, C.score_opts(statistic="rms"))
+    none = C.conduit_score_ex_workspace_size(kv, b, 0, C.score_opts(value_norm="none"))
+    side = C.conduit_score_ex_workspace_size(kv, b, 0, C.score_opts(value_norm="side_cache", vnorm=vn))
+    assert rms > base > none == side == C.conduit_score_with_norms_workspace_size(kv, b)
+    # a workspace sized for the mean is short for the RMS statistic
+    ws = torch.zeros(base, dtype=torch.uint8)
+    assert call(C.score_opts(statistic="rms"), ws) == C.ERR_WORKSPACE
 
 
 def test_kv_cache_python_checks(C):

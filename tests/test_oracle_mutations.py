@@ -25,7 +25,7 @@ def _logits_no_scale(q_h, k_g):
     return q_h @ k_g.T
 
 
-def _head_mean_wrong_gqa(q_l, k_l):
+def _head_mean_wrong_gqa(q_l, k_l, extra_lse_l=None):
     hq, n_q, _ = q_l.shape
     hkv = k_l.shape[0]
     total = np.zeros(k_l.shape[1])
@@ -34,13 +34,35 @@ def _head_mean_wrong_gqa(q_l, k_l):
     return total / (n_q * hq)
 
 
-def _head_mean_wrong_divisor(q_l, k_l):
+def _head_mean_wrong_divisor(q_l, k_l, extra_lse_l=None):
     hq, n_q, _ = q_l.shape
     hkv = k_l.shape[0]
     total = np.zeros(k_l.shape[1])
     for h in range(hq):
         total += O.softmax_over_visual_keys(O.cached_key_logits(q_l[h], k_l[h // (hq // hkv)])).sum(axis=0)
     return total / (n_q * hkv)
+
+
+def _outside_keys_dropped(x, extra_lse):
+    return O.softmax_over_visual_keys(x)
+
+
+def _outside_keys_twice(x, extra_lse):
+    c = np.maximum(x.max(axis=1), extra_lse)[:, None]
+    e = np.exp(x - c)
+    return e / (e.sum(axis=1, keepdims=True) + 2 * np.exp(extra_lse[:, None] - c))
+
+
+def _rms_without_root(q_l, k_l, extra_lse_l=None):
+    hq, n_q, _ = q_l.shape
+    alpha = O._attention_rows(q_l, k_l, extra_lse_l)
+    return (alpha * alpha).sum(axis=(0, 1)) / (n_q * hq)
+
+
+def _rms_over_queries_only(q_l, k_l, extra_lse_l=None):
+    hq, n_q, _ = q_l.shape
+    alpha = O._attention_rows(q_l, k_l, extra_lse_l)
+    return np.sqrt((alpha * alpha).sum(axis=(0, 1)) / n_q)
 
 
 def _value_norm_mean_of_heads(v_l):
@@ -118,6 +140,10 @@ MUTANTS = {
     "GQA head h -> h % Hkv": ("head_query_mean_attention", _head_mean_wrong_gqa),
     "divide by Hkv": ("head_query_mean_attention", _head_mean_wrong_divisor),
     "mean of per-head norms": ("value_norms", _value_norm_mean_of_heads),
+    "outside keys dropped": ("softmax_with_outside_keys", _outside_keys_dropped),
+    "outside keys counted twice": ("softmax_with_outside_keys", _outside_keys_twice),
+    "RMS without the root": ("head_query_rms_attention", _rms_without_root),
+    "RMS divides by |Q| only": ("head_query_rms_attention", _rms_over_queries_only),
     "layer sum instead of mean": ("throughput_score", _throughput_sum),
     "g without 1/|L|": ("image_mean_attention", _image_mean_no_layer_divisor),
     "lambda ignored": ("image_coefficients", _coefficients_ignore_lambda),

@@ -268,6 +268,94 @@ def test_scored_layer_subset():
     np.testing.assert_allclose(one["g"], alone["g"], rtol=1e-15)
 
 
+# ------------------------------------------------- value-norm side cache
+def test_stored_norms_give_the_same_scores():
+    """Sec. 4.3 / App. C.2: norms kept from cache construction leave the scores unchanged."""
+    q, k, v, spans = _rand_request(16, L=3)
+    stored = np.stack([np.linalg.norm(np.concatenate(list(v[l]), axis=1), axis=1) for l in range(3)])
+    for layers in (None, [0, 2]):
+        live = O.score_request(q, k, v, spans, layers=layers)
+        kept = O.score_request(q, k, None, spans, layers=layers, vnorm=stored)
+        for key in ("a", "vn", "s", "A", "g"):
+            np.testing.assert_allclose(kept[key], live[key], rtol=1e-14, atol=0)
+
+
+def test_stored_norms_are_read_per_scored_layer():
+    """Norms constant per layer (c_l) give s = sum_l c_l a^(l) / |L| over the scored layers."""
+    q, k, v, spans = _rand_request(17, L=4)
+    N = k.shape[2]
+    c = np.array([1.0, 10.0, 100.0, 1000.0])
+    vnorm = np.repeat(c[:, None], N, axis=1)
+    kept = O.score_request(q, k, None, spans, layers=[1, 3], vnorm=vnorm)
+    a = [O.head_query_mean_attention(q[l], k[l]) for l in (1, 3)]
+    np.testing.assert_allclose(kept["s"], (10.0 * a[0] + 1000.0 * a[1]) / 2, rtol=1e-13)
+    # unit norms: s is the layer-mean attention A / |L|
+    ones = O.score_request(q, k, None, spans, vnorm=np.ones((4, N)))
+    np.testing.assert_allclose(ones["s"], ones["A"] / 4, rtol=1e-14)
+
+
+# ------------------------------------------------ statistic variants
+def _softmax_rows(x):
+    """Library softmax of each row (scipy), for the pins below."""
+    sp = pytest.importorskip("scipy.special")
+    return sp.softmax(x, axis=-1)
+
+
+def test_rms_statistic_brute_force_and_special_cases():
+    """Eq. 4: abar_t = sqrt(mean over (q, h) of alpha^2), against scipy softmax;
+    one query row and one head give abar = alpha exactly; abar >= a (power means)."""
+    q, k, v, spans = _rand_request(18, L=2)
+    L, hq, n_q, d = q.shape
+    G = hq // k.shape[1]
+    got = O.score_request(q, k, v, spans, statistic="rms")
+    for l in range(L):
+        alpha = np.stack([_softmax_rows(q[l, h] @ k[l, h // G].T / math.sqrt(d)) for h in range(hq)])
+        want = np.sqrt((alpha ** 2).mean(axis=(0, 1)))
+        np.testing.assert_allclose(got["stat"][l], want, rtol=1e-12)
+    assert np.all(got["stat"] >= got["a"] * (1 - 1e-12))
+    np.testing.assert_allclose(got["A"], O.score_request(q, k, v, spans)["A"], rtol=1e-15)
+    one = O.score_request(q[:, :1, :1], k[:, :1], v, spans, statistic="rms")
+    np.testing.assert_allclose(one["stat"], one["a"], rtol=1e-13)
+
+
+def test_attention_alone_ablation():
+    """Dropping the value norm (Sec. 4.4 factor ablation): s = A / |L| exactly."""
+    q, k, v, spans = _rand_request(19, L=3)
+    got = O.score_request(q, k, None, spans, use_value_norm=False)
+    np.testing.assert_allclose(got["s"], got["A"] / 3, rtol=1e-14)
+
+
+def test_full_context_softmax_matches_softmax_over_all_keys():
+    """Outside keys entering through their log-sum-exp give the visual columns
+    of a library softmax over visual + outside keys; without outside keys the
+    visual-only softmax comes back."""
+    sp = pytest.importorskip("scipy.special")
+    rng = np.random.default_rng(20)
+    L, hq, hkv, n_q, N, n_text, d = 2, 4, 2, 3, 40, 25, 16
+    q = rng.standard_normal((L, hq, n_q, d))
+    k = rng.standard_normal((L, hkv, N, d)) * 1.5
+    k_text = rng.standard_normal((L, hkv, n_text, d)) * 1.5
+    v = rng.standard_normal((L, hkv, N, d))
+    spans = [0, 15, N]
+    G = hq // hkv
+    extra = np.zeros((L, hq, n_q))
+    want_a = np.zeros((L, N))
+    for l in range(L):
+        for h in range(hq):
+            xt = q[l, h] @ k_text[l, h // G].T / math.sqrt(d)
+            extra[l, h] = sp.logsumexp(xt, axis=1)
+            x_all = np.concatenate([q[l, h] @ k[l, h // G].T / math.sqrt(d), xt], axis=1)
+            want_a[l] += _softmax_rows(x_all)[:, :N].sum(axis=0)
+    want_a /= n_q * hq
+    got = O.score_request(q, k, v, spans, extra_lse=extra)
+    np.testing.assert_allclose(got["a"], want_a, rtol=1e-12)
+    assert np.all(got["a"].sum(axis=1) < 1.0)
+    none = O.score_request(q, k, v, spans, extra_lse=np.full((L, hq, n_q), -np.inf))
+    plain = O.score_request(q, k, v, spans)
+    for key in ("a", "s", "A", "g"):
+        np.testing.assert_allclose(none[key], plain[key], rtol=1e-14)
+
+
 # --------------------------------------------------------- refresh step
 def test_gather_scatter_roundtrip():
     rng = np.random.default_rng(15)
