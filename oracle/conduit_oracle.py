@@ -60,6 +60,9 @@ __all__ = [
     "image_coefficients",
     "composite_score",
     "topk_select",
+    "image_coefficients_f32",
+    "image_quotas",
+    "quota_select",
     "refresh_mask",
     "score_request",
     "kv_gather",
@@ -236,6 +239,93 @@ def topk_select(s_hat: np.ndarray, k: int) -> np.ndarray:
         raise ValueError("budget k must lie in [0, N]")
     order = sorted(range(n), key=lambda t: (-float(s_hat[t]), t))
     return np.array(sorted(order[:k]), dtype=np.int64)
+
+
+# --------------------------------------------------------------------------
+# App. D.3 ("explicit" cross-image variant): quotas k_j proportional to
+# c_j n_j, then a top-k_j inside each image.
+# --------------------------------------------------------------------------
+def image_coefficients_f32(g: np.ndarray, lam: float) -> np.ndarray:
+    """Eq. 9 evaluated in binary32, one rounding per operation, for decisions
+    that turn c_j into integers (the quotas below) in the kernel's precision:
+    g_bar = (((g_0 + g_1) + g_2) + ...) / K, c_j = (1 - lambda) + lambda * (g_j / g_bar),
+    c = 1 for K == 1 or g_bar == 0.
+    """
+    f = np.float32
+    g = np.asarray(g, dtype=np.float32)
+    k_img = g.shape[0]
+    lam32 = f(lam)
+    if k_img == 1:
+        return np.ones(1, dtype=np.float32)
+    total = f(0.0)
+    for j in range(k_img):
+        total = f(total + g[j])
+    g_bar = f(total / f(k_img))
+    if g_bar == 0:
+        return np.ones(k_img, dtype=np.float32)
+    one_minus = f(f(1.0) - lam32)
+    return np.array([f(one_minus + f(lam32 * f(g[j] / g_bar))) for j in range(k_img)],
+                    dtype=np.float32)
+
+
+def image_quotas(c: np.ndarray, n: Sequence[int], k: int) -> np.ndarray:
+    """k_j proportional to c_j n_j with sum_j k_j = k and 0 <= k_j <= n_j.
+
+    The paper states the proportionality only; the integer rule taken here is
+    the largest-remainder (Hamilton) rule in float64: w_j = c_j n_j,
+    W = w_0 + w_1 + ... (left to right), ideal_j = (kk w_j) / W over the
+    images still open; an image whose ideal exceeds n_j is closed at n_j and
+    the rest of the budget is shared again; otherwise k_j = floor(ideal_j)
+    and the leftover units go to the largest remainders ideal_j - floor,
+    ties to the lower image index. If every open image has weight 0, the
+    weights become n_j (size-proportional).
+    """
+    n = [int(x) for x in n]
+    k_img = len(n)
+    if not (0 <= k <= sum(n)):
+        raise ValueError("budget k must lie in [0, sum n_j]")
+    quota = [0] * k_img
+    open_ = [j for j in range(k_img)]
+    kk = int(k)
+    while True:
+        w = {j: float(np.float64(c[j]) * float(n[j])) for j in open_}
+        if all(w[j] == 0.0 for j in open_):
+            w = {j: float(n[j]) for j in open_}
+        total = 0.0
+        for j in open_:
+            total = total + w[j]
+        ideal = {j: (float(kk) * w[j]) / total if total > 0 else 0.0 for j in open_}
+        over = [j for j in open_ if ideal[j] > n[j]]
+        if over:
+            for j in over:
+                quota[j] = n[j]
+                kk -= n[j]
+            open_ = [j for j in open_ if j not in over]
+            continue
+        base = {j: int(math.floor(ideal[j])) for j in open_}
+        left = kk - sum(base.values())
+        order = sorted(open_, key=lambda j: (-(ideal[j] - base[j]), j))
+        for j in open_:
+            quota[j] = base[j]
+        for j in order[:left]:
+            quota[j] += 1
+        return np.array(quota, dtype=np.int64)
+
+
+def quota_select(s: np.ndarray, c: np.ndarray, img_off: Sequence[int], k: int) -> dict:
+    """The explicit variant for one request: quotas from image_quotas, then in
+    image j the k_j tokens of largest s_t (Eq. 7; c_j is constant inside an
+    image, so it decides only the quotas), ties to the lowest index.
+
+    Returns the quotas and the ascending request-local indices.
+    """
+    n = [int(img_off[j + 1]) - int(img_off[j]) for j in range(len(img_off) - 1)]
+    quota = image_quotas(c, n, k)
+    idx = []
+    for j in range(len(n)):
+        lo, hi = int(img_off[j]), int(img_off[j + 1])
+        idx.extend((lo + topk_select(np.asarray(s[lo:hi], dtype=np.float64), int(quota[j]))).tolist())
+    return {"quota": quota, "idx": np.array(sorted(idx), dtype=np.int64)}
 
 
 def score_request(q: np.ndarray, k: np.ndarray, v: Optional[np.ndarray],

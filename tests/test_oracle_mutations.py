@@ -65,6 +65,42 @@ def _rms_over_queries_only(q_l, k_l, extra_lse_l=None):
     return np.sqrt((alpha * alpha).sum(axis=(0, 1)) / n_q)
 
 
+def _quotas_floor_only(c, n, k):
+    w = np.asarray(c, dtype=np.float64) * np.asarray(n, dtype=np.float64)
+    return np.floor(k * w / w.sum()).astype(np.int64)
+
+
+def _quotas_ties_high(c, n, k):
+    w = np.asarray(c, dtype=np.float64) * np.asarray(n, dtype=np.float64)
+    ideal = k * w / w.sum()
+    base = np.floor(ideal).astype(np.int64)
+    order = sorted(range(len(n)), key=lambda j: (-(ideal[j] - base[j]), -j))
+    for j in order[:k - int(base.sum())]:
+        base[j] += 1
+    return np.minimum(base, np.asarray(n))
+
+
+def _quotas_ignore_sizes(c, n, k):
+    return _quotas_ties_high_free(np.asarray(c, dtype=np.float64), len(n), k)
+
+
+def _quotas_ties_high_free(w, K, k):
+    ideal = k * w / w.sum()
+    base = np.floor(ideal).astype(np.int64)
+    order = sorted(range(K), key=lambda j: (-(ideal[j] - base[j]), j))
+    for j in order[:k - int(base.sum())]:
+        base[j] += 1
+    return base
+
+
+def _coefficients_f32_mean_over_k_minus_1(g, lam):
+    g = np.asarray(g, dtype=np.float32)
+    if g.shape[0] == 1:
+        return np.ones(1, dtype=np.float32)
+    gbar = np.float32(g.sum() / np.float32(g.shape[0] - 1))
+    return (np.float32(1 - lam) + np.float32(lam) * (g / gbar)).astype(np.float32)
+
+
 def _value_norm_mean_of_heads(v_l):
     return np.sqrt((v_l * v_l).sum(axis=2)).mean(axis=0)
 
@@ -140,6 +176,10 @@ MUTANTS = {
     "GQA head h -> h % Hkv": ("head_query_mean_attention", _head_mean_wrong_gqa),
     "divide by Hkv": ("head_query_mean_attention", _head_mean_wrong_divisor),
     "mean of per-head norms": ("value_norms", _value_norm_mean_of_heads),
+    "quotas floored, leftover dropped": ("image_quotas", _quotas_floor_only),
+    "quota remainder ties to the higher index": ("image_quotas", _quotas_ties_high),
+    "quotas ignore image sizes": ("image_quotas", _quotas_ignore_sizes),
+    "f32 coefficients divide by K - 1": ("image_coefficients_f32", _coefficients_f32_mean_over_k_minus_1),
     "outside keys dropped": ("softmax_with_outside_keys", _outside_keys_dropped),
     "outside keys counted twice": ("softmax_with_outside_keys", _outside_keys_twice),
     "RMS without the root": ("head_query_rms_attention", _rms_without_root),

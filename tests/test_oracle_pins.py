@@ -356,6 +356,77 @@ def test_full_context_softmax_matches_softmax_over_all_keys():
         np.testing.assert_allclose(none[key], plain[key], rtol=1e-14)
 
 
+# ------------------------------------------- explicit per-image quotas
+def test_quotas_textbook_largest_remainder():
+    """Hamilton's rule on hand-checked cases: a remainder tie goes to the lower
+    index; sizes 6, 6, 2 give 4, 4, 2 seats of 10 and 5, 5, 1 of 11 (the
+    Alabama paradox, a known property of the largest-remainder rule)."""
+    assert O.image_quotas(np.ones(3), [55, 30, 15], 10).tolist() == [6, 3, 1]
+    assert O.image_quotas(np.ones(3), [6, 6, 2], 10).tolist() == [4, 4, 2]
+    assert O.image_quotas(np.ones(3), [6, 6, 2], 11).tolist() == [5, 5, 1]
+    # coefficients scale the sizes: c n = (20, 10, 10) of 8 -> 4, 2, 2
+    assert O.image_quotas(np.array([2.0, 1.0, 0.5]), [10, 10, 20], 8).tolist() == [4, 2, 2]
+
+
+def test_quotas_cap_and_degenerate_cases():
+    # image 0 would take 8.3 of 50 but holds 2 tokens: capped, the rest re-shared
+    assert O.image_quotas(np.array([10.0, 1.0]), [2, 100], 50).tolist() == [2, 48]
+    assert O.image_quotas(np.array([3.0]), [17], 9).tolist() == [9]            # K = 1: k_1 = k
+    assert O.image_quotas(np.zeros(3), [4, 8, 4], 8).tolist() == [2, 4, 2]     # all c = 0: sizes
+    assert O.image_quotas(np.array([0.0, 1.0]), [5, 5], 3).tolist() == [0, 3]
+    assert O.image_quotas(np.ones(2), [3, 4], 7).tolist() == [3, 4]            # k = sum n_j
+    assert O.image_quotas(np.ones(2), [3, 4], 0).tolist() == [0, 0]
+
+
+def test_quotas_minimise_deviation_brute_force():
+    """Without caps, the largest-remainder quotas minimise sum |k_j - ideal_j|
+    over every integer split of k (enumerated), and lie between floor and ceil."""
+    rng = np.random.default_rng(21)
+    for _ in range(200):
+        K = int(rng.integers(1, 5))
+        n = rng.integers(5, 12, size=K).tolist()
+        c = rng.uniform(0.2, 2.0, size=K)
+        k = int(rng.integers(0, min(n) + 1))  # small enough that no ideal exceeds n_j
+        w = c * np.array(n, dtype=np.float64)
+        ideal = k * w / w.sum()
+        if np.any(ideal > np.array(n)):
+            continue
+        got = O.image_quotas(c, n, k)
+        assert got.sum() == k and np.all(got >= np.floor(ideal)) and np.all(got <= np.ceil(ideal))
+        best = min(sum(abs(x - q) for x, q in zip(split, ideal))
+                   for split in itertools.product(*[range(k + 1)] * K) if sum(split) == k)
+        assert abs(np.abs(got - ideal).sum() - best) < 1e-9
+
+
+def test_coefficients_f32_follow_eq9():
+    rng = np.random.default_rng(22)
+    for lam in (0.0, 0.3, 1.0):
+        g = rng.uniform(0.0, 0.01, size=7).astype(np.float32)
+        c32 = O.image_coefficients_f32(g, lam)
+        assert c32.dtype == np.float32
+        np.testing.assert_allclose(c32, O.image_coefficients(g.astype(np.float64), lam), rtol=2e-6)
+    assert O.image_coefficients_f32(np.array([0.2], dtype=np.float32), 0.7).tolist() == [1.0]
+    assert O.image_coefficients_f32(np.zeros(3, dtype=np.float32), 1.0).tolist() == [1.0] * 3
+
+
+def test_quota_select_per_image_top():
+    rng = np.random.default_rng(23)
+    s = rng.uniform(size=40)
+    s[[3, 7]] = s[5]                       # a three-way tie inside image 0
+    spans = [0, 10, 25, 40]
+    c = np.array([1.0, 2.0, 0.5])
+    out = O.quota_select(s, c, spans, 12)
+    q = out["quota"]
+    assert q.tolist() == O.image_quotas(c, [10, 15, 15], 12).tolist() and q.sum() == 12
+    for j in range(3):
+        lo, hi = spans[j], spans[j + 1]
+        mine = [t - lo for t in out["idx"] if lo <= t < hi]
+        order = sorted(range(hi - lo), key=lambda t: (-s[lo + t], t))   # brute-force ranking
+        assert sorted(mine) == sorted(order[:q[j]])
+    one = O.quota_select(s, np.array([1.3]), [0, 40], 9)               # one image: the global top-k
+    assert one["idx"].tolist() == O.topk_select(s, 9).tolist()
+
+
 # --------------------------------------------------------- refresh step
 def test_gather_scatter_roundtrip():
     rng = np.random.default_rng(15)
