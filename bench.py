@@ -167,6 +167,8 @@ def work_model(pipe) -> dict:
     score_flops = sum(2 * L * Hq * (qo[r + 1] - qo[r]) * (tok[r + 1] - tok[r]) * d for r in range(R))
     k_sel = pipe.n_sel
     sel_bytes = 4 * n_tot + 4 * K + 4 * n_tot + n_tot + 4 * k_sel + 4 * K
+    if pipe.selection == "quota":  # coefficients, quotas and offsets through the workspace
+        sel_bytes += 2 * 12 * K
     copy_bytes = 2 * 2 * Lall * k_sel * Hkv * d * esz
     idx = pipe.idx[:k_sel].cpu().tolist()
     off = pipe.idx_off.tolist()
@@ -211,7 +213,8 @@ def call_kernels(pipe) -> dict:
     norms = (["vnorm_halves_kernel" if tc else "vnorm_rows_kernel"], "hbm", "vnorm.cu")
     if pipe.value_norm != "v" and not tc:  # no separate value pass
         score = (["rowstats_kernel", "colsum_kernel"] + tail, "alu", "score_simt.cu")
-    return {"score": score, "select": (["select_kernel"], "hbm", "select.cu"),
+    sel = ["quota_kernel", "select_kernel"] if pipe.selection == "quota" else ["select_kernel"]
+    return {"score": score, "select": (sel, "hbm", "select.cu"),
             "exchange": (["kv_copy_kernel"], "hbm", "kvcopy.cu"), "refresh": refresh,
             "norm_update": norms, "side_cache": norms}
 
@@ -238,14 +241,14 @@ def _traffic(call: str, workload: str, src: str):
 
 # -------------------------------------------------------------- our arm
 def build_pipeline(cfg: str, device, ratio=None, statistic="mean", value_norm="v",
-                   full_context=False):
+                   full_context=False, selection="global"):
     from paper_2609_05821_gb300 import pipeline, synth
     w = synth.workload(cfg)
     inputs = synth.make_inputs(w, device=device)
     _with_ratio(inputs, ratio)  # one refresh ratio for every request (e.g. the long-document budgets)
     extra = synth.make_extra_lse(inputs) if full_context else None
     return pipeline.from_inputs(inputs, statistic=statistic, value_norm=value_norm,
-                                extra_lse=extra), w
+                                extra_lse=extra, selection=selection), w
 
 
 def time_steps(fn, steps: int, flush=None):
@@ -275,7 +278,7 @@ def run_conduit(args):
     from paper_2609_05821_gb300 import conduit as C
 
     pipe, w = build_pipeline(args.config, dev, args.ratio, args.statistic, args.value_norm,
-                             args.full_context)
+                             args.full_context, args.selection)
     n_tok = pipe.batch.n_tot
     flush_buf = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
     flush = lambda: flush_buf.zero_()
@@ -366,7 +369,7 @@ def run_conduit(args):
         achieved, peak, unit = model[dom]["flops"] / sec / 1e12, ALU_FP32_TFLOPS, "TFLOP/s"
         peak_note = "fp32 FMA: 152 SMs x 128 lanes x 2 FLOP x 2.07 GHz"
     # committed ncu traffic covers the default scoring pass only
-    traffic = _traffic(dom, args.config, src) if pipe.plain else None
+    traffic = _traffic(dom, args.config, src) if pipe.plain and pipe.selection == "global" else None
     roofline = {"bound": bound, "achieved": round(achieved, 3), "peak": round(peak, 1), "unit": unit,
                 "frac": round(achieved / peak, 4), "traffic": traffic, "kernel": dom,
                 "kernels": kernels, "peak_source": peak_note,
@@ -405,7 +408,9 @@ def run_conduit(args):
                                                  "updated for the rewritten rows inside it",
                                    "none": "not used (attention alone)"}[args.value_norm],
                    "softmax": ("full context (seeded outside-key log-sum-exps)" if args.full_context
-                               else "visual keys")},
+                               else "visual keys"),
+                   "selection": {"global": "one global top-k (Eq. 11)",
+                                 "quota": "per-image quotas (App. D.3)"}[args.selection]},
         "score_select_tokens_per_s": round(n_tok / ((call_ms["score"] + call_ms["select"]) / 1e3), 1),
         "refresh_pass_us": round((call_ms["exchange"] + call_ms.get("norm_update", 0.0)
                                   + call_ms["refresh"]) * 1e3, 2),
@@ -419,7 +424,8 @@ def run_conduit(args):
         "status": status,
         "wall_s_timed": round(wall, 3),
     }
-    if rank == 0 and world == 1 and not args.no_cpu_baseline and pipe.plain:  # the oracle arm times the default pass
+    default = pipe.plain and pipe.selection == "global"
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and default:  # the oracle arm times the default pass
         out["cpu_baseline"] = cpu_baseline(args.config, args.cpu_seconds, args.ratio)
     if world > 1:
         import torch.distributed as dist
@@ -557,6 +563,8 @@ def main():
                     help="value norms from V (default), the side cache (Sec. 4.3), or none")
     ap.add_argument("--statistic", default="mean", choices=["mean", "rms"],
                     help="attention statistic in s: mean (Eq. 6, default) or RMS (Eq. 4)")
+    ap.add_argument("--selection", default="global", choices=["global", "quota"],
+                    help="one global top-k (default) or explicit per-image quotas (App. D.3)")
     ap.add_argument("--full-context", action="store_true",
                     help="softmax denominators include outside keys (seeded log-sum-exps)")
     ap.add_argument("--ratio", type=float, default=None,

@@ -240,7 +240,8 @@ conduit_status conduit_score_with_norms(const conduit_kv* kv, const conduit_batc
  * Image-level amplification and one global top-k per request (Sec. 3.4-3.5,
  * Eqs. 9-11; Algorithm 1 last loops).
  *   c_j    = (1 - lambda) + lambda g_j / g_bar, g_bar = mean of the request's g_j;
- *            exactly 1 when the request has one image (Sec. 3.5) or g_bar == 0
+ *            exactly 1 when the request has one image (Sec. 3.5) or g_bar == 0;
+ *            binary32, one rounding per operation, g_bar = (((g_0 + g_1) + ...) / K
  *   s_hat_t = s_t c_{pi(t)}                                          Eq. 10
  *   T_r    = TopK_t(s_hat, k_r), ties to the lowest index            Eq. 11
  *  s, g       device fp32 [N_tot], [K] (outputs of conduit_score)
@@ -259,6 +260,32 @@ conduit_status conduit_select_topk(const conduit_batch* batch, const float* s, c
                                    int32_t* idx, uint8_t* mask, float* s_hat, float* coeff,
                                    void* workspace, size_t workspace_bytes, int32_t* status,
                                    void* stream);
+
+/*
+ * Explicit per-image quotas instead of the global ranking (App. D.3: the
+ * "explicit" variant of the cross-image diagnostic, compared there with the
+ * deployed global rule). Per request, with c_j of conduit_select_topk:
+ *   k_j proportional to c_j n_j, sum_j k_j = k_r, 0 <= k_j <= n_j
+ * by the largest remainder: w_j = c_j n_j (float64), W summed left to right
+ * over the open images, ideal_j = (kk w_j) / W; an image whose ideal exceeds
+ * n_j is closed at n_j and the rest kk of the budget is shared again over
+ * the others; otherwise k_j = floor(ideal_j) plus one unit for the
+ * k_r - sum floor largest remainders, ties to the lower image index. If every
+ * open weight is 0 (lambda = 1 and g_j = 0), the weights become n_j.
+ * Then T_r = union over j of the k_j tokens of image j with the largest s_t
+ * (c_j is constant inside an image), ties to the lowest index.
+ * Arguments as for conduit_select_topk, plus
+ *  quota  device int32 [K] k_j, or NULL
+ * idx holds request r's indices ascending (image by image); s_hat = s c_pi(t)
+ * is written for reference. status: NONFINITE for a NaN / Inf or negative s,
+ * or a non-finite c_j (that request's budget is then shared by image size).
+ */
+conduit_status conduit_select_quota_workspace_size(const conduit_batch* batch, size_t* bytes);
+conduit_status conduit_select_quota(const conduit_batch* batch, const float* s, const float* g,
+                                    float lambda, const int32_t* idx_off,
+                                    const int32_t* idx_off_dev, int32_t* idx, uint8_t* mask,
+                                    float* s_hat, float* coeff, int32_t* quota, void* workspace,
+                                    size_t workspace_bytes, int32_t* status, void* stream);
 
 /*
  * conduit_select_topk without a caller workspace. The paper has no

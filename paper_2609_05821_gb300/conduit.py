@@ -87,6 +87,8 @@ def _load():
         "conduit_select_workspace_size": (st, [P, ctypes.POINTER(SZ)]),
         "conduit_select_topk": (st, [P, P, P, ctypes.c_float, P, P, P, P, P, P, P, SZ, P, P]),
         "conduit_select_topk_noalloc": (st, [P, P, P, ctypes.c_float, P, P, P, P, P, P, P, P]),
+        "conduit_select_quota_workspace_size": (st, [P, ctypes.POINTER(SZ)]),
+        "conduit_select_quota": (st, [P, P, P, ctypes.c_float, P, P, P, P, P, P, P, P, SZ, P, P]),
         "conduit_kv_gather": (st, [P, P, P, P, P, P, P, P]),
         "conduit_kv_scatter": (st, [P, P, P, P, P, P, P, P]),
         "conduit_kv_exchange": (st, [P, P, P, P, P, P, P, P, P, P]),
@@ -350,6 +352,28 @@ def conduit_select_topk(batch: Batch, s: torch.Tensor, g: torch.Tensor, lam: flo
                                     _ptr(coeff), _ptr(ws), ws.numel(), _ptr(status),
                                     _stream_ptr(stream)))
     return idx[:n_sel], mask, s_hat, coeff
+
+
+def conduit_select_quota_workspace_size(batch: Batch) -> int:
+    n = ctypes.c_size_t(0)
+    _check(_lib.conduit_select_quota_workspace_size(batch.ref(), ctypes.byref(n)))
+    return int(n.value)
+
+
+def conduit_select_quota(batch: Batch, s: torch.Tensor, g: torch.Tensor, lam: float,
+                         idx_off: torch.Tensor, idx_off_dev: torch.Tensor, idx=None, mask=None,
+                         s_hat=None, coeff=None, quota=None, workspace=None, status=None,
+                         stream=None):
+    """Explicit per-image quotas (App. D.3). Returns (idx, mask, s_hat, coeff, quota)."""
+    dev = s.device
+    n_sel = int(idx_off[-1])
+    idx = torch.empty(max(n_sel, 1), dtype=torch.int32, device=dev) if idx is None else idx
+    ws = _workspace(conduit_select_quota_workspace_size(batch), dev, workspace)
+    _check(_lib.conduit_select_quota(batch.ref(), _ptr(s), _ptr(g), float(lam), _ptr(idx_off),
+                                     _ptr(idx_off_dev), _ptr(idx), _ptr(mask), _ptr(s_hat),
+                                     _ptr(coeff), _ptr(quota), _ptr(ws), ws.numel(), _ptr(status),
+                                     _stream_ptr(stream)))
+    return idx[:n_sel], mask, s_hat, coeff, quota
 
 
 NOALLOC_MAX_TOKENS = 1 << 20

@@ -471,6 +471,44 @@ conduit_status conduit_select_topk_noalloc(const conduit_batch* batch, const flo
   return CONDUIT_OK;
 }
 
+conduit_status conduit_select_quota_workspace_size(const conduit_batch* batch, size_t* bytes) {
+  conduit_status st;
+  if (!bytes) return fail(CONDUIT_ERR_INVALID_ARG, "bytes is NULL");
+  if ((st = check_batch(batch))) return st;
+  *bytes = align_up(size_t(batch->tok_off[batch->num_requests]) * sizeof(uint32_t)) +
+           align_up(quota_scratch_bytes(batch->num_images));
+  return CONDUIT_OK;
+}
+
+conduit_status conduit_select_quota(const conduit_batch* batch, const float* s, const float* g,
+                                    float lambda, const int32_t* idx_off,
+                                    const int32_t* idx_off_dev, int32_t* idx, uint8_t* mask,
+                                    float* s_hat, float* coeff, int32_t* quota, void* workspace,
+                                    size_t workspace_bytes, int32_t* status, void* stream) {
+  conduit_status st;
+  if ((st = check_batch(batch))) return st;
+  if (!s || !g) return fail(CONDUIT_ERR_INVALID_ARG, "s and g are required");
+  if (!(lambda >= 0.f && lambda <= 1.f))
+    return fail(CONDUIT_ERR_INVALID_ARG, "lambda must lie in [0, 1]");
+  if ((st = check_selection(batch, idx_off, idx_off_dev, true, idx))) return st;
+  size_t need = 0;
+  conduit_select_quota_workspace_size(batch, &need);
+  if ((st = check_workspace(workspace, workspace_bytes, need))) return st;
+  int max_images = 0, max_image_tokens = 0;
+  for (int r = 0; r < batch->num_requests; ++r)
+    max_images = std::max(max_images, batch->req_img_off[r + 1] - batch->req_img_off[r]);
+  for (int j = 0; j < batch->num_images; ++j)
+    max_image_tokens = std::max(max_image_tokens, batch->img_off[j + 1] - batch->img_off[j]);
+  char* ws = static_cast<char*>(workspace);
+  const size_t keys_bytes = align_up(size_t(batch->tok_off[batch->num_requests]) * sizeof(uint32_t));
+  cudaError_t err = launch_select_quota(make_batch(batch), max_images, max_image_tokens, s, g, lambda,
+                                        idx_off_dev, idx, mask, s_hat, coeff, quota,
+                                        reinterpret_cast<uint32_t*>(ws), ws + keys_bytes, status,
+                                        static_cast<cudaStream_t>(stream));
+  if (err) return cuda_fail(err, "select_quota");
+  return CONDUIT_OK;
+}
+
 static conduit_status kv_copy(const conduit_kv* kv, const conduit_batch* batch,
                               const int32_t* idx, const int32_t* idx_off,
                               const int32_t* idx_off_dev, void* rows_k, void* rows_v,

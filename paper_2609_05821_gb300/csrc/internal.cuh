@@ -169,6 +169,14 @@ cudaError_t launch_select(const BatchDev& b, int max_tokens, const float* s, con
                           float lambda, const int32_t* idx_off_dev, int32_t* idx, uint8_t* mask,
                           float* s_hat, float* coeff, uint32_t* keys, int32_t* status,
                           cudaStream_t stream);
+// Explicit per-image quotas (App. D.3): quota_kernel per request, then one
+// selection CTA per image. scratch holds quota_scratch_bytes(K) bytes.
+size_t quota_scratch_bytes(int total_images);
+cudaError_t launch_select_quota(const BatchDev& b, int max_images, int max_image_tokens,
+                                const float* s, const float* g, float lambda,
+                                const int32_t* idx_off_dev, int32_t* idx, uint8_t* mask,
+                                float* s_hat, float* coeff, int32_t* quota, uint32_t* keys,
+                                void* scratch, int32_t* status, cudaStream_t stream);
 // Same selection with the keys in the library's static device array.
 int64_t select_noalloc_max_tokens();
 cudaError_t launch_select_noalloc(const BatchDev& b, int max_tokens, const float* s, const float* g,

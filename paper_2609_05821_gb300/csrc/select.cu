@@ -8,6 +8,12 @@
 //   key exactly; every key above it is taken, and keys equal to it are taken
 //   in ascending token order until k are chosen (ties to the lowest index).
 //   Selected indices are written in ascending order together with the mask.
+//
+// Explicit per-image quotas (App. D.3, the variant the paper compares with the
+// global rule): quota_kernel (one CTA per request) turns the same c_j into
+// quotas k_j proportional to c_j n_j (largest remainder, float64), and the
+// selection kernel runs one CTA per image with budget k_j over the keys s_t,
+// writing its indices after those of the request's earlier images.
 #include <mutex>
 
 #include "internal.cuh"
@@ -16,6 +22,20 @@ namespace conduit {
 namespace {
 
 constexpr int kSelThreads = 1024;
+constexpr int kQuotaThreads = 256;
+
+// Eq. 9 with one rounding per operation (no contraction), so that the
+// coefficient that decides integer quotas is reproducible:
+//   g_bar = (((g_0 + g_1) + g_2) + ...) / K,  c_j = (1 - lambda) + lambda (g_j / g_bar).
+__device__ __forceinline__ float image_mean_f32(const float* g, int K) {
+  float sum = 0.f;
+  for (int j = 0; j < K; ++j) sum = __fadd_rn(sum, g[j]);
+  return __fdiv_rn(sum, float(K));
+}
+__device__ __forceinline__ float image_coefficient(float gj, float gbar, float lambda, int K) {
+  if (K == 1 || gbar == 0.f) return 1.f;
+  return __fadd_rn(__fsub_rn(1.f, lambda), __fmul_rn(lambda, __fdiv_rn(gj, gbar)));
+}
 
 // Block-wide exclusive scan of one int per thread; returns the prefix and
 // stores the block total in *total.
@@ -45,13 +65,19 @@ __device__ __forceinline__ int block_exclusive_scan(int v, int* warp_s, int* tot
   return before;
 }
 
-template <int kRegKeys>  // keys a thread keeps in registers (0: keys in the workspace)
+// Segment selection. kQuota = false: one CTA per request, keys s_hat = s c_pi(t),
+// budget k_r (Eqs. 10-11). kQuota = true: one CTA per image j, keys s_t,
+// budget quota[j], output at the request's slice + qoff[j] (App. D.3).
+template <int kRegKeys, bool kQuota>  // keys a thread keeps in registers (0: keys in the workspace)
 __global__ void __launch_bounds__(kSelThreads) select_kernel(BatchDev b, const float* s,
                                                              const float* g, float lambda,
                                                              const int32_t* idx_off, int32_t* idx,
                                                              uint8_t* mask, float* s_hat,
                                                              float* coeff, uint32_t* keys,
-                                                             int32_t* status) {
+                                                             int32_t* status,
+                                                             const float* seg_coeff,
+                                                             const int32_t* seg_quota,
+                                                             const int32_t* seg_qoff) {
   __shared__ float c_s[kMaxImagesPerRequest];
   __shared__ int img_s[kMaxImagesPerRequest + 1];
   __shared__ unsigned hist[256];
@@ -60,29 +86,43 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(BatchDev b, const f
   __shared__ int remaining_s;
   __shared__ float gbar_s;
 
-  const int r = blockIdx.x;
-  const int t0 = b.tok_off[r], N = b.tok_off[r + 1] - t0;
-  const int j0 = b.req_img_off[r], K = b.req_img_off[r + 1] - j0;
-  const int k = idx_off[r + 1] - idx_off[r];
-  int32_t* out = idx + idx_off[r];
-
-  // c_j (Eq. 9): g_bar in a fixed order by one thread.
-  for (int j = threadIdx.x; j <= K; j += blockDim.x) img_s[j] = b.img_off[j0 + j] - t0;
-  if (threadIdx.x == 0) {
-    float sum = 0.f;
-    for (int j = 0; j < K; ++j) sum += g[j0 + j];
-    gbar_s = sum / float(K);
+  int t0, N, k, K, base_t;
+  int32_t* out;
+  float c_seg = 1.f;
+  if (kQuota) {  // segment = image blockIdx.x
+    const int j = blockIdx.x;
+    const int r = request_of(b.req_img_off, b.R, j);
+    t0 = b.img_off[j];
+    N = b.img_off[j + 1] - t0;
+    k = min(max(seg_quota[j], 0), N);  // quota_kernel keeps 0 <= k_j <= n_j
+    K = 1;
+    base_t = t0 - b.tok_off[r];  // request-local index of the image's first token
+    out = idx + idx_off[r] + seg_qoff[j];
+    c_seg = seg_coeff[j];
+  } else {       // segment = request blockIdx.x
+    const int r = blockIdx.x;
+    t0 = b.tok_off[r];
+    N = b.tok_off[r + 1] - t0;
+    const int j0 = b.req_img_off[r];
+    K = b.req_img_off[r + 1] - j0;
+    k = idx_off[r + 1] - idx_off[r];
+    base_t = 0;
+    out = idx + idx_off[r];
+    // c_j (Eq. 9): g_bar in a fixed order by one thread.
+    for (int j = threadIdx.x; j <= K; j += blockDim.x) img_s[j] = b.img_off[j0 + j] - t0;
+    if (threadIdx.x == 0) gbar_s = image_mean_f32(g + j0, K);
+    __syncthreads();
+    const float gbar = gbar_s;
+    for (int j = threadIdx.x; j < K; j += blockDim.x) {
+      const float c = image_coefficient(g[j0 + j], gbar, lambda, K);
+      c_s[j] = c;
+      if (coeff) coeff[j0 + j] = c;
+    }
+    __syncthreads();
   }
-  __syncthreads();
-  const float gbar = gbar_s;
-  for (int j = threadIdx.x; j < K; j += blockDim.x) {
-    const float c = (K == 1 || gbar == 0.f) ? 1.f : (1.f - lambda) + lambda * (g[j0 + j] / gbar);
-    c_s[j] = c;
-    if (coeff) coeff[j0 + j] = c;
-  }
-  __syncthreads();
 
-  // s_hat (Eq. 10) and its sortable key. Each thread owns the contiguous
+  // s_hat (Eq. 10) and its sortable key (s itself in quota mode, where c_j is
+  // constant over the segment and decides only the quota). Each thread owns the contiguous
   // tokens [lo, hi); up to kRegKeys of them stay in registers for the radix
   // passes (requests of up to 1024 x kRegKeys tokens), otherwise the keys go
   // through the workspace.
@@ -93,7 +133,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(BatchDev b, const f
   bool bad = false;
   {
     int img = 0;  // image of token lo
-    {
+    if (!kQuota) {
       int a0 = 0, a1 = K - 1;
       while (a0 < a1) {
         const int mid = (a0 + a1 + 1) >> 1;
@@ -102,12 +142,20 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(BatchDev b, const f
       img = a0;
     }
     auto key_of = [&](int t) -> uint32_t {
-      while (img + 1 < K && img_s[img + 1] <= t) ++img;
-      float sh = s[t0 + t] * c_s[img];
-      if (!isfinite(sh) || sh < 0.f) bad = true;
-      if (sh == 0.f) sh = 0.f;  // -0 -> +0
-      if (s_hat) s_hat[t0 + t] = sh;
-      return __float_as_uint(sh);
+      float key;
+      if (kQuota) {
+        key = s[t0 + t];
+        const float sh = key * c_seg;
+        if (!isfinite(sh) || sh < 0.f || !isfinite(key) || key < 0.f) bad = true;
+        if (s_hat) s_hat[t0 + t] = sh == 0.f ? 0.f : sh;
+      } else {
+        while (img + 1 < K && img_s[img + 1] <= t) ++img;
+        key = s[t0 + t] * c_s[img];
+        if (!isfinite(key) || key < 0.f) bad = true;
+        if (s_hat) s_hat[t0 + t] = key == 0.f ? 0.f : key;
+      }
+      if (key == 0.f) key = 0.f;  // -0 -> +0
+      return __float_as_uint(key);
     };
     if (in_regs) {
 #pragma unroll
@@ -206,7 +254,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(BatchDev b, const f
       sel = seen_eq < take_eq;
       ++seen_eq;
     }
-    if (sel) out[pos++] = t;
+    if (sel) out[pos++] = base_t + t;
     if (mask) mask[t0 + t] = sel ? 1 : 0;
   };
   if (in_regs) {
@@ -215,6 +263,126 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(BatchDev b, const f
       if (lo + j < hi) emit(lo + j, kr[j]);
   } else {
     for (int t = lo; t < hi; ++t) emit(t, keys[t0 + t]);
+  }
+}
+
+// Quotas of one request (App. D.3): c_j as the global rule computes it, then
+// k_j proportional to c_j n_j with sum k_j = k_r and k_j <= n_j, by the largest
+// remainder in float64 (w_j = c_j n_j, W summed left to right over the open
+// images, ideal_j = (kk w_j) / W; images whose ideal exceeds n_j close at n_j
+// and the rest is shared again; leftover units go to the largest remainders,
+// ties to the lower index; all-zero weights fall back to n_j). Also the offset
+// of each image's indices within the request's slice.
+// Dynamic shared memory: K_max doubles (remainders), ints (quotas), bytes (open).
+__global__ void __launch_bounds__(kQuotaThreads) quota_kernel(BatchDev b, const float* g, float lambda,
+                                                              const int32_t* idx_off, float* c_out,
+                                                              int32_t* quota_out, int32_t* qoff_out,
+                                                              float* coeff, int32_t* quota_user,
+                                                              int32_t* status) {
+  extern __shared__ __align__(8) unsigned char qsm[];
+  __shared__ float gbar_s;
+  __shared__ double total_s;
+  __shared__ int kk_s, any_s, zero_s, left_s;
+  const int r = blockIdx.x;
+  const int j0 = b.req_img_off[r], K = b.req_img_off[r + 1] - j0;
+  double* rem_s = reinterpret_cast<double*>(qsm);
+  int* quota_s = reinterpret_cast<int*>(rem_s + K);
+  unsigned char* open_s = reinterpret_cast<unsigned char*>(quota_s + K);
+  if (threadIdx.x == 0) {
+    gbar_s = image_mean_f32(g + j0, K);
+    kk_s = idx_off[r + 1] - idx_off[r];
+  }
+  __syncthreads();
+  for (int j = threadIdx.x; j < K; j += blockDim.x) {
+    const float c = image_coefficient(g[j0 + j], gbar_s, lambda, K);
+    c_out[j0 + j] = c;
+    if (coeff) coeff[j0 + j] = c;
+    quota_s[j] = 0;
+    open_s[j] = 1;
+  }
+  __syncthreads();
+  auto n_of = [&](int j) { return b.img_off[j0 + j + 1] - b.img_off[j0 + j]; };
+  for (int round = 0; round <= K; ++round) {  // each round closes at least one image or ends
+    if (threadIdx.x == 0) {  // W in index order; size weights if every open weight is zero
+      int zero = 1;
+      for (int j = 0; j < K; ++j)
+        if (open_s[j] && double(c_out[j0 + j]) * double(n_of(j)) != 0.0) zero = 0;
+      for (int j = 0; j < K; ++j)  // a non-finite c_j (from g): flag it, share by size
+        if (open_s[j] && !isfinite(c_out[j0 + j])) {
+          zero = 1;
+          flag_status(status, CONDUIT_FLAG_NONFINITE);
+        }
+      double total = 0.0;
+      for (int j = 0; j < K; ++j)
+        if (open_s[j]) total = total + (zero ? double(n_of(j)) : double(c_out[j0 + j]) * double(n_of(j)));
+      zero_s = zero;
+      total_s = total;
+      any_s = 0;
+    }
+    __syncthreads();
+    const double total = total_s, kk = double(kk_s);
+    for (int j = threadIdx.x; j < K; j += blockDim.x) {
+      if (!open_s[j]) continue;
+      const double w = zero_s ? double(n_of(j)) : double(c_out[j0 + j]) * double(n_of(j));
+      const double ideal = total > 0.0 ? (kk * w) / total : 0.0;
+      rem_s[j] = ideal;
+      if (ideal > double(n_of(j))) any_s = 1;
+    }
+    __syncthreads();
+    if (any_s) {  // close the images over their size
+      if (threadIdx.x == 0) {
+        int kk2 = kk_s;
+        for (int j = 0; j < K; ++j)
+          if (open_s[j] && rem_s[j] > double(n_of(j))) {
+            quota_s[j] = n_of(j);
+            kk2 -= n_of(j);
+            open_s[j] = 0;
+          }
+        kk_s = kk2;
+      }
+      __syncthreads();
+      continue;
+    }
+    // floors, then the leftover units by remainder rank
+    for (int j = threadIdx.x; j < K; j += blockDim.x) {
+      if (!open_s[j]) continue;
+      const double fl = floor(rem_s[j]);
+      quota_s[j] = int(fl);
+      rem_s[j] = rem_s[j] - fl;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      int used = 0;
+      for (int j = 0; j < K; ++j)
+        if (open_s[j]) used += quota_s[j];
+      left_s = kk_s - used;
+    }
+    __syncthreads();
+    const int left = left_s;
+    int add[(kMaxImagesPerRequest + kQuotaThreads - 1) / kQuotaThreads];
+    int na = 0;
+    for (int j = threadIdx.x; j < K; j += blockDim.x, ++na) {
+      add[na] = 0;
+      if (!open_s[j]) continue;
+      int rank = 0;
+      for (int i = 0; i < K; ++i)
+        if (open_s[i] && (rem_s[i] > rem_s[j] || (rem_s[i] == rem_s[j] && i < j))) ++rank;
+      add[na] = rank < left ? 1 : 0;
+    }
+    __syncthreads();
+    na = 0;
+    for (int j = threadIdx.x; j < K; j += blockDim.x, ++na) quota_s[j] += add[na];
+    break;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int off = 0;
+    for (int j = 0; j < K; ++j) {
+      quota_out[j0 + j] = quota_s[j];
+      qoff_out[j0 + j] = off;
+      if (quota_user) quota_user[j0 + j] = quota_s[j];
+      off += quota_s[j];
+    }
   }
 }
 
@@ -265,15 +433,48 @@ cudaError_t launch_select(const BatchDev& b, int max_tokens, const float* s, con
                           cudaStream_t stream) {
   // the smallest register budget that holds every request's keys
   if (max_tokens <= kSelThreads)
-    select_kernel<1><<<b.R, kSelThreads, 0, stream>>>(b, s, g, lambda, idx_off_dev, idx, mask, s_hat,
-                                                      coeff, keys, status);
+    select_kernel<1, false><<<b.R, kSelThreads, 0, stream>>>(
+        b, s, g, lambda, idx_off_dev, idx, mask, s_hat, coeff, keys, status, nullptr, nullptr, nullptr);
   else if (max_tokens <= 8 * kSelThreads)
-    select_kernel<8><<<b.R, kSelThreads, 0, stream>>>(b, s, g, lambda, idx_off_dev, idx, mask, s_hat,
-                                                      coeff, keys, status);
+    select_kernel<8, false><<<b.R, kSelThreads, 0, stream>>>(
+        b, s, g, lambda, idx_off_dev, idx, mask, s_hat, coeff, keys, status, nullptr, nullptr, nullptr);
   else
-    select_kernel<0><<<b.R, kSelThreads, 0, stream>>>(b, s, g, lambda, idx_off_dev, idx, mask, s_hat,
-                                                      coeff, keys, status);
+    select_kernel<0, false><<<b.R, kSelThreads, 0, stream>>>(
+        b, s, g, lambda, idx_off_dev, idx, mask, s_hat, coeff, keys, status, nullptr, nullptr, nullptr);
   count_launches(1);
+  return cudaGetLastError();
+}
+
+size_t quota_scratch_bytes(int total_images) {
+  return size_t(total_images) * (sizeof(float) + 2 * sizeof(int32_t));
+}
+
+cudaError_t launch_select_quota(const BatchDev& b, int max_images, int max_image_tokens,
+                                const float* s, const float* g, float lambda,
+                                const int32_t* idx_off_dev, int32_t* idx, uint8_t* mask,
+                                float* s_hat, float* coeff, int32_t* quota, uint32_t* keys,
+                                void* scratch, int32_t* status, cudaStream_t stream) {
+  float* c_seg = static_cast<float*>(scratch);
+  int32_t* q_seg = reinterpret_cast<int32_t*>(c_seg + b.K);
+  int32_t* qoff = q_seg + b.K;
+  const size_t smem = size_t(max_images) * (sizeof(double) + sizeof(int) + 1);
+  cudaError_t err;
+  if (smem > 48 * 1024 &&
+      (err = cudaFuncSetAttribute(quota_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem))))
+    return err;
+  quota_kernel<<<b.R, kQuotaThreads, smem, stream>>>(b, g, lambda, idx_off_dev, c_seg, q_seg, qoff,
+                                                     coeff, quota, status);
+  if ((err = cudaGetLastError())) return err;
+  if (max_image_tokens <= kSelThreads)
+    select_kernel<1, true><<<b.K, kSelThreads, 0, stream>>>(
+        b, s, g, lambda, idx_off_dev, idx, mask, s_hat, coeff, keys, status, c_seg, q_seg, qoff);
+  else if (max_image_tokens <= 8 * kSelThreads)
+    select_kernel<8, true><<<b.K, kSelThreads, 0, stream>>>(
+        b, s, g, lambda, idx_off_dev, idx, mask, s_hat, coeff, keys, status, c_seg, q_seg, qoff);
+  else
+    select_kernel<0, true><<<b.K, kSelThreads, 0, stream>>>(
+        b, s, g, lambda, idx_off_dev, idx, mask, s_hat, coeff, keys, status, c_seg, q_seg, qoff);
+  count_launches(2);
   return cudaGetLastError();
 }
 

@@ -6,7 +6,8 @@
   3. conduit_kv_exchange  stale K/V rows of the selected tokens out, fresh rows in
                           (conduit_kv_gather + conduit_kv_scatter in one launch)
   4. conduit_refresh_attn causal attention of the refreshed rows over the patched cache
-Scoring variants (conduit_score_ex): ``statistic="rms"`` (Eq. 4),
+``selection="quota"`` replaces step 2 by conduit_select_quota (explicit
+per-image quotas, App. D.3). Scoring variants (conduit_score_ex): ``statistic="rms"`` (Eq. 4),
 ``value_norm="none"`` (attention alone) and ``extra_lse`` (full-context
 softmax). With ``value_norm="side_cache"`` the pipeline keeps the value-norm
 side cache (Sec. 4.3, App. C.2): it is built once at construction
@@ -34,7 +35,8 @@ class RefreshPipeline:
                  fresh: dict, lam: float = 1.0, layers: Optional[Sequence[int]] = None,
                  page_size: int = 0, page_table: Optional[torch.Tensor] = None,
                  budgets: Optional[Sequence[int]] = None, statistic: str = "mean",
-                 value_norm: str = "v", extra_lse: Optional[torch.Tensor] = None):
+                 value_norm: str = "v", extra_lse: Optional[torch.Tensor] = None,
+                 selection: str = "global"):
         dev = k.device
         self.device = dev
         self.kv = C.KvCache(k, v, num_q_heads, page_size, page_table)
@@ -66,8 +68,13 @@ class RefreshPipeline:
         opts = C.score_opts(statistic, value_norm, self.vnorm, extra_lse)
         self.ws_score = torch.empty(max(C.conduit_score_ex_workspace_size(self.kv, self.batch, nl, opts), 1),
                                     dtype=torch.uint8, device=dev)
-        self.ws_sel = torch.empty(max(C.conduit_select_workspace_size(self.batch), 1),
-                                  dtype=torch.uint8, device=dev)
+        if selection not in ("global", "quota"):
+            raise ValueError("selection must be 'global' or 'quota'")
+        self.selection = selection
+        self.quota = torch.empty(K, dtype=torch.int32, device=dev) if selection == "quota" else None
+        sel_ws = (C.conduit_select_quota_workspace_size if selection == "quota"
+                  else C.conduit_select_workspace_size)(self.batch)
+        self.ws_sel = torch.empty(max(sel_ws, 1), dtype=torch.uint8, device=dev)
         need = C.conduit_refresh_workspace_size(self.kv, self.batch, self.idx_off)
         self.ws_ref = torch.empty(need, dtype=torch.uint8, device=dev) if need else None
         L, Hkv, Hq, d = self.kv.num_layers, self.kv.num_kv_heads, num_q_heads, self.kv.head_dim
@@ -91,9 +98,14 @@ class RefreshPipeline:
                                self.g, self.ws_score, self.status, stream)
 
     def select(self, stream=None):
-        C.conduit_select_topk(self.batch, self.s, self.g, self.lam, self.idx_off, self.idx_off_dev,
-                              self.idx, self.mask, self.s_hat, self.coeff, self.ws_sel,
-                              self.status, stream)
+        if self.selection == "quota":
+            C.conduit_select_quota(self.batch, self.s, self.g, self.lam, self.idx_off, self.idx_off_dev,
+                                   self.idx, self.mask, self.s_hat, self.coeff, self.quota, self.ws_sel,
+                                   self.status, stream)
+        else:
+            C.conduit_select_topk(self.batch, self.s, self.g, self.lam, self.idx_off, self.idx_off_dev,
+                                  self.idx, self.mask, self.s_hat, self.coeff, self.ws_sel,
+                                  self.status, stream)
 
     def exchange(self, stream=None):
         C.conduit_kv_exchange(self.kv, self.batch, self.idx, self.idx_off, self.idx_off_dev,

@@ -36,7 +36,8 @@ def test_header_declares_the_boundary():
                  "conduit_kv_gather", "conduit_budget", "conduit_score_workspace_size",
                  "conduit_read_status", "conduit_value_norms", "conduit_value_norms_update",
                  "conduit_score_with_norms", "conduit_score_with_norms_workspace_size",
-                 "conduit_score_ex", "conduit_score_ex_workspace_size"):
+                 "conduit_score_ex", "conduit_score_ex_workspace_size",
+                 "conduit_select_quota", "conduit_select_quota_workspace_size"):
         assert want in names
 
 
@@ -129,6 +130,25 @@ def test_select_rejects_bad_budgets_and_lambda(C):
     ws = torch.zeros(8, dtype=torch.uint8)
     _expect(C, C.ERR_WORKSPACE, C.conduit_select_topk, b, s, g, 1.0, off, off_d, None, None, None,
             None, ws)
+
+
+def test_quota_select_rejects_bad_arguments(C):
+    b = _batch(C)
+    s = torch.zeros(128)
+    g = torch.zeros(3)
+    off, off_d = C.idx_offsets([10, 65], "cpu")
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_select_quota, b, s, g, 1.0, off, off_d, match="budget")
+    off, off_d = C.idx_offsets([10, 5], "cpu")
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_select_quota, b, s, g, -0.5, off, off_d, match="lambda")
+    idx = torch.zeros(15, dtype=torch.int32)
+    assert C._lib.conduit_select_quota(b.ref(), None, C._ptr(g), 1.0, C._ptr(off), C._ptr(off_d),
+                                       C._ptr(idx), None, None, None, None, None, 0, None,
+                                       None) == C.ERR_INVALID_ARG
+    need = C.conduit_select_quota_workspace_size(b)
+    assert need > C.conduit_select_workspace_size(b)        # plus coefficients, quotas, offsets
+    ws = torch.zeros(need - 256, dtype=torch.uint8)
+    _expect(C, C.ERR_WORKSPACE, C.conduit_select_quota, b, s, g, 1.0, off, off_d, None, None, None,
+            None, None, ws)
 
 
 def test_kv_copy_and_refresh_reject_bad_arguments(C):
