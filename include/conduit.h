@@ -361,6 +361,10 @@ conduit_status conduit_kv_exchange(const conduit_kv* kv, const conduit_batch* ba
  * Softmax and accumulation in fp32; out is written in the cache dtype.
  *  q_rows, out  device [L][idx_off[R]][Hq][d], dtype of kv
  *  idx must be ascending within each request (conduit_select_topk's order).
+ *  workspace    device, 256-byte aligned, conduit_refresh_workspace_size
+ *               bytes (256 for bf16 caches with head_dim 128: the work
+ *               counter of the persistent kernel; 0 otherwise); calls that
+ *               overlap on the GPU need workspaces of their own.
  */
 conduit_status conduit_refresh_workspace_size(const conduit_kv* kv, const conduit_batch* batch,
                                               const int32_t* idx_off, size_t* bytes);

@@ -562,7 +562,8 @@ conduit_status conduit_refresh_workspace_size(const conduit_kv* kv, const condui
   if (!bytes) return fail(CONDUIT_ERR_INVALID_ARG, "bytes is NULL");
   if ((st = check_batch(batch)) || (st = check_kv(kv, batch))) return st;
   (void)idx_off;
-  *bytes = 0;
+  // the tensor-core kernel takes its work items from a counter in the workspace
+  *bytes = refresh_tc_supported(make_kv(kv, batch)) ? kAlign : 0;
   return CONDUIT_OK;
 }
 
@@ -577,16 +578,15 @@ conduit_status conduit_refresh_attn(const conduit_kv* kv, const conduit_batch* b
   const int n_sel = idx_off[batch->num_requests];
   if (n_sel == 0) return CONDUIT_OK;
   if (!q_rows || !out) return fail(CONDUIT_ERR_INVALID_ARG, "q_rows and out are required");
-  (void)workspace;
-  (void)workspace_bytes;
-  (void)status;
   const KvDev kd = make_kv(kv, batch);
+  const bool tc = refresh_tc_supported(kd);
+  if ((st = check_workspace(workspace, workspace_bytes, tc ? kAlign : 0))) return st;
   cudaError_t err =
-      refresh_tc_supported(kd)
-          ? launch_refresh_tc(kd, make_batch(batch), idx, idx_off_dev, idx_off, n_sel, q_rows, out,
-                              status, static_cast<cudaStream_t>(stream))
-          : launch_refresh_simt(kd, make_batch(batch), idx, idx_off_dev, n_sel, q_rows, out,
-                                static_cast<cudaStream_t>(stream));
+      tc ? launch_refresh_tc(kd, make_batch(batch), idx, idx_off_dev, idx_off, n_sel, q_rows, out,
+                             static_cast<int32_t*>(workspace), status,
+                             static_cast<cudaStream_t>(stream))
+         : launch_refresh_simt(kd, make_batch(batch), idx, idx_off_dev, n_sel, q_rows, out,
+                               static_cast<cudaStream_t>(stream));
   if (err) return cuda_fail(err, "refresh_attn");
   return CONDUIT_OK;
 }

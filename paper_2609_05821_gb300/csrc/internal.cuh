@@ -193,7 +193,8 @@ cudaError_t launch_kv_copy(const KvDev& kv, const BatchDev& b, const int32_t* id
 bool refresh_tc_supported(const KvDev& kv);
 cudaError_t launch_refresh_tc(const KvDev& kv, const BatchDev& b, const int32_t* idx,
                               const int32_t* idx_off_dev, const int32_t* idx_off_host, int32_t n_sel,
-                              const void* q_rows, void* out, int32_t* status, cudaStream_t stream);
+                              const void* q_rows, void* out, int32_t* work_counter, int32_t* status,
+                              cudaStream_t stream);
 cudaError_t launch_refresh_simt(const KvDev& kv, const BatchDev& b, const int32_t* idx,
                                 const int32_t* idx_off_dev, int32_t n_sel, const void* q_rows,
                                 void* out, cudaStream_t stream);

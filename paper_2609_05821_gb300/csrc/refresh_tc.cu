@@ -2,15 +2,19 @@
 // (selective recompute, Conduit Sec. 3.1 / 4.3):
 //   out[l][i][h] = sum_{j <= p_i} softmax_j(<q[l][i][h], K'[l][h/G][j]> / sqrt(d)) V'[l][h/G][j]
 //
-// One CTA owns one query tile of 128 rows of one (layer, KV head, request):
+// Work item: one query tile of 128 rows of one (layer, KV head, request),
 // floor(128/G) consecutive selected rows times the G query heads that share
 // the KV head. Keys stream in tiles of 128 (a tcgen05.mma costs about the same
 // issue time for N = 64 and N = 128, so wide tiles halve the instruction
-// count). Roles (320 threads):
-//   warp 0     TMA loads: the query tile (a 3-D box of 64 dims x G heads x
-//              floor(128/G) rows lands in the tile's row order), then K tiles
-//              (three-stage ring) and V tiles (two stages); the lanes issue
-//              the copies of a tile together (one per page half when paged)
+// count). The kernel is persistent: one CTA per SM takes items from an atomic
+// counter (largest positions first within each (layer, KV head), so the CTAs
+// in flight share K/V in L2), and the query tile of the next item loads into
+// a second buffer while the current item computes. Roles (320 threads):
+//   warp 0     TMA loads: the query tile of each item (a 3-D box of 64 dims x
+//              G heads x floor(128/G) rows lands in the tile's row order) into
+//              one of two buffers, then its K and V tiles (two stages each);
+//              the lanes issue the copies of a tile together (one per page
+//              half when paged)
 //   warp 1     one thread issues tcgen05 MMAs: S(t) = Q K(t)^T into one of two
 //              TMEM buffers, O += P(t) V(t) with P read from TMEM
 //   warps 2-9  softmax, two warps per TMEM lane quarter: each thread owns one
@@ -20,14 +24,18 @@
 //              a lazy running max (O and the row sum are rescaled only when
 //              the max grows by 2^8; warp-uniform, since tcgen05.ld/st are
 //              warp-collective), writes its half of P as bf16 pairs over the
-//              upper half of S(t), and finally writes its half of O / rowsum
+//              upper half of S(t), and at the item's end writes its half of
+//              O / rowsum
 // TMEM: S buffers at columns [0, 128) and [128, 256) (P in the upper 64 of
 // each), O at [256, 384). S(t+1) is computed while the softmax works on
 // S(t); S(t+2) reuses the buffer of P(t), so it is issued once P(t) V(t) has
-// completed. Rows are sorted by position, so the tile needs keys up to its
-// last row's position only. Every wait is bounded by one second; a role that
-// gives up raises an abort flag the others watch, the kernel sets
-// CONDUIT_FLAG_TIMEOUT, drains its copies and MMAs, and frees TMEM.
+// completed; the next item's first S tiles are computed while the softmax
+// writes the previous item's O. Rows are sorted by position, so an item needs
+// keys up to its last row's position only. Every barrier phase follows from
+// per-CTA sequence numbers (items n, key tiles T) that all roles advance
+// alike. Every wait is bounded by one second; a role that gives up raises an
+// abort flag the others watch, the kernel sets CONDUIT_FLAG_TIMEOUT, drains
+// its copies and MMAs, and frees TMEM.
 #include <cuda.h>
 
 #include "internal.cuh"
@@ -41,13 +49,16 @@ constexpr int kKT = 128;                         // keys per tile
 constexpr int kRows = 128;                       // rows per query tile
 constexpr int kSoftThreads = 256;
 constexpr int kThreads = 64 + kSoftThreads;
-constexpr int kKStages = 3;
+constexpr int kKStages = 2;
 constexpr int kVStages = 2;
+constexpr int kQBufs = 2;
 constexpr uint32_t kQHalf = kRows * 128;         // 16 KB: one 64-dim half of the query tile
 constexpr uint32_t kQBytes = 2 * kQHalf;         // 32 KB
 constexpr uint32_t kTileHalf = kKT * 128;        // 16 KB: one 64-dim half of a K or V tile
 constexpr uint32_t kTileBytes = 2 * kTileHalf;   // 32 KB
-constexpr uint32_t kSmem = 1024 + kQBytes + (kKStages + kVStages) * kTileBytes + 256 + 2 * 2 * 128 * 4 + 2 * 128 * 4;
+constexpr int kRecInts = 8;                      // decoded item record (see Smem::rec)
+constexpr uint32_t kSmem = 1024 + kQBufs * kQBytes + (kKStages + kVStages) * kTileBytes + 256 +
+                           2 * 2 * 128 * 4 + 2 * 128 * 4 + kQBufs * (kRecInts + kRows) * 4;
 constexpr uint32_t kTmemCols = 512;              // 384 used; allocations are powers of two
 constexpr uint32_t kSCols = 128;                 // one S buffer
 constexpr uint32_t kPCol = 64;                   // P (bf16 pairs) over the upper half of S
@@ -63,32 +74,87 @@ struct RefArgs {
   __nv_bfloat16* out;
   int32_t n_sel;
   int32_t rows_per_tile;   // selected rows per query tile, floor(128 / G)
-  int32_t n_blocks;        // CTAs per (layer, KV head)
+  int32_t n_blocks;        // query tiles per (layer, KV head)
+  int32_t n_items;         // n_blocks * Hkv * L
+  int32_t blocks_major;    // item order: query tile (largest first) outer, or (layer, head) outer
+  int32_t* next_item;      // work counter, zero at launch
   float scale_log2;
   int32_t* status;
 };
 
+// A work item: query tile `blk` of (layer l, KV head g), counted from the
+// largest positions, and the request, first selected row and row count.
+// Every layer and head of a request has the same selected positions, so the
+// blocks-major order (all (layer, head) pairs of the largest tile first) is
+// longest-first scheduling; the (layer, head)-major order keeps the CTAs in
+// flight on few K/V prefixes, which L2 then shares when the cache exceeds it.
+struct Item {
+  int l, g, r, i0, cnt;
+};
+
+__device__ __forceinline__ Item decode_item(const RefArgs& a, int u) {
+  Item it;
+  const int n_lg = a.kv.Hkv * a.kv.L;
+  const int x = a.blocks_major ? u / n_lg : u % a.n_blocks;
+  const int lg = a.blocks_major ? u % n_lg : u / a.n_blocks;
+  it.g = lg % a.kv.Hkv;
+  it.l = lg / a.kv.Hkv;
+  int blk = a.n_blocks - 1 - x;
+  it.r = 0;
+  it.i0 = -1;
+  it.cnt = 0;
+  const int span = a.rows_per_tile;
+  for (int rr = 0; rr < a.b.R; ++rr) {
+    const int k0 = a.idx_off[rr], kr = a.idx_off[rr + 1] - k0;
+    const int nb = (kr + span - 1) / span;
+    if (blk < nb) {
+      it.r = rr;
+      it.i0 = k0 + blk * span;
+      it.cnt = min(span, kr - blk * span);
+      break;
+    }
+    blk -= nb;
+  }
+  return it;
+}
+
+// Key tiles of an item: up to its last row's position.
+__device__ __forceinline__ int item_tiles(const RefArgs& a, const Item& it) {
+  if (it.i0 < 0) return 0;
+  const int N = a.b.tok_off[it.r + 1] - a.b.tok_off[it.r];
+  const int p_max = min(a.idx[it.i0 + it.cnt - 1], N - 1);
+  return p_max < 0 ? 0 : p_max / kKT + 1;
+}
+
 struct Smem {
-  uint8_t* q;        // [2 halves][128 rows][128 B]
+  uint8_t* q;        // [kQBufs][2 halves][128 rows][128 B]
   uint8_t* k;        // [kKStages][2 halves][128 keys][128 B]
   uint8_t* v;        // [kVStages][2 halves][128 keys][128 B]
   uint64_t *kfull, *kempty;   // [kKStages]
   uint64_t *vfull, *vempty;   // [kVStages]
   uint64_t *sfull, *pfull;    // [2] per S buffer
   uint64_t *pvdone;           // once per key tile
-  uint64_t *qready, *mdone;
+  uint64_t *qfull, *qempty;   // [kQBufs] query tile (and item index) of one item
+  uint64_t *ofull, *oempty;   // once per item: O complete / O read out
+  uint64_t *mdone;
   uint32_t* tmem_slot;
   volatile int* abort;
   uint32_t* counters;  // [0] K loads, [1] V loads, [2] K consumed, [3] V consumed
   float* xmax;         // [2 tile parities][2 halves][128 rows] half-row maxima
   float* xsum;         // [2 halves][128 rows] half-row sums at the end
+  // per query buffer, written by the loader with the query tile: the decoded
+  // item {u (-1: no more work), l, g, r, i0, cnt, key tiles, N_r} and the
+  // positions of its selected rows, so the other roles read no global memory
+  // between items
+  volatile int* rec;   // [kQBufs][kRecInts]
+  volatile int* pos;   // [kQBufs][kRows]
 };
 
 __device__ __forceinline__ Smem carve(uint8_t* raw) {
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(raw) + 1023) & ~uintptr_t(1023));
   Smem s;
   s.q = base;
-  s.k = s.q + kQBytes;
+  s.k = s.q + kQBufs * kQBytes;
   s.v = s.k + kKStages * kTileBytes;
   uint64_t* bar = reinterpret_cast<uint64_t*>(s.v + kVStages * kTileBytes);
   s.kfull = bar;
@@ -98,13 +164,18 @@ __device__ __forceinline__ Smem carve(uint8_t* raw) {
   s.sfull = s.vempty + kVStages;
   s.pfull = s.sfull + 2;
   s.pvdone = s.pfull + 2;
-  s.qready = s.pvdone + 1;
-  s.mdone = s.qready + 1;
+  s.qfull = s.pvdone + 1;
+  s.qempty = s.qfull + kQBufs;
+  s.ofull = s.qempty + kQBufs;
+  s.oempty = s.ofull + 1;
+  s.mdone = s.oempty + 1;
   s.tmem_slot = reinterpret_cast<uint32_t*>(s.mdone + 1);
   s.abort = reinterpret_cast<volatile int*>(s.tmem_slot + 1);
   s.counters = reinterpret_cast<uint32_t*>(s.tmem_slot + 2);
   s.xmax = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bar) + 256);
   s.xsum = s.xmax + 2 * 2 * 128;
+  s.rec = reinterpret_cast<volatile int*>(s.xsum + 2 * 128);
+  s.pos = s.rec + kQBufs * kRecInts;
   return s;
 }
 
@@ -152,37 +223,26 @@ __device__ __forceinline__ void load_tile(const RefArgs& a, const CUtensorMap* m
   }
 }
 
+// Agreement of the 256 softmax threads (named barrier 1 with an AND
+// reduction): every thread arrives, so all of them take the same branch.
+__device__ __forceinline__ bool softmax_all(bool pred) {
+  uint32_t out;
+  asm volatile(
+      "{\n.reg .pred pi, po;\nsetp.ne.u32 pi, %1, 0;\nbar.red.and.pred po, 1, %2, pi;\nselp.u32 %0, 1, 0, po;\n}\n"
+      : "=r"(out)
+      : "r"(uint32_t(pred)), "n"(kSoftThreads)
+      : "memory");
+  return out != 0;
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
     refresh_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
                       const __grid_constant__ CUtensorMap qmap, const __grid_constant__ RefArgs a) {
   extern __shared__ uint8_t smem_raw[];
   const Smem s = carve(smem_raw);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int l = blockIdx.z, g = blockIdx.y;
   const KvDev& kv = a.kv;
   const int G = kv.G, Hq = kv.Hq;
-
-  // CTA -> (request, first selected row, row count); larger positions first
-  // within each (layer, KV head), whose CTAs run together and share K/V in L2
-  const int span = a.rows_per_tile;
-  int blk = a.n_blocks - 1 - int(blockIdx.x);
-  int r = 0, i0 = -1, cnt = 0;
-  for (int rr = 0; rr < a.b.R; ++rr) {
-    const int k0 = a.idx_off[rr], kr = a.idx_off[rr + 1] - k0;
-    const int nb = (kr + span - 1) / span;
-    if (blk < nb) {
-      r = rr;
-      i0 = k0 + blk * span;
-      cnt = min(span, kr - blk * span);
-      break;
-    }
-    blk -= nb;
-  }
-  if (i0 < 0) return;
-  const int t0 = a.b.tok_off[r], N = a.b.tok_off[r + 1] - t0;
-  const int p_max = min(a.idx[i0 + cnt - 1], N - 1);
-  if (p_max < 0) return;
-  const int ntiles = p_max / kKT + 1;
   const int qrows = a.rows_per_tile * G;          // rows the query box fills
 
   if (tid == 0) {
@@ -200,8 +260,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       // wait: P(t+2) needs S(t+2), issued only after the wait for P(t)
       tc::mbar_init(&s.pfull[i], kSoftThreads);
     }
+    for (int i = 0; i < kQBufs; ++i) {
+      tc::mbar_init(&s.qfull[i], 1);   // the loader's expect-tx (or plain arrive at the end)
+      tc::mbar_init(&s.qempty[i], 2);  // the MMA thread's commit + the softmax warps' read of the item
+    }
     tc::mbar_init(s.pvdone, 1);
-    tc::mbar_init(s.qready, 2);  // the loader's expect-tx plus the softmax warps
+    tc::mbar_init(s.ofull, 1);
+    tc::mbar_init(s.oempty, kSoftThreads);
     tc::mbar_init(s.mdone, 1);
     *s.abort = 0;
     for (int i = 0; i < 4; ++i) s.counters[i] = 0;
@@ -217,27 +282,73 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     // ------------------------------------------------------- loads (warp 0)
-    if (lane == 0) {
-      tc::mbar_arrive_expect_tx(s.qready, 2u * 128u * uint32_t(qrows));
-      for (int hf = 0; hf < 2; ++hf)
-        tc::tma_load_3d(s.q + hf * kQHalf, &qmap, s.qready, hf * 64, g * G, l * a.n_sel + i0);
-    }
-    uint32_t nk = 0, nv = 0;
-    for (int t = 0; t < ntiles; ++t) {
-      const int sk = t % kKStages;
-      if (!__all_sync(0xffffffffu, wait_or_abort(&s.kempty[sk], ((t / kKStages) & 1) ^ 1, s.abort))) {
+    uint32_t nk = 0, nv = 0, T = 0;
+    bool ok = true;
+    for (uint32_t n = 0; ok; ++n) {
+      int u = 0;
+      if (lane == 0) {
+        u = n == 0 ? int(blockIdx.x) : int(gridDim.x) + atomicAdd(a.next_item, 1);
+        if (u >= a.n_items) u = -1;
+      }
+      u = __shfl_sync(0xffffffffu, u, 0);
+      const Item it = decode_item(a, u < 0 ? 0 : u);
+      const int nt = u < 0 ? 0 : item_tiles(a, it);
+      const int t0 = a.b.tok_off[it.r], N = a.b.tok_off[it.r + 1] - t0;
+      int my_pos[kRows / 32];  // positions of the item's rows, loaded before the buffer is free
+#pragma unroll
+      for (int k = 0; k < kRows / 32; ++k) {
+        const int i = lane + 32 * k;
+        my_pos[k] = (u >= 0 && i < it.cnt) ? a.idx[it.i0 + i] : -1;
+      }
+      const int qs = n & 1;
+      if (!__all_sync(0xffffffffu, wait_or_abort(&s.qempty[qs], ((n >> 1) & 1) ^ 1, s.abort))) {
         if (lane == 0) raise_abort(a, s, tc::kSiteLoad);
         break;
       }
-      load_tile(a, &kmap, s.k + sk * kTileBytes, &s.kfull[sk], l, g, r, t0, N, t * kKT, lane);
-      ++nk;
-      const int sv = t % kVStages;
-      if (!__all_sync(0xffffffffu, wait_or_abort(&s.vempty[sv], ((t / kVStages) & 1) ^ 1, s.abort))) {
-        if (lane == 0) raise_abort(a, s, tc::kSiteLoad);
-        break;
+#pragma unroll
+      for (int k = 0; k < kRows / 32; ++k) s.pos[qs * kRows + lane + 32 * k] = my_pos[k];
+      if (lane == 0) {
+        volatile int* rec = s.rec + qs * kRecInts;
+        rec[0] = u;
+        rec[1] = it.l;
+        rec[2] = it.g;
+        rec[3] = it.r;
+        rec[4] = it.i0;
+        rec[5] = it.cnt;
+        rec[6] = nt;
+        rec[7] = N;
       }
-      load_tile(a, &vmap, s.v + sv * kTileBytes, &s.vfull[sv], l, g, r, t0, N, t * kKT, lane);
-      ++nv;
+      __threadfence_block();
+      __syncwarp();  // the lanes' positions are ordered before lane 0's release below
+      if (lane == 0) {
+        if (u < 0) {
+          tc::mbar_arrive(&s.qfull[qs]);  // no more work: the others stop at this buffer
+        } else {
+          tc::mbar_arrive_expect_tx(&s.qfull[qs], 2u * 128u * uint32_t(qrows));
+          for (int hf = 0; hf < 2; ++hf)
+            tc::tma_load_3d(s.q + qs * kQBytes + hf * kQHalf, &qmap, &s.qfull[qs], hf * 64,
+                            it.g * G, it.l * a.n_sel + max(it.i0, 0));
+        }
+      }
+      if (u < 0) break;
+      for (int t = 0; t < nt; ++t, ++T) {
+        const int sk = T % kKStages;
+        if (!__all_sync(0xffffffffu, wait_or_abort(&s.kempty[sk], ((T / kKStages) & 1) ^ 1, s.abort))) {
+          if (lane == 0) raise_abort(a, s, tc::kSiteLoad);
+          ok = false;
+          break;
+        }
+        load_tile(a, &kmap, s.k + sk * kTileBytes, &s.kfull[sk], it.l, it.g, it.r, t0, N, t * kKT, lane);
+        ++nk;
+        const int sv = T % kVStages;
+        if (!__all_sync(0xffffffffu, wait_or_abort(&s.vempty[sv], ((T / kVStages) & 1) ^ 1, s.abort))) {
+          if (lane == 0) raise_abort(a, s, tc::kSiteLoad);
+          ok = false;
+          break;
+        }
+        load_tile(a, &vmap, s.v + sv * kTileBytes, &s.vfull[sv], it.l, it.g, it.r, t0, N, t * kKT, lane);
+        ++nv;
+      }
     }
     if (lane == 0) {
       s.counters[0] = nk;
@@ -245,49 +356,68 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == 1 && lane == 0) {
     // ------------------------------------------------------------------ MMA
-    uint32_t ck = 0, cv = 0;
+    uint32_t ck = 0, cv = 0, T = 0;
+    bool ok = true, any_pv = false;
     const uint32_t idesc_s = tc::idesc_bf16(kRows, kKT);
     const uint32_t idesc_o = tc::idesc_bf16(kRows, kD, /*b_mn_major=*/true);
-    const uint32_t q_addr = tc::smem_u32(s.q);
-    // S(t) = Q K(t)^T into S buffer t & 1
-    auto issue_s = [&](int t) -> bool {
-      const int sk = t % kKStages;
-      if (!wait_or_abort(&s.kfull[sk], (t / kKStages) & 1, s.abort)) return false;
+    // S(T) = Q K(T)^T into S buffer T & 1
+    auto issue_s = [&](uint32_t q_addr, uint32_t Ts) -> bool {
+      const int sk = Ts % kKStages;
+      if (!wait_or_abort(&s.kfull[sk], (Ts / kKStages) & 1, s.abort)) return false;
       ++ck;
       tc::tc_fence_after();
       const uint32_t k_addr = tc::smem_u32(s.k + sk * kTileBytes);
 #pragma unroll
       for (int kk = 0; kk < 8; ++kk) {
         const uint32_t off = (kk & 3) * 32;
-        tc::mma_bf16(tmem + uint32_t(t & 1) * kSCols, tc::desc_sw128(q_addr + (kk >> 2) * kQHalf + off),
+        tc::mma_bf16(tmem + (Ts & 1) * kSCols, tc::desc_sw128(q_addr + (kk >> 2) * kQHalf + off),
                      tc::desc_sw128(k_addr + (kk >> 2) * kTileHalf + off), idesc_s, kk > 0);
       }
-      tc::mma_commit(&s.sfull[t & 1]);
+      tc::mma_commit(&s.sfull[Ts & 1]);
       tc::mma_commit(&s.kempty[sk]);
       return true;
     };
-    bool ok = wait_or_abort(s.qready, 0, s.abort);
-    if (ok) ok = issue_s(0);
-    if (ok && ntiles > 1) ok = issue_s(1);
-    for (int t = 0; t < ntiles && ok; ++t) {
-      const int sv = t % kVStages;
-      if (!wait_or_abort(&s.vfull[sv], (t / kVStages) & 1, s.abort)) { ok = false; break; }
-      ++cv;
-      if (!wait_or_abort(&s.pfull[t & 1], (t >> 1) & 1, s.abort)) { ok = false; break; }
+    for (uint32_t n = 0; ok; ++n) {
+      const int qs = n & 1;
+      if (!wait_or_abort(&s.qfull[qs], (n >> 1) & 1, s.abort)) { ok = false; break; }
+      if (s.rec[qs * kRecInts] < 0) break;
+      const int nt = s.rec[qs * kRecInts + 6];
+      const uint32_t q_addr = tc::smem_u32(s.q + qs * kQBytes);
       tc::tc_fence_after();
-      const uint32_t v_addr = tc::smem_u32(s.v + sv * kTileBytes);
-      const uint32_t pb = tmem + uint32_t(t & 1) * kSCols + kPCol;
+      // the S buffers are free once the previous item's last P.V has completed
+      // (the latest pvdone commit, so its parity cannot alias)
+      if (any_pv && nt > 0 && !wait_or_abort(s.pvdone, (T - 1) & 1, s.abort)) { ok = false; break; }
+      if (nt > 0 && !issue_s(q_addr, T)) { ok = false; break; }
+      if (nt > 1 && !issue_s(q_addr, T + 1)) { ok = false; break; }
+      if (nt <= 2) tc::mma_commit(&s.qempty[qs]);  // every S of this item is issued
+      for (int t = 0; t < nt; ++t) {
+        const uint32_t Tc = T + t;
+        const int sv = Tc % kVStages;
+        if (!wait_or_abort(&s.vfull[sv], (Tc / kVStages) & 1, s.abort)) { ok = false; break; }
+        ++cv;
+        if (!wait_or_abort(&s.pfull[Tc & 1], (Tc >> 1) & 1, s.abort)) { ok = false; break; }
+        // O of the previous item must have been read out before P(0) V(0) overwrites it
+        if (t == 0 && n > 0 && !wait_or_abort(s.oempty, (n - 1) & 1, s.abort)) { ok = false; break; }
+        tc::tc_fence_after();
+        const uint32_t v_addr = tc::smem_u32(s.v + sv * kTileBytes);
+        const uint32_t pb = tmem + (Tc & 1) * kSCols + kPCol;
 #pragma unroll
-      for (int kk = 0; kk < kKT / 16; ++kk)  // O += P(t) V(t)
-        tc::mma_bf16_ts(tmem + kOCol, pb + kk * 8, tc::desc_sw128_mn(v_addr + kk * 2048, kTileHalf),
-                        idesc_o, t > 0 || kk > 0);
-      tc::mma_commit(s.pvdone);
-      tc::mma_commit(&s.vempty[sv]);
-      if (t + 2 < ntiles) {
-        // S(t+2) overwrites P(t): wait until P(t) V(t) has completed
-        if (!wait_or_abort(s.pvdone, t & 1, s.abort)) { ok = false; break; }
-        if (!issue_s(t + 2)) { ok = false; break; }
+        for (int kk = 0; kk < kKT / 16; ++kk)  // O += P(t) V(t)
+          tc::mma_bf16_ts(tmem + kOCol, pb + kk * 8, tc::desc_sw128_mn(v_addr + kk * 2048, kTileHalf),
+                          idesc_o, t > 0 || kk > 0);
+        tc::mma_commit(s.pvdone);
+        tc::mma_commit(&s.vempty[sv]);
+        any_pv = true;
+        if (t + 2 < nt) {
+          // S(t+2) overwrites P(t): wait until P(t) V(t) has completed
+          if (!wait_or_abort(s.pvdone, Tc & 1, s.abort)) { ok = false; break; }
+          if (!issue_s(q_addr, Tc + 2)) { ok = false; break; }
+          if (t + 3 == nt) tc::mma_commit(&s.qempty[qs]);  // that was the item's last S
+        }
       }
+      if (!ok) break;
+      T += nt;
+      tc::mma_commit(s.ofull);  // O of this item is complete once this arrives
     }
     if (!ok) raise_abort(a, s, tc::kSiteMma);
     s.counters[2] = ck;
@@ -302,131 +432,151 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int row = quarter * 32 + lane;                 // TMEM lane = query row of the tile
     const uint32_t lane_base = uint32_t(quarter * 32) << 16;
     const uint32_t tl = tmem + lane_base;
-    const bool row_ok = row < cnt * G;
-    const int i_row = i0 + (row_ok ? row / G : 0);
-    const int h_row = g * G + (row_ok ? row % G : 0);
-    int p_row = row_ok ? a.idx[i_row] : -1;
-    if (p_row >= N) p_row = -1;
-    if (qrows < kRows) {  // rows past the query box: zero (their S is masked anyway)
-      for (int x = et; x < (kRows - qrows) * 16; x += kSoftThreads) {
-        const int rr = qrows + (x >> 4), ch = x & 15;
-        *reinterpret_cast<uint4*>(s.q + (ch >> 3) * kQHalf + tc::sw128_offset(rr, ch & 7)) = make_uint4(0u, 0u, 0u, 0u);
-      }
-      tc::fence_proxy_async_smem();
-    }
-    asm volatile("bar.sync 1, %0;" ::"n"(kSoftThreads) : "memory");
-    if (et == 0) tc::mbar_arrive(s.qready);
-
     bool ok = true;
-    float m_ref = -INFINITY, lsum = 0.f;  // running max (scaled, log2 units, same in both halves) and half-row sum
-    for (int t = 0; t < ntiles; ++t) {
-      const uint32_t sb = tl + uint32_t(t & 1) * kSCols;
-      // the tcgen05.ld below is warp-collective: the whole warp goes on or stops
-      const bool got = __all_sync(0xffffffffu, ok && wait_or_abort(&s.sfull[t & 1], (t >> 1) & 1, s.abort));
-      if (!got) {
-        if (ok) raise_abort(a, s, tc::kSiteMma);
+    uint32_t T = 0;
+    for (uint32_t n = 0;; ++n) {
+      const int qs = n & 1;
+      // all 256 threads agree to go on, so the named barriers below stay uniform
+      const bool got = wait_or_abort(&s.qfull[qs], (n >> 1) & 1, s.abort);
+      if (!softmax_all(ok && got)) {
+        if (ok) raise_abort(a, s, tc::kSiteLoad);
+        break;
+      }
+      const volatile int* rec = s.rec + qs * kRecInts;
+      const int u = rec[0];
+      Item it;
+      it.l = rec[1];
+      it.g = rec[2];
+      it.r = rec[3];
+      it.i0 = rec[4];
+      it.cnt = rec[5];
+      const int nt = rec[6], N = rec[7];
+      const bool row_ok = u >= 0 && row < it.cnt * G;
+      const int i_row = it.i0 + (row_ok ? row / G : 0);
+      const int h_row = it.g * G + (row_ok ? row % G : 0);
+      int p_row = row_ok ? s.pos[qs * kRows + row / G] : -1;  // rows past the item (or the box) are fully masked
+      if (p_row >= N) p_row = -1;
+      asm volatile("bar.sync 1, %0;" ::"n"(kSoftThreads) : "memory");  // everyone has read the record
+      if (et == 0) tc::mbar_arrive(&s.qempty[qs]);
+      if (u < 0) break;
+
+      float m_ref = -INFINITY, lsum = 0.f;  // running max (scaled, log2 units, same in both halves) and half-row sum
+      for (int t = 0; t < nt; ++t) {
+        const uint32_t Tc = T + t;
+        const uint32_t sb = tl + (Tc & 1) * kSCols;
+        // the tcgen05.ld below is warp-collective: the whole warp goes on or stops
+        const bool gs = __all_sync(0xffffffffu, ok && wait_or_abort(&s.sfull[Tc & 1], (Tc >> 1) & 1, s.abort));
+        if (!gs) {
+          if (ok) raise_abort(a, s, tc::kSiteMma);
+          ok = false;
+        }
+        float sv[64];
+        float hmax = -INFINITY;
+        const int j0 = t * kKT + hh * 64;
+        if (gs) {
+          tc::tc_fence_after();
+          tc::tmem_ld64(sb + hh * 64, sv);
+          if (j0 + 63 > p_row) {  // part of this half is past this row's position
+#pragma unroll
+            for (int i = 0; i < 64; ++i)
+              if (j0 + i > p_row) sv[i] = -INFINITY;
+          }
+          float tm[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+          for (int i = 0; i < 32; ++i) tm[i & 3] = tc::fmax3(tm[i & 3], sv[2 * i], sv[2 * i + 1]);
+          hmax = fmaxf(fmaxf(tm[0], tm[1]), fmaxf(tm[2], tm[3]));
+        }
+        // exchange the half-row maxima (buffers alternate with the tile, so a
+        // half that runs ahead never overwrites a value its partner still reads)
+        float* xm = s.xmax + (Tc & 1) * 256;
+        xm[hh * 128 + row] = hmax;
+        asm volatile("bar.sync 1, %0;" ::"n"(kSoftThreads) : "memory");
+        if (!ok) continue;
+        const float tmax = fmaxf(hmax, xm[(hh ^ 1) * 128 + row]) * a.scale_log2;
+        const bool need = tmax > m_ref + kRescaleLog2 || (m_ref == -INFINITY && tmax != -INFINITY);
+        const float alpha = need ? tc::ex2(m_ref - tmax) : 1.f;  // 0 when m_ref is -inf
+        if (need) {
+          lsum *= alpha;
+          m_ref = tmax;
+        }
+        // this half of P = 2^(S scale - m) in bf16 pairs over the upper half of S
+        // (one packed FMA per pair for scale and bias, packed adds for the sum).
+        // A row with no visible key yet (m = -inf) uses bias 0: its logits are
+        // all -inf and its P is 0.
+        const float2 sc2 = make_float2(a.scale_log2, a.scale_log2);
+        const float2 nb2 = m_ref == -INFINITY ? make_float2(0.f, 0.f) : make_float2(-m_ref, -m_ref);
+        float2 ls2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+        {
+          uint32_t pw[32];
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const float2 y = tc::ffma2(make_float2(sv[2 * i], sv[2 * i + 1]), sc2, nb2);
+            const float2 pp = make_float2(tc::ex2(y.x), tc::ex2(y.y));
+            ls2[i & 1] = tc::fadd2(ls2[i & 1], pp);
+            __nv_bfloat162 pr = __floats2bfloat162_rn(pp.x, pp.y);
+            pw[i] = *reinterpret_cast<uint32_t*>(&pr);
+          }
+          tc::tmem_st32u(sb + kPCol + hh * 32, pw);
+        }
+        const float ls[4] = {ls2[0].x, ls2[0].y, ls2[1].x, ls2[1].y};
+        lsum += (ls[0] + ls[1]) + (ls[2] + ls[3]);
+        if (__any_sync(0xffffffffu, need) && t > 0) {
+          // P(t-1) V(t-1) must have completed before this warp rescales its half
+          // of O. S(t) was issued after P(t-2) V(t-2) completed, so pvdone is at
+          // most one phase behind here and its parity cannot alias; P(t) V(t)
+          // waits for this warp's pfull arrival below.
+          if (!__all_sync(0xffffffffu, wait_or_abort(s.pvdone, (Tc - 1) & 1, s.abort))) {
+            raise_abort(a, s, tc::kSiteMma);
+            ok = false;
+            continue;
+          }
+          tc::tc_fence_after();
+          for (int c = hh * 64; c < hh * 64 + 64; c += 32) {
+            float o[32];
+            tc::tmem_ld32(tl + kOCol + c, o);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) o[i] *= alpha;
+            tc::tmem_st32(tl + kOCol + c, o);
+          }
+        }
+        tc::tc_fence_before();
+        tc::mbar_arrive(&s.pfull[Tc & 1]);
+      }
+      T += nt;
+      // row sum = the two halves' sums (same running max in both)
+      s.xsum[hh * 128 + row] = lsum;
+      asm volatile("bar.sync 1, %0;" ::"n"(kSoftThreads) : "memory");
+      const float total = s.xsum[row] + s.xsum[128 + row];
+      // O of this item is complete once the MMA thread's per-item commit has
+      // arrived (it cannot run a phase ahead: the next one needs this warp's P)
+      const bool fin = __all_sync(0xffffffffu, ok && wait_or_abort(s.ofull, n & 1, s.abort));
+      if (!fin && ok) {
+        raise_abort(a, s, tc::kSiteFinal);
         ok = false;
       }
-      float sv[64];
-      float hmax = -INFINITY;
-      const int j0 = t * kKT + hh * 64;
-      if (got) {
+      if (fin) {
         tc::tc_fence_after();
-        tc::tmem_ld64(sb + hh * 64, sv);
-        if (j0 + 63 > p_row) {  // part of this half is past this row's position
-#pragma unroll
-          for (int i = 0; i < 64; ++i)
-            if (j0 + i > p_row) sv[i] = -INFINITY;
-        }
-        float tm[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-#pragma unroll
-        for (int i = 0; i < 32; ++i) tm[i & 3] = tc::fmax3(tm[i & 3], sv[2 * i], sv[2 * i + 1]);
-        hmax = fmaxf(fmaxf(tm[0], tm[1]), fmaxf(tm[2], tm[3]));
-      }
-      // exchange the half-row maxima (buffers alternate with the tile, so a
-      // half that runs ahead never overwrites a value its partner still reads)
-      float* xm = s.xmax + (t & 1) * 256;
-      xm[hh * 128 + row] = hmax;
-      asm volatile("bar.sync 1, %0;" ::"n"(kSoftThreads) : "memory");
-      if (!ok) continue;
-      const float tmax = fmaxf(hmax, xm[(hh ^ 1) * 128 + row]) * a.scale_log2;
-      const bool need = tmax > m_ref + kRescaleLog2 || (m_ref == -INFINITY && tmax != -INFINITY);
-      const float alpha = need ? tc::ex2(m_ref - tmax) : 1.f;  // 0 when m_ref is -inf
-      if (need) {
-        lsum *= alpha;
-        m_ref = tmax;
-      }
-      // this half of P = 2^(S scale - m) in bf16 pairs over the upper half of S
-      // (one packed FMA per pair for scale and bias, packed adds for the sum).
-      // A row with no visible key yet (m = -inf) uses bias 0: its logits are
-      // all -inf and its P is 0.
-      const float2 sc2 = make_float2(a.scale_log2, a.scale_log2);
-      const float2 nb2 = m_ref == -INFINITY ? make_float2(0.f, 0.f) : make_float2(-m_ref, -m_ref);
-      float2 ls2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
-      {
-        uint32_t pw[32];
-#pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          const float2 y = tc::ffma2(make_float2(sv[2 * i], sv[2 * i + 1]), sc2, nb2);
-          const float2 pp = make_float2(tc::ex2(y.x), tc::ex2(y.y));
-          ls2[i & 1] = tc::fadd2(ls2[i & 1], pp);
-          __nv_bfloat162 pr = __floats2bfloat162_rn(pp.x, pp.y);
-          pw[i] = *reinterpret_cast<uint32_t*>(&pr);
-        }
-        tc::tmem_st32u(sb + kPCol + hh * 32, pw);
-      }
-      const float ls[4] = {ls2[0].x, ls2[0].y, ls2[1].x, ls2[1].y};
-      lsum += (ls[0] + ls[1]) + (ls[2] + ls[3]);
-      if (__any_sync(0xffffffffu, need) && t > 0) {
-        // P(t-1) V(t-1) must have completed before this warp rescales its half
-        // of O. S(t) was issued after P(t-2) V(t-2) completed, so pvdone is at
-        // most one phase behind here and its parity cannot alias; P(t) V(t)
-        // waits for this warp's pfull arrival below.
-        if (!__all_sync(0xffffffffu, wait_or_abort(s.pvdone, (t - 1) & 1, s.abort))) {
-          raise_abort(a, s, tc::kSiteMma);
-          ok = false;
-          continue;
-        }
-        tc::tc_fence_after();
+        const float inv = total > 0.f ? 1.f / total : 0.f;
+        __nv_bfloat16* dst = a.out + ((int64_t(it.l) * a.n_sel + i_row) * Hq + h_row) * kD;
         for (int c = hh * 64; c < hh * 64 + 64; c += 32) {
           float o[32];
           tc::tmem_ld32(tl + kOCol + c, o);
+          if (row_ok && p_row >= 0) {
 #pragma unroll
-          for (int i = 0; i < 32; ++i) o[i] *= alpha;
-          tc::tmem_st32(tl + kOCol + c, o);
-        }
-      }
-      tc::tc_fence_before();
-      tc::mbar_arrive(&s.pfull[t & 1]);
-    }
-    // row sum = the two halves' sums (same running max in both)
-    s.xsum[hh * 128 + row] = lsum;
-    asm volatile("bar.sync 1, %0;" ::"n"(kSoftThreads) : "memory");
-    const float total = s.xsum[row] + s.xsum[128 + row];
-    // O is complete once every MMA has: wait on the MMA thread's single-use
-    // final commit (pvdone could be two phases behind here and alias)
-    const bool fin = __all_sync(0xffffffffu, ok && wait_or_abort(s.mdone, 0, s.abort));
-    if (!fin && ok) raise_abort(a, s, tc::kSiteFinal);
-    if (fin) {
-      tc::tc_fence_after();
-      const float inv = total > 0.f ? 1.f / total : 0.f;
-      __nv_bfloat16* dst = a.out + ((int64_t(l) * a.n_sel + i_row) * Hq + h_row) * kD;
-      for (int c = hh * 64; c < hh * 64 + 64; c += 32) {
-        float o[32];
-        tc::tmem_ld32(tl + kOCol + c, o);
-        if (row_ok && p_row >= 0) {
+            for (int u4 = 0; u4 < 4; ++u4) {
+              uint32_t w4[4];
 #pragma unroll
-          for (int u = 0; u < 4; ++u) {
-            uint32_t w4[4];
-#pragma unroll
-            for (int k2 = 0; k2 < 4; ++k2) {
-              __nv_bfloat162 pr = __floats2bfloat162_rn(o[u * 8 + 2 * k2] * inv, o[u * 8 + 2 * k2 + 1] * inv);
-              w4[k2] = *reinterpret_cast<uint32_t*>(&pr);
+              for (int k2 = 0; k2 < 4; ++k2) {
+                __nv_bfloat162 pr = __floats2bfloat162_rn(o[u4 * 8 + 2 * k2] * inv, o[u4 * 8 + 2 * k2 + 1] * inv);
+                w4[k2] = *reinterpret_cast<uint32_t*>(&pr);
+              }
+              *reinterpret_cast<uint4*>(dst + c + u4 * 8) = make_uint4(w4[0], w4[1], w4[2], w4[3]);
             }
-            *reinterpret_cast<uint4*>(dst + c + u * 8) = make_uint4(w4[0], w4[1], w4[2], w4[3]);
           }
         }
       }
+      tc::tc_fence_before();
+      tc::mbar_arrive(s.oempty);  // O may be overwritten by the next item
     }
   }
   __syncthreads();
@@ -503,7 +653,8 @@ bool refresh_tc_supported(const KvDev& kv) {
 
 cudaError_t launch_refresh_tc(const KvDev& kv, const BatchDev& b, const int32_t* idx,
                               const int32_t* idx_off_dev, const int32_t* idx_off_host, int32_t n_sel,
-                              const void* q_rows, void* out, int32_t* status, cudaStream_t stream) {
+                              const void* q_rows, void* out, int32_t* work_counter, int32_t* status,
+                              cudaStream_t stream) {
   if (n_sel == 0) return cudaSuccess;
   CUtensorMap kmap, vmap, qmap;
   if (!make_map(&kmap, kv, kv.k) || !make_map(&vmap, kv, kv.v) ||
@@ -524,14 +675,26 @@ cudaError_t launch_refresh_tc(const KvDev& kv, const BatchDev& b, const int32_t*
     blocks += (kr + a.rows_per_tile - 1) / a.rows_per_tile;
   }
   a.n_blocks = blocks;
+  a.n_items = blocks * kv.Hkv * kv.L;
+  a.next_item = work_counter;
   a.scale_log2 = kLog2e / sqrtf(float(kD));
   a.status = status;
   if (blocks == 0) return cudaSuccess;
-  cudaError_t err = cudaFuncSetAttribute(refresh_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         int(kSmem));
-  if (err) return err;
-  const dim3 grid(blocks, kv.Hkv, kv.L);
-  refresh_tc_kernel<<<grid, kThreads, kSmem, stream>>>(kmap, vmap, qmap, a);
+  int dev = 0, sms = 0;
+  cudaError_t err;
+  if ((err = cudaGetDevice(&dev))) return err;
+  if ((err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev))) return err;
+  int l2 = 0;
+  if ((err = cudaDeviceGetAttribute(&l2, cudaDevAttrL2CacheSize, dev))) return err;
+  // longest-first when the whole K/V of the batch fits in half of L2 (the rest
+  // holds queries and outputs), else (layer, head)-major
+  const double kv_bytes = 2.0 * double(kv.L) * kv.Hkv * double(kv.n_tot) * kD * 2;
+  a.blocks_major = kv_bytes <= 0.5 * double(l2) ? 1 : 0;
+  if ((err = cudaFuncSetAttribute(refresh_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  int(kSmem))))
+    return err;
+  if ((err = cudaMemsetAsync(work_counter, 0, sizeof(int32_t), stream))) return err;
+  refresh_tc_kernel<<<std::min(a.n_items, sms), kThreads, kSmem, stream>>>(kmap, vmap, qmap, a);
   count_launches(1);
   return cudaGetLastError();
 }
