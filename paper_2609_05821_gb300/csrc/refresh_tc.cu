@@ -7,14 +7,15 @@
 // the KV head. Keys stream in tiles of 128 (a tcgen05.mma costs about the same
 // issue time for N = 64 and N = 128, so wide tiles halve the instruction
 // count). The kernel is persistent: one CTA per SM takes items from an atomic
-// counter (largest positions first within each (layer, KV head), so the CTAs
-// in flight share K/V in L2), and the query tile of the next item loads into
-// a second buffer while the current item computes. Roles (320 threads):
+// counter, and the query tile of the next item loads into a second buffer
+// while the current item computes. Roles (352 threads):
 //   warp 0     TMA loads: the query tile of each item (a 3-D box of 64 dims x
 //              G heads x floor(128/G) rows lands in the tile's row order) into
-//              one of two buffers, then its K and V tiles (two stages each);
-//              the lanes issue the copies of a tile together (one per page
-//              half when paged)
+//              one of two buffers, then its K tiles (two stages); the lanes
+//              issue the copies of a tile together (one per page half when
+//              paged)
+//   warp 10    the same for the V tiles (two stages), so that a V stage
+//              waiting for its P.V never holds back K and the next query tile
 //   warp 1     one thread issues tcgen05 MMAs: S(t) = Q K(t)^T into one of two
 //              TMEM buffers, O += P(t) V(t) with P read from TMEM
 //   warps 2-9  softmax, two warps per TMEM lane quarter: each thread owns one
@@ -48,7 +49,8 @@ constexpr int kD = 128;
 constexpr int kKT = 128;                         // keys per tile
 constexpr int kRows = 128;                       // rows per query tile
 constexpr int kSoftThreads = 256;
-constexpr int kThreads = 64 + kSoftThreads;
+constexpr int kVWarp = 10;                       // after the loader, MMA and eight softmax warps
+constexpr int kThreads = 64 + kSoftThreads + 32;
 constexpr int kKStages = 2;
 constexpr int kVStages = 2;
 constexpr int kQBufs = 2;
@@ -56,7 +58,7 @@ constexpr uint32_t kQHalf = kRows * 128;         // 16 KB: one 64-dim half of th
 constexpr uint32_t kQBytes = 2 * kQHalf;         // 32 KB
 constexpr uint32_t kTileHalf = kKT * 128;        // 16 KB: one 64-dim half of a K or V tile
 constexpr uint32_t kTileBytes = 2 * kTileHalf;   // 32 KB
-constexpr int kRecInts = 8;                      // decoded item record (see Smem::rec)
+constexpr int kRecInts = 9;                      // decoded item record (see Smem::rec)
 constexpr uint32_t kSmem = 1024 + kQBufs * kQBytes + (kKStages + kVStages) * kTileBytes + 256 +
                            2 * 2 * 128 * 4 + 2 * 128 * 4 + kQBufs * (kRecInts + kRows) * 4;
 constexpr uint32_t kTmemCols = 512;              // 384 used; allocations are powers of two
@@ -143,7 +145,7 @@ struct Smem {
   float* xmax;         // [2 tile parities][2 halves][128 rows] half-row maxima
   float* xsum;         // [2 halves][128 rows] half-row sums at the end
   // per query buffer, written by the loader with the query tile: the decoded
-  // item {u (-1: no more work), l, g, r, i0, cnt, key tiles, N_r} and the
+  // item {u (-1: no more work), l, g, r, i0, cnt, key tiles, N_r, t0} and the
   // positions of its selected rows, so the other roles read no global memory
   // between items
   volatile int* rec;   // [kQBufs][kRecInts]
@@ -262,7 +264,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int i = 0; i < kQBufs; ++i) {
       tc::mbar_init(&s.qfull[i], 1);   // the loader's expect-tx (or plain arrive at the end)
-      tc::mbar_init(&s.qempty[i], 2);  // the MMA thread's commit + the softmax warps' read of the item
+      tc::mbar_init(&s.qempty[i], 3);  // the MMA thread's commit + the softmax and V warps' reads of the item
     }
     tc::mbar_init(s.pvdone, 1);
     tc::mbar_init(s.ofull, 1);
@@ -282,7 +284,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     // ------------------------------------------------------- loads (warp 0)
-    uint32_t nk = 0, nv = 0, T = 0;
+    uint32_t nk = 0, T = 0;
     bool ok = true;
     for (uint32_t n = 0; ok; ++n) {
       int u = 0;
@@ -317,6 +319,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         rec[5] = it.cnt;
         rec[6] = nt;
         rec[7] = N;
+        rec[8] = t0;
       }
       __threadfence_block();
       __syncwarp();  // the lanes' positions are ordered before lane 0's release below
@@ -340,20 +343,40 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         load_tile(a, &kmap, s.k + sk * kTileBytes, &s.kfull[sk], it.l, it.g, it.r, t0, N, t * kKT, lane);
         ++nk;
+      }
+    }
+    if (lane == 0) s.counters[0] = nk;
+  } else if (warp == kVWarp) {
+    // --------------------------------------------------- V loads (warp 10)
+    // on a warp of their own: a V stage frees only once its P.V has
+    // completed, and waiting for it must not hold back the K tiles and the
+    // next item's query tile
+    uint32_t nv = 0, T = 0;
+    for (uint32_t n = 0;; ++n) {
+      const int qs = n & 1;
+      if (!__all_sync(0xffffffffu, wait_or_abort(&s.qfull[qs], (n >> 1) & 1, s.abort))) {
+        if (lane == 0) raise_abort(a, s, tc::kSiteLoad);
+        break;
+      }
+      const volatile int* rec = s.rec + qs * kRecInts;
+      const int u = rec[0], l = rec[1], g = rec[2], r = rec[3], nt = rec[6], N = rec[7], t0 = rec[8];
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&s.qempty[qs]);  // this warp is done with the record
+      if (u < 0) break;
+      bool ok = true;
+      for (int t = 0; t < nt; ++t, ++T) {
         const int sv = T % kVStages;
         if (!__all_sync(0xffffffffu, wait_or_abort(&s.vempty[sv], ((T / kVStages) & 1) ^ 1, s.abort))) {
           if (lane == 0) raise_abort(a, s, tc::kSiteLoad);
           ok = false;
           break;
         }
-        load_tile(a, &vmap, s.v + sv * kTileBytes, &s.vfull[sv], it.l, it.g, it.r, t0, N, t * kKT, lane);
+        load_tile(a, &vmap, s.v + sv * kTileBytes, &s.vfull[sv], l, g, r, t0, N, t * kKT, lane);
         ++nv;
       }
+      if (!ok) break;
     }
-    if (lane == 0) {
-      s.counters[0] = nk;
-      s.counters[1] = nv;
-    }
+    if (lane == 0) s.counters[1] = nv;
   } else if (warp == 1 && lane == 0) {
     // ------------------------------------------------------------------ MMA
     uint32_t ck = 0, cv = 0, T = 0;
@@ -424,7 +447,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     s.counters[3] = cv;
     tc::mma_commit(s.mdone);  // every MMA issued above has completed once this arrives
     tc::mbar_wait(s.mdone, 0);
-  } else if (warp >= 2) {
+  } else if (warp >= 2 && warp < kVWarp) {
     // -------------------------------------------------------------- softmax
     const int et = tid - 64;                             // 0..255
     const int hh = et >> 7;                              // half of the key tile / of O
