@@ -172,7 +172,7 @@ def work_model(pipe) -> dict:
     copy_bytes = 2 * 2 * Lall * k_sel * Hkv * d * esz
     idx = pipe.idx[:k_sel].cpu().tolist()
     off = pipe.idx_off.tolist()
-    ref_flops, ref_bytes = 0, 2 * 2 * Lall * k_sel * Hq * d * esz
+    ref_flops, ref_bytes = 0, 2 * Lall * k_sel * Hq * d * esz  # the query rows in, the output out
     for r in range(R):
         ps = idx[off[r]:off[r + 1]]
         ref_flops += sum(4 * Hq * d * (p + 1) for p in ps) * Lall
