@@ -65,6 +65,7 @@ __all__ = [
     "quota_select",
     "refresh_mask",
     "score_request",
+    "staleness_iso",
     "kv_gather",
     "kv_scatter",
     "refresh_attention",
@@ -393,6 +394,45 @@ def refresh_mask(q: np.ndarray, k: np.ndarray, v: np.ndarray, img_off: Sequence[
     out = dict(sc)
     out.update({"k": kk, "c": c, "s_hat": s_hat, "idx": idx, "mask": mask})
     return out
+
+
+# --------------------------------------------------------------------------
+# App. D (Monte Carlo staleness estimator, isotropic): the error a refresh
+# set T leaves, under sampled stale value displacements.
+# --------------------------------------------------------------------------
+def staleness_iso(q: np.ndarray, k: np.ndarray, v: np.ndarray, refreshed: np.ndarray,
+                  z: np.ndarray, kappa: float) -> float:
+    """E_iso(T) = sum_{l, h, q} (1/M) sum_m || sum_{t not in T} alpha_{q,t} xi_t^(m) ||^2.
+
+    xi_t^(m) = kappa ||V_t|| / sqrt(d) * z_t^(m), so xi ~ N(0, kappa^2 ||V_t||^2 / d I)
+    with z the standard normal draws (an input, the random numbers the
+    estimator uses). Readings: xi is drawn per layer, KV head and token with
+    ||V_t|| that head's value norm and d its dimension (the local model of
+    Sec. 3.2 is one layer and head), the G query heads of a KV group read the
+    same xi, alpha is the cached-key softmax over all N visual keys (Eq. 6's
+    alpha), and the functional is summed over the layers, query heads and
+    scoring rows.
+    q: [L, Hq, n_q, d]; k, v: [L, Hkv, N, d]; refreshed: [N] (1 = in T);
+    z: [M, L, Hkv, N, d].
+    """
+    f64 = lambda x: np.asarray(x, dtype=np.float64)
+    n_m = z.shape[0]
+    n_layers, hq = len(k), np.asarray(q[0]).shape[0]
+    keep = 1.0 - f64(refreshed)
+    total = 0.0
+    for l in range(n_layers):
+        q_l, k_l, v_l = f64(q[l]), f64(k[l]), f64(v[l])
+        hkv, n, d = k_l.shape
+        group = hq // hkv
+        for g in range(hkv):
+            scale = kappa * np.sqrt((v_l[g] * v_l[g]).sum(axis=1)) / math.sqrt(d)   # [N]
+            xi = f64(z[:, l, g]) * (scale * keep)[None, :, None]                    # [M, N, d]
+            for h in range(g * group, (g + 1) * group):
+                alpha = softmax_over_visual_keys(cached_key_logits(q_l[h], k_l[g]))  # [n_q, N]
+                for m in range(n_m):
+                    r = alpha @ xi[m]                                                # [n_q, d]
+                    total += (r * r).sum() / n_m
+    return float(total)
 
 
 # --------------------------------------------------------------------------

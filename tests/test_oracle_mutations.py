@@ -101,6 +101,17 @@ def _coefficients_f32_mean_over_k_minus_1(g, lam):
     return (np.float32(1 - lam) + np.float32(lam) * (g / gbar)).astype(np.float32)
 
 
+_staleness_iso = O.staleness_iso  # the original, for the mutants that wrap it
+
+
+def _staleness_no_dim_divisor(q, k, v, refreshed, z, kappa):
+    return _staleness_iso(q, k, v, refreshed, z, kappa) * np.asarray(q).shape[-1]
+
+
+def _staleness_keeps_refreshed(q, k, v, refreshed, z, kappa):
+    return _staleness_iso(q, k, v, np.zeros_like(np.asarray(refreshed, dtype=float)), z, kappa)
+
+
 def _value_norm_mean_of_heads(v_l):
     return np.sqrt((v_l * v_l).sum(axis=2)).mean(axis=0)
 
@@ -176,6 +187,8 @@ MUTANTS = {
     "GQA head h -> h % Hkv": ("head_query_mean_attention", _head_mean_wrong_gqa),
     "divide by Hkv": ("head_query_mean_attention", _head_mean_wrong_divisor),
     "mean of per-head norms": ("value_norms", _value_norm_mean_of_heads),
+    "staleness without the 1/d variance": ("staleness_iso", _staleness_no_dim_divisor),
+    "staleness counts refreshed tokens": ("staleness_iso", _staleness_keeps_refreshed),
     "quotas floored, leftover dropped": ("image_quotas", _quotas_floor_only),
     "quota remainder ties to the higher index": ("image_quotas", _quotas_ties_high),
     "quotas ignore image sizes": ("image_quotas", _quotas_ignore_sizes),

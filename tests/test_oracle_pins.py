@@ -427,6 +427,64 @@ def test_quota_select_per_image_top():
     assert one["idx"].tolist() == O.topk_select(s, 9).tolist()
 
 
+# ------------------------------------------- isotropic staleness (App. D)
+def _stale_case(seed, L=2, hq=4, hkv=2, n_q=3, N=24, d=8, M=3):
+    rng = np.random.default_rng(seed)
+    q = rng.standard_normal((L, hq, n_q, d))
+    k = rng.standard_normal((L, hkv, N, d))
+    v = rng.standard_normal((L, hkv, N, d)) * rng.uniform(0.5, 2.0, size=(L, hkv, N, 1))
+    z = rng.standard_normal((M, L, hkv, N, d))
+    return q, k, v, z
+
+
+def test_staleness_matches_its_expectation():
+    """E[E_iso] = kappa^2 sum_{l,h,q} sum_{t not in T} alpha^2 ||V_t||^2 (the draws are
+    independent, zero-mean, E||xi||^2 = kappa^2 ||V||^2): a large M lands within the
+    Monte Carlo error of that closed form (scipy softmax for alpha)."""
+    q, k, v, _ = _stale_case(30, M=1)
+    L, hq, n_q, d = q.shape
+    hkv, N = k.shape[1], k.shape[2]
+    T = np.zeros(N)
+    T[[1, 5, 9, 20]] = 1
+    M = 4000
+    z = np.random.default_rng(31).standard_normal((M, L, hkv, N, d))
+    got = O.staleness_iso(q, k, v, T, z, 0.7)
+    want = 0.0
+    for l in range(L):
+        for h in range(hq):
+            g = h // (hq // hkv)
+            alpha = _softmax_rows(q[l, h] @ k[l, g].T / math.sqrt(d))
+            vn2 = (v[l, g] ** 2).sum(axis=1)
+            want += 0.49 * ((alpha ** 2) * (vn2 * (1 - T))[None, :]).sum()
+    assert abs(got - want) < 0.05 * want   # MC standard error ~ sqrt(2 / M) ~ 2 %
+
+
+def test_staleness_special_cases():
+    q, k, v, z = _stale_case(32)
+    N = k.shape[2]
+    assert O.staleness_iso(q, k, v, np.ones(N), z, 1.0) == 0.0          # everything refreshed
+    e1 = O.staleness_iso(q, k, v, np.zeros(N), z, 1.0)
+    np.testing.assert_allclose(O.staleness_iso(q, k, v, np.zeros(N), z, 3.0), 9.0 * e1, rtol=1e-13)
+    # one key, one head, one row: alpha = 1, so E = kappa^2 ||V||^2 / d * mean_m ||z_m||^2
+    q1, k1, v1 = q[:1, :1, :1], k[:1, :1, :1], v[:1, :1, :1]
+    z1 = z[:, :1, :1, :1]
+    d = q.shape[-1]
+    want = 4.0 * (v1[0, 0, 0] ** 2).sum() / d * (z1[:, 0, 0, 0] ** 2).sum(axis=1).mean()
+    np.testing.assert_allclose(O.staleness_iso(q1, k1, v1, np.zeros(1), z1, 2.0), want, rtol=1e-13)
+    # refreshing more tokens never raises the error for the same draws when the
+    # displacement directions are orthogonal across tokens (one-hot z)
+    hkv, Nn, dd = k.shape[1], k.shape[2], k.shape[3]
+    zo = np.zeros((1, q.shape[0], hkv, Nn, Nn))
+    for t in range(Nn):
+        zo[0, :, :, t, t] = 1.0
+    qo = np.random.default_rng(33).standard_normal(q.shape[:3] + (Nn,))
+    ko = np.random.default_rng(34).standard_normal(k.shape[:3] + (Nn,))
+    vo = np.random.default_rng(35).standard_normal(k.shape[:3] + (Nn,))
+    T1 = np.zeros(Nn); T1[[2, 3]] = 1
+    T2 = T1.copy(); T2[[10, 11, 12]] = 1
+    assert O.staleness_iso(qo, ko, vo, T2, zo, 1.0) <= O.staleness_iso(qo, ko, vo, T1, zo, 1.0)
+
+
 # --------------------------------------------------------- refresh step
 def test_gather_scatter_roundtrip():
     rng = np.random.default_rng(15)
