@@ -549,6 +549,83 @@ def run_reference(args):
     print(json.dumps(out), flush=True)
 
 
+# ------------------------------------------- staleness diagnostic (App. D)
+def run_staleness(args):
+    """The cross-image diagnostic of App. D.3 on a synthetic workload: the
+    isotropic Monte Carlo staleness E_iso(T) of the refresh sets of Conduit's
+    global rule, the explicit per-image quotas, the global rule without image
+    reweighting (lambda = 0) and a uniform random set of the same budgets,
+    all under the same draws (M = 5); printed as E / E_uniform with the
+    device time of one estimator call and its tensor roofline."""
+    world, rank, local = dist_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    from paper_2609_05821_gb300 import conduit as C
+    from paper_2609_05821_gb300 import pipeline, synth
+    w = synth.workload(args.config)
+    inputs = synth.make_inputs(w, device=dev)
+    _with_ratio(inputs, args.ratio)
+    M, kappa = 5, 0.5
+    L, Hkv, n_tot, d = inputs["k"].shape
+    gen = torch.Generator().manual_seed(w.seed + 101)
+    z = torch.randn((M, L, Hkv, n_tot, d), generator=gen).to(inputs["k"].dtype).to(dev)
+    masks = {}
+    for name, kw in (("conduit", {}), ("explicit_quota", {"selection": "quota"}),
+                     ("global_no_reweight", {"lam": 0.0})):
+        pipe = pipeline.from_inputs(inputs, **kw)
+        pipe.score_select()
+        masks[name] = pipe.mask.clone()
+    tok = inputs["tok_off"].tolist()
+    rng = torch.Generator().manual_seed(w.seed + 202)
+    uni = torch.zeros(n_tot, dtype=torch.uint8)
+    for r in range(len(tok) - 1):
+        n_r = tok[r + 1] - tok[r]
+        k_r = int(masks["conduit"][tok[r]:tok[r + 1]].sum().item())
+        uni[tok[r] + torch.randperm(n_r, generator=rng)[:k_r]] = 1
+    masks["uniform"] = uni.to(dev)
+    ws = torch.empty(C.conduit_staleness_iso_workspace_size(pipe.kv, pipe.batch, M), dtype=torch.uint8,
+                     device=dev)
+    err = torch.empty(pipe.batch.num_requests, dtype=torch.float64, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    call = lambda m: C.conduit_staleness_iso(pipe.kv, pipe.batch, pipe.q, m, z, kappa, err=err,
+                                             workspace=ws, status=status)
+    results = {}
+    for name, m in masks.items():
+        call(m)
+        results[name] = err.sum().item()
+    flush_buf = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    for _ in range(args.warmup):
+        call(masks["conduit"])
+    torch.cuda.synchronize()
+    launches0 = C.conduit_launch_count()
+    ms = time_steps(lambda: call(masks["conduit"]), args.steps, lambda: flush_buf.zero_())
+    launches = (C.conduit_launch_count() - launches0) // max(args.steps, 1)
+    mean_ms = sum(ms) / len(ms)
+    qo = inputs["q_off"].tolist()
+    flops = M * sum(4 * w.num_q_heads * d * (tok[r + 1] - tok[r]) * (qo[r + 1] - qo[r]) * L
+                    for r in range(len(tok) - 1))
+    hbm, tc, _, peak_src = _peaks()
+    achieved = flops / (mean_ms / 1e3) / 1e12
+    out = {
+        "metric": "isotropic staleness evaluations/s (App. D, M = 5 draws)",
+        "value": round(1e3 / mean_ms, 3), "unit": "evaluations/s", "n_gpus": 1, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(mean_ms, 4), "higher_is_better": True,
+        "dtype": "bf16" if inputs["k"].dtype == torch.bfloat16 else "f32",
+        "data": "synthetic (seeded; shapes and value laws of the paper's workloads; seeded draws)",
+        "config": {"workload": DESCR[args.config], "name": args.config, "M": M, "kappa": kappa,
+                   "l2": f"flushed between timed calls ({L2_FLUSH_BYTES >> 20} MB write)"},
+        "E_over_E_uniform": {k: round(v / results["uniform"], 4) for k, v in results.items()},
+        "E": {k: v for k, v in results.items()},
+        "roofline": {"bound": "tensor", "achieved": round(achieved, 3), "peak": round(tc, 1),
+                     "unit": "TFLOP/s", "frac": round(achieved / tc, 4), "traffic": None,
+                     "kernel": "staleness (refresh attention over the draws)",
+                     "peak_source": f"bf16 dense burst, {peak_src}"},
+        "gpu_launches": launches * args.steps,
+        "status": C.conduit_read_status(status),
+    }
+    print(json.dumps(out), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -569,8 +646,12 @@ def main():
                     help="softmax denominators include outside keys (seeded log-sum-exps)")
     ap.add_argument("--ratio", type=float, default=None,
                     help="refresh ratio r for every request (default: the workload's own)")
+    ap.add_argument("--diagnostic", default=None, choices=["staleness"],
+                    help="run the App. D staleness diagnostic instead of the step")
     args = ap.parse_args()
-    if args.impl == "reference":
+    if args.diagnostic == "staleness":
+        run_staleness(args)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_conduit(args)

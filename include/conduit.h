@@ -375,6 +375,35 @@ conduit_status conduit_refresh_attn(const conduit_kv* kv, const conduit_batch* b
                                     void* stream);
 
 /*
+ * Isotropic Monte Carlo staleness estimator (App. D): the residual error a
+ * refresh set T leaves under sampled stale value displacements, per request
+ *   E_r = sum_{l, h, q in Q_r} (1/M) sum_m || sum_{t not in T} alpha_{q,t} xi_t^(m) ||^2
+ *   xi_{l,g,t}^(m) = kappa ||V_{l,g,t}|| / sqrt(d) z_{l,g,t}^(m)
+ * with alpha the cached-key softmax over the request's N_r visual keys (Eq. 6's
+ * alpha), query head h reading KV head h / G, ||V_{l,g,t}|| that head's value
+ * norm and z standard normal draws. Comparing E for the sets of different
+ * selection rules (and a uniform random set) under the same z is the
+ * cross-image diagnostic of App. D.3.
+ *  q          device [L][Hq][Q_tot][d], dtype of kv (the scoring queries)
+ *  refreshed  device uint8 [N_tot], 1 = token in T (e.g. conduit_select_topk's mask)
+ *  z          device [M][L][Hkv][N_tot][d], dtype of kv (the random draws; the
+ *             caller generates them)
+ *  M >= 1, kappa >= 0
+ *  err        device double [R] E_r (written)
+ *  err_layers device double [R][L] the per-layer terms of E_r, or NULL
+ *  workspace  conduit_staleness_iso_workspace_size bytes (it holds one draw of
+ *             xi in the cache's layout and the per-draw attention outputs)
+ * Attention runs with the refresh kernels (bf16 P and outputs for bf16
+ * caches); the reduction of ||O||^2 is in a fixed order.
+ */
+conduit_status conduit_staleness_iso_workspace_size(const conduit_kv* kv, const conduit_batch* batch,
+                                                   int32_t M, size_t* bytes);
+conduit_status conduit_staleness_iso(const conduit_kv* kv, const conduit_batch* batch, const void* q,
+                                     const uint8_t* refreshed, const void* z, int32_t M, float kappa,
+                                     double* err, double* err_layers, void* workspace,
+                                     size_t workspace_bytes, int32_t* status, void* stream);
+
+/*
  * Number of kernels this library has enqueued in this process (launched, or
  * recorded into a stream capture) since it was loaded. Diagnostic only.
  */

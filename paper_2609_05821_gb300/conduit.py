@@ -80,6 +80,8 @@ def _load():
         "conduit_score": (st, [P, P, P, P, I32, P, P, P, P, SZ, P, P]),
         "conduit_score_ex_workspace_size": (st, [P, P, I32, P, ctypes.POINTER(SZ)]),
         "conduit_score_ex": (st, [P, P, P, P, I32, P, P, P, P, P, SZ, P, P]),
+        "conduit_staleness_iso_workspace_size": (st, [P, P, I32, ctypes.POINTER(SZ)]),
+        "conduit_staleness_iso": (st, [P, P, P, P, P, I32, ctypes.c_float, P, P, P, SZ, P, P]),
         "conduit_value_norms": (st, [P, P, P, P]),
         "conduit_value_norms_update": (st, [P, P, P, P, P, P, P]),
         "conduit_score_with_norms_workspace_size": (st, [P, P, I32, ctypes.POINTER(SZ)]),
@@ -282,6 +284,27 @@ def conduit_score_ex(kv: KvCache, batch: Batch, q: torch.Tensor, layers=None, st
                                  _ptr(s), _ptr(attn_sum), _ptr(g), _ptr(ws), ws.numel(),
                                  _ptr(status), _stream_ptr(stream)))
     return s, attn_sum, g
+
+
+def conduit_staleness_iso_workspace_size(kv: KvCache, batch: Batch, M: int) -> int:
+    n = ctypes.c_size_t(0)
+    _check(_lib.conduit_staleness_iso_workspace_size(kv.ref(), batch.ref(), int(M), ctypes.byref(n)))
+    return int(n.value)
+
+
+def conduit_staleness_iso(kv: KvCache, batch: Batch, q: torch.Tensor, refreshed: torch.Tensor,
+                          z: torch.Tensor, kappa: float, err=None, err_layers=None, workspace=None,
+                          status=None, stream=None):
+    """Isotropic Monte Carlo staleness of a refresh set (App. D). z: [M][L][Hkv][N_tot][d].
+    Returns (err [R], err_layers [R, L] or None), float64."""
+    dev = kv.k.device
+    M = int(z.shape[0])
+    err = torch.empty(batch.num_requests, dtype=torch.float64, device=dev) if err is None else err
+    ws = _workspace(conduit_staleness_iso_workspace_size(kv, batch, M), dev, workspace)
+    _check(_lib.conduit_staleness_iso(kv.ref(), batch.ref(), _ptr(q), _ptr(refreshed), _ptr(z), M,
+                                      float(kappa), _ptr(err), _ptr(err_layers), _ptr(ws), ws.numel(),
+                                      _ptr(status), _stream_ptr(stream)))
+    return err, err_layers
 
 
 def conduit_value_norms(kv: KvCache, batch: Batch, vnorm=None, stream=None) -> torch.Tensor:

@@ -591,6 +591,39 @@ conduit_status conduit_refresh_attn(const conduit_kv* kv, const conduit_batch* b
   return CONDUIT_OK;
 }
 
+conduit_status conduit_staleness_iso_workspace_size(const conduit_kv* kv, const conduit_batch* batch,
+                                                   int32_t M, size_t* bytes) {
+  conduit_status st;
+  if (!bytes) return fail(CONDUIT_ERR_INVALID_ARG, "bytes is NULL");
+  if ((st = check_batch(batch)) || (st = check_kv(kv, batch))) return st;
+  if (M < 1) return fail(CONDUIT_ERR_INVALID_ARG, "M must be >= 1");
+  *bytes = stale_layout(make_kv(kv, batch), make_batch(batch), batch->q_off[batch->num_requests], M).total;
+  return CONDUIT_OK;
+}
+
+conduit_status conduit_staleness_iso(const conduit_kv* kv, const conduit_batch* batch, const void* q,
+                                     const uint8_t* refreshed, const void* z, int32_t M, float kappa,
+                                     double* err, double* err_layers, void* workspace,
+                                     size_t workspace_bytes, int32_t* status, void* stream) {
+  conduit_status st;
+  if ((st = check_batch(batch)) || (st = check_kv(kv, batch))) return st;
+  if (!q || !refreshed || !z || !err)
+    return fail(CONDUIT_ERR_INVALID_ARG, "q, refreshed, z and err are required");
+  if (!aligned16(q) || !aligned16(z)) return fail(CONDUIT_ERR_INVALID_ARG, "q and z must be 16-byte aligned");
+  if (M < 1) return fail(CONDUIT_ERR_INVALID_ARG, "M must be >= 1");
+  if (!(kappa >= 0.f) || !std::isfinite(kappa))
+    return fail(CONDUIT_ERR_INVALID_ARG, "kappa must be finite and >= 0");
+  const KvDev kd = make_kv(kv, batch);
+  const BatchDev bd = make_batch(batch);
+  const int32_t q_tot = batch->q_off[batch->num_requests];
+  if ((st = check_workspace(workspace, workspace_bytes, stale_layout(kd, bd, q_tot, M).total))) return st;
+  cudaError_t err_c = launch_staleness_iso(kd, bd, batch->q_off, q_tot, q, refreshed, z, M, kappa, err,
+                                           err_layers, workspace, status,
+                                           static_cast<cudaStream_t>(stream));
+  if (err_c) return cuda_fail(err_c, "staleness_iso");
+  return CONDUIT_OK;
+}
+
 conduit_status conduit_clear_status(int32_t* status, void* stream) {
   if (!status) return fail(CONDUIT_ERR_INVALID_ARG, "status is NULL");
   cudaError_t err = cudaMemsetAsync(status, 0, sizeof(int32_t), static_cast<cudaStream_t>(stream));

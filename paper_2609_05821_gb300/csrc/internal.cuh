@@ -164,6 +164,17 @@ cudaError_t launch_finalize(const float* pa, const float* pa2, const float* ss, 
 cudaError_t launch_value_norms(const KvDev& kv, const BatchDev& b, const int32_t* idx,
                                const int32_t* idx_off_dev, int64_t n_rows, float* vnorm,
                                cudaStream_t stream);
+// Isotropic Monte Carlo staleness estimator (App. D): workspace carving and
+// the launcher (M draws of refresh attention over (K, xi^(m)), then ||O||^2).
+struct StaleLayout {
+  size_t xi, rows, out, pos, part, counter, total;
+  size_t xi_bytes;
+};
+StaleLayout stale_layout(const KvDev& kv, const BatchDev& b, int32_t q_tot, int M);
+cudaError_t launch_staleness_iso(const KvDev& kv, const BatchDev& b, const int32_t* q_off_host,
+                                 int32_t q_tot, const void* q, const uint8_t* refreshed,
+                                 const void* z, int M, float kappa, double* err, double* err_rl,
+                                 void* workspace, int32_t* status, cudaStream_t stream);
 // max_tokens: the largest request (picks how many keys a thread keeps in registers).
 cudaError_t launch_select(const BatchDev& b, int max_tokens, const float* s, const float* g,
                           float lambda, const int32_t* idx_off_dev, int32_t* idx, uint8_t* mask,

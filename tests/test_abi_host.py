@@ -37,7 +37,8 @@ def test_header_declares_the_boundary():
                  "conduit_read_status", "conduit_value_norms", "conduit_value_norms_update",
                  "conduit_score_with_norms", "conduit_score_with_norms_workspace_size",
                  "conduit_score_ex", "conduit_score_ex_workspace_size",
-                 "conduit_select_quota", "conduit_select_quota_workspace_size"):
+                 "conduit_select_quota", "conduit_select_quota_workspace_size",
+                 "conduit_staleness_iso", "conduit_staleness_iso_workspace_size"):
         assert want in names
 
 
@@ -149,6 +150,33 @@ def test_quota_select_rejects_bad_arguments(C):
     ws = torch.zeros(need - 256, dtype=torch.uint8)
     _expect(C, C.ERR_WORKSPACE, C.conduit_select_quota, b, s, g, 1.0, off, off_d, None, None, None,
             None, None, ws)
+
+
+def test_staleness_rejects_bad_arguments(C):
+    kv, b = _kv(C), _batch(C)
+    lib = C._lib
+    q = torch.zeros((2, 4, 8, 64), dtype=torch.bfloat16)
+    mask = torch.zeros(128, dtype=torch.uint8)
+    z = torch.zeros((2, 2, 2, 128, 64), dtype=torch.bfloat16)
+    err = torch.zeros(2, dtype=torch.float64)
+    n = ctypes.c_size_t(0)
+    assert lib.conduit_staleness_iso_workspace_size(kv.ref(), b.ref(), 0, ctypes.byref(n)) == C.ERR_INVALID_ARG
+    assert lib.conduit_staleness_iso_workspace_size(kv.ref(), b.ref(), 2, ctypes.byref(n)) == C.OK
+    need = n.value
+    assert need > 0
+
+    def call(mq=q, mz=z, M=2, kappa=1.0, ws_bytes=need):
+        ws = torch.zeros(max(ws_bytes, 1), dtype=torch.uint8)
+        return lib.conduit_staleness_iso(kv.ref(), b.ref(), C._ptr(mq), C._ptr(mask), C._ptr(mz), M, kappa,
+                                         C._ptr(err), None, C._ptr(ws) if ws_bytes else None, ws_bytes,
+                                         None, None)
+
+    assert call(mz=None) == C.ERR_INVALID_ARG
+    assert call(M=0) == C.ERR_INVALID_ARG
+    assert call(kappa=-1.0) == C.ERR_INVALID_ARG
+    assert call(kappa=float("nan")) == C.ERR_INVALID_ARG
+    assert call(ws_bytes=0) == C.ERR_WORKSPACE
+    assert call(ws_bytes=need - 256) == C.ERR_WORKSPACE
 
 
 def test_kv_copy_and_refresh_reject_bad_arguments(C):
