@@ -167,7 +167,7 @@ cudaError_t launch_value_norms(const KvDev& kv, const BatchDev& b, const int32_t
 // Isotropic Monte Carlo staleness estimator (App. D): workspace carving and
 // the launcher (M draws of refresh attention over (K, xi^(m)), then ||O||^2).
 struct StaleLayout {
-  size_t xi, rows, out, pos, part, counter, total;
+  size_t xi, rows, out, pos, part, scale, counter, total;
   size_t xi_bytes;
 };
 StaleLayout stale_layout(const KvDev& kv, const BatchDev& b, int32_t q_tot, int M);

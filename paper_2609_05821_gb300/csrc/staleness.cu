@@ -12,27 +12,43 @@
 namespace conduit {
 namespace {
 
-// xi^(m) rows in the layout of kv.v (contiguous or paged): one warp per
-// (layer, KV head, token) row.
+// Per (layer, KV head, token) row: the standard deviation of its draws,
+// kappa ||V|| / sqrt(d), or 0 when the token is refreshed (the same for every
+// draw, so computed once). One warp per row.
 template <typename T>
-__global__ void __launch_bounds__(256) stale_values_kernel(KvDev kv, BatchDev b,
-                                                           const uint8_t* refreshed, const T* z,
-                                                           float kappa, T* xi) {
+__global__ void __launch_bounds__(256) stale_scale_kernel(KvDev kv, BatchDev b,
+                                                          const uint8_t* refreshed, float kappa,
+                                                          float* scale) {
   const int64_t row = int64_t(blockIdx.x) * 8 + threadIdx.x / 32;
   const int lane = threadIdx.x % 32;
   const int64_t rows = int64_t(kv.L) * kv.Hkv * kv.n_tot;
   if (row >= rows) return;
   const int64_t tg = row % kv.n_tot;
   const int lg = int(row / kv.n_tot);
-  const int l = lg / kv.Hkv, g = lg % kv.Hkv;
   const int r = request_of(b.tok_off, b.R, tg);
   const int t = int(tg - b.tok_off[r]);
-  const int64_t off = kv.row(l, g, r, tg, t);
   const T* vb = static_cast<const T*>(kv.v);
-  const float ss = warp_row_sumsq(vb + off, kv.d, lane);
-  const float scale = refreshed[tg] ? 0.f : kappa * sqrtf(ss / float(kv.d));
+  const float ss = warp_row_sumsq(vb + kv.row(lg / kv.Hkv, lg % kv.Hkv, r, tg, t), kv.d, lane);
+  if (lane == 0) scale[row] = refreshed[tg] ? 0.f : kappa * sqrtf(ss / float(kv.d));
+}
+
+// xi^(m) rows in the layout of kv.v (contiguous or paged): one warp per
+// (layer, KV head, token) row, xi = scale * z.
+template <typename T>
+__global__ void __launch_bounds__(256) stale_values_kernel(KvDev kv, BatchDev b, const float* scale,
+                                                           const T* z, T* xi) {
+  const int64_t row = int64_t(blockIdx.x) * 8 + threadIdx.x / 32;
+  const int lane = threadIdx.x % 32;
+  const int64_t rows = int64_t(kv.L) * kv.Hkv * kv.n_tot;
+  if (row >= rows) return;
+  const int64_t tg = row % kv.n_tot;
+  const int lg = int(row / kv.n_tot);
+  const int r = request_of(b.tok_off, b.R, tg);
+  const int t = int(tg - b.tok_off[r]);
+  const int64_t off = kv.row(lg / kv.Hkv, lg % kv.Hkv, r, tg, t);
+  const float sc = scale[row];
   const T* zr = z + row * kv.d;  // z is [L][Hkv][N_tot][d]
-  for (int e = lane; e < kv.d; e += 32) xi[off + e] = from_float<T>(scale * to_float(zr[e]));
+  for (int e = lane; e < kv.d; e += 32) xi[off + e] = from_float<T>(sc * to_float(zr[e]));
 }
 
 // q [L][Hq][Q_tot][d] -> rows [L][Q_tot][Hq][d] (the refresh kernels' row layout).
@@ -121,6 +137,8 @@ StaleLayout stale_layout(const KvDev& kv, const BatchDev& b, int32_t q_tot, int 
   off += up(size_t(q_tot) * 4);
   s.part = off;
   off += up(size_t(b.R) * kv.L * 8);
+  s.scale = off;
+  off += up(size_t(kv.L) * kv.Hkv * size_t(kv.n_tot) * 4);
   s.counter = off;
   off += 256;
   s.total = off;
@@ -138,9 +156,9 @@ cudaError_t launch_staleness_iso(const KvDev& kv, const BatchDev& b, const int32
   void* out = ws + lay.out;
   int32_t* pos = reinterpret_cast<int32_t*>(ws + lay.pos);
   double* part = reinterpret_cast<double*>(ws + lay.part);
+  float* scale = reinterpret_cast<float*>(ws + lay.scale);
   int32_t* counter = reinterpret_cast<int32_t*>(ws + lay.counter);
   const bool bf16 = kv.dtype == CONDUIT_BF16;
-  const size_t esz = bf16 ? 2 : 4;
   cudaError_t err_c;
   // pool rows that hold no token (a partial last page) stay zero for every draw
   if ((err_c = cudaMemsetAsync(xi, 0, lay.xi_bytes, stream))) return err_c;
@@ -162,16 +180,22 @@ cudaError_t launch_staleness_iso(const KvDev& kv, const BatchDev& b, const int32
   kx.v = xi;
   const int64_t vrows = int64_t(kv.L) * kv.Hkv * kv.n_tot;
   const int64_t zdraw = vrows * kv.d;  // elements of one draw
+  const unsigned vblocks = unsigned((vrows + 7) / 8);
+  if (vrows > 0) {
+    if (bf16)
+      stale_scale_kernel<__nv_bfloat16><<<vblocks, 256, 0, stream>>>(kv, b, refreshed, kappa, scale);
+    else
+      stale_scale_kernel<float><<<vblocks, 256, 0, stream>>>(kv, b, refreshed, kappa, scale);
+    count_launches(1);
+    if ((err_c = cudaGetLastError())) return err_c;
+  }
   for (int m = 0; m < M; ++m) {
-    const unsigned vblocks = unsigned((vrows + 7) / 8);
     if (bf16)
       stale_values_kernel<__nv_bfloat16><<<vblocks, 256, 0, stream>>>(
-          kv, b, refreshed, static_cast<const __nv_bfloat16*>(z) + m * zdraw, kappa,
-          static_cast<__nv_bfloat16*>(xi));
+          kv, b, scale, static_cast<const __nv_bfloat16*>(z) + m * zdraw, static_cast<__nv_bfloat16*>(xi));
     else
-      stale_values_kernel<float><<<vblocks, 256, 0, stream>>>(kv, b, refreshed,
-                                                              static_cast<const float*>(z) + m * zdraw,
-                                                              kappa, static_cast<float*>(xi));
+      stale_values_kernel<float><<<vblocks, 256, 0, stream>>>(
+          kv, b, scale, static_cast<const float*>(z) + m * zdraw, static_cast<float*>(xi));
     count_launches(1);
     if ((err_c = cudaGetLastError())) return err_c;
     if (q_tot > 0) {
@@ -191,7 +215,6 @@ cudaError_t launch_staleness_iso(const KvDev& kv, const BatchDev& b, const int32
       if ((err_c = cudaGetLastError())) return err_c;
     }
   }
-  (void)esz;
   stale_final_kernel<<<(b.R + 127) / 128, 128, 0, stream>>>(part, b.R, kv.L, M, err, err_rl);
   count_launches(1);
   return cudaGetLastError();

@@ -40,6 +40,7 @@ class RefreshPipeline:
         dev = k.device
         self.device = dev
         self.kv = C.KvCache(k, v, num_q_heads, page_size, page_table)
+        self._page_size = page_size
         self.batch = C.Batch(tok_off, img_off, req_img_off, q_off, device=dev)
         self.q = q
         self.lam = float(lam)
@@ -86,6 +87,8 @@ class RefreshPipeline:
         self.v_old = torch.empty_like(self.k_old)
         self.out = torch.empty_like(self.q_rows)
         self.graph = None
+        self._copy = None  # copy stream and events of step_from_host
+        self._out_graph = None  # refresh with the output copied out per layer chunk (step_from_host)
 
     # ----------------------------------------------------------------- steps
     def score(self, stream=None):
@@ -129,16 +132,31 @@ class RefreshPipeline:
         self.norm_update(stream)
         self.refresh_attn(stream)
 
+    def _score_select_step(self):
+        if self.graph is not None:
+            self.graph[0].replay()
+        else:
+            self.score_select()
+
+    def _refresh_step(self):
+        if self.graph is not None:
+            self.graph[1].replay()
+        else:
+            self.refresh()
+
     def step(self, stream=None):
         """One pass of the whole hot path (launches only; asynchronous)."""
         if self.graph is not None:
-            self.graph.replay()
+            self._score_select_step()
+            self._refresh_step()
             return
         self.score_select(stream)
         self.refresh(stream)
 
     def capture(self):
-        """Capture one step in a CUDA graph; later step() calls replay it."""
+        """Capture the step as two CUDA graphs (scoring and selection; exchange
+        and refresh), so that step_from_host can start the first while the
+        second's inputs are still arriving; later step() calls replay them."""
         s = torch.cuda.Stream(device=self.device)
         s.wait_stream(torch.cuda.current_stream())
         with torch.cuda.stream(s):
@@ -146,11 +164,12 @@ class RefreshPipeline:
             self.refresh(s)
         torch.cuda.current_stream().wait_stream(s)
         torch.cuda.synchronize()
-        g = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g):
+        g1, g2 = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g1):
             self.score_select()
+        with torch.cuda.graph(g2):
             self.refresh()
-        self.graph = g
+        self.graph = (g1, g2)
 
     # ------------------------------------------------------------- end to end
     def host_buffers(self) -> dict:
@@ -164,13 +183,68 @@ class RefreshPipeline:
         }
 
     def step_from_host(self, host: dict):
-        """H2D copy of the cache, queries and fresh rows; the step; D2H of idx and out."""
-        for name, dst in (("k", self.kv.k), ("v", self.kv.v), ("q", self.q),
-                          ("q_rows", self.q_rows), ("k_rows", self.k_rows), ("v_rows", self.v_rows)):
-            dst.copy_(host[name], non_blocking=True)
-        self.step()
+        """H2D copy of the cache, queries and fresh rows; the step; D2H of idx and out.
+
+        The copies run on a stream of their own: the scoring pass starts once
+        the cache and the queries have arrived, while the fresh rows (needed
+        only by the exchange and the refresh) are still being copied; the
+        refresh runs in layer chunks, each chunk's output copied back while
+        the next chunks compute.
+        """
+        cs = torch.cuda.current_stream(self.device)
+        if self._copy is None:
+            self._copy = (torch.cuda.Stream(device=self.device), torch.cuda.Event(), torch.cuda.Event())
+        xs, ev_in, ev_fresh = self._copy
+        xs.wait_stream(cs)  # the device buffers are free once the previous step is done
+        with torch.cuda.stream(xs):
+            for name, dst in (("k", self.kv.k), ("v", self.kv.v), ("q", self.q)):
+                dst.copy_(host[name], non_blocking=True)
+            ev_in.record(xs)
+            for name, dst in (("q_rows", self.q_rows), ("k_rows", self.k_rows), ("v_rows", self.v_rows)):
+                dst.copy_(host[name], non_blocking=True)
+            ev_fresh.record(xs)
+        cs.wait_event(ev_in)
+        self._score_select_step()
         host["idx"].copy_(self.idx, non_blocking=True)
-        host["out"].copy_(self.out, non_blocking=True)
+        cs.wait_event(ev_fresh)
+        self._refresh_to_host(host["out"])
+
+    def _refresh_chunks(self, host_out, side):
+        """Exchange, then the refresh attention layer chunk by layer chunk, each
+        chunk's output copied to host_out on `side` while later chunks run."""
+        cs = torch.cuda.current_stream(self.device)
+        self.exchange()
+        self.norm_update()
+        for view, (l0, l1) in self._chunk_views:
+            C.conduit_refresh_attn(view, self.batch, self.idx, self.idx_off, self.idx_off_dev,
+                                   self.q_rows[l0:l1], self.out[l0:l1], self.ws_ref, self.status)
+            side.wait_stream(cs)
+            with torch.cuda.stream(side):
+                host_out[l0:l1].copy_(self.out[l0:l1], non_blocking=True)
+        cs.wait_stream(side)
+
+    def _refresh_to_host(self, host_out, chunks: int = 4):
+        if self._out_graph is None or self._out_graph[1] is not host_out:
+            L = self.kv.num_layers
+            bounds = sorted({round(i * L / chunks) for i in range(chunks + 1)})
+            kv = self.kv
+            self._chunk_views = [
+                (C.KvCache(kv.k[l0:l1], kv.v[l0:l1], kv.num_q_heads, self._page_size, kv.page_table),
+                 (l0, l1))
+                for l0, l1 in zip(bounds[:-1], bounds[1:])]
+            side = torch.cuda.Stream(device=self.device)
+            if self.graph is None:
+                self._out_graph = (None, host_out, side)
+            else:
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g):
+                    self._refresh_chunks(host_out, side)
+                self._out_graph = (g, host_out, side)
+        g, _, side = self._out_graph
+        if g is not None:
+            g.replay()
+        else:
+            self._refresh_chunks(host_out, side)
 
     def h2d_bytes(self) -> int:
         ts = (self.kv.k, self.kv.v, self.q, self.q_rows, self.k_rows, self.v_rows)

@@ -347,3 +347,19 @@ def test_nonfinite_input_sets_status_word(C, P):
     assert C.conduit_read_status(pipe.status) == C.ERR_NONFINITE
     C.conduit_clear_status(pipe.status)
     assert C.conduit_read_status(pipe.status) == C.OK
+
+
+def test_step_from_host_equals_step(C, P):
+    """The end-to-end form (host copies on their own stream, the step as two
+    graphs) gives bitwise the selection and output of the plain step."""
+    inputs = _small_multi(num_layers=3)
+    a = P.from_inputs({**inputs, "k": inputs["k"].clone(), "v": inputs["v"].clone()})
+    b = P.from_inputs({**inputs, "k": inputs["k"].clone(), "v": inputs["v"].clone()})
+    host = a.host_buffers()          # the cache before any step
+    a.capture()                      # the capture runs one step on a's buffers
+    a.step_from_host(host)           # the copies restore them first
+    b.step()
+    torch.cuda.synchronize()
+    assert torch.equal(host["idx"].cuda(), b.idx)
+    assert torch.equal(host["out"].cuda(), b.out)
+    assert torch.equal(a.kv.k, b.kv.k) and torch.equal(a.kv.v, b.kv.v)
