@@ -363,3 +363,36 @@ def test_step_from_host_equals_step(C, P):
     assert torch.equal(host["idx"].cuda(), b.idx)
     assert torch.equal(host["out"].cuda(), b.out)
     assert torch.equal(a.kv.k, b.kv.k) and torch.equal(a.kv.v, b.kv.v)
+
+
+@pytest.mark.parametrize("page_size,tokens_per_image", [(8, 208), (32, 208), (64, 224), (128, 192)])
+def test_paged_caches_of_every_page_size_equal_contiguous(C, P, page_size, tokens_per_image):
+    """Scoring, selection, exchange and refresh over a paged cache (pages in a
+    seeded shuffled pool order) give bitwise the results of the contiguous
+    cache, for every page size the tensor-core kernels take (one TMA copy per
+    page half: 32 copies per tile at page size 8). Requests of 416 and 448
+    tokens end in a ragged key tile."""
+    w = synth.workload("multi", num_layers=2, images_per_request=2, tokens_per_image=tokens_per_image,
+                       num_requests=3, n_q=None, n_q_lo=5, n_q_hi=40, page_size=page_size)
+    inputs = synth.make_inputs(w, device="cuda")
+    paged = _run(P, inputs, paged=True)
+    flat = _run(P, inputs, paged=False)
+    assert paged.kv.k.dim() == 5 and paged.kv.k.shape[3] == page_size
+    for name in ("s", "attn_sum", "g", "coeff", "s_hat", "idx", "mask", "k_old", "v_old", "out"):
+        assert torch.equal(getattr(paged, name), getattr(flat, name)), name
+
+
+def test_tensor_core_refresh_mixed_budgets(C, P):
+    """One launch of the tensor-core path over requests with budgets 0, N_r,
+    1 and 17: items of a single row, whole requests and empty requests share
+    the persistent grid and its work counter."""
+    w = synth.workload("multi", num_layers=2, images_per_request=2, tokens_per_image=128, num_requests=4,
+                       n_q=None, n_q_lo=3, n_q_hi=30)
+    inputs = synth.make_inputs(w, device="cuda")
+    budgets = [0, 256, 1, 17]
+    pipe = _run(P, inputs, budgets=budgets)
+    ref = _oracle(inputs, budgets=budgets)
+    PT.compare_score_select(pipe, inputs, ref, PT.RTOL[torch.bfloat16])
+    _check_refresh(pipe, inputs, ref, None)
+    _patched_equals_scatter(C, pipe, inputs)
+    assert C.conduit_read_status(pipe.status) == C.OK
