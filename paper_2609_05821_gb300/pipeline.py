@@ -17,7 +17,9 @@ bitwise those of the pass that reads V.
 All buffers are allocated once at construction, so a step allocates nothing
 and can be captured in a CUDA graph (``capture()``). ``step_from_host()`` is
 the end-to-end form: it copies the step's inputs from pinned host memory,
-runs the step, and copies the selection and the refresh output back.
+runs the step, and copies the selection and the refresh output back;
+``DoubleBuffered`` alternates two pipelines so that one step's copies overlap
+the previous step's kernels.
 """
 
 from __future__ import annotations
@@ -182,20 +184,26 @@ class RefreshPipeline:
             "out": torch.empty(self.out.shape, dtype=self.out.dtype, pin_memory=True),
         }
 
-    def step_from_host(self, host: dict):
+    def step_from_host(self, host: dict, after: Optional[torch.cuda.Event] = None):
         """H2D copy of the cache, queries and fresh rows; the step; D2H of idx and out.
 
         The copies run on a stream of their own: the scoring pass starts once
         the cache and the queries have arrived, while the fresh rows (needed
         only by the exchange and the refresh) are still being copied; the
         refresh runs in layer chunks, each chunk's output copied back while
-        the next chunks compute.
+        the next chunks compute. The copies wait for everything enqueued on
+        the current stream before the call, or, given ``after``, for that
+        event only (the caller vouches that this pipeline's buffers are free
+        once it has fired; see ``DoubleBuffered``).
         """
         cs = torch.cuda.current_stream(self.device)
         if self._copy is None:
             self._copy = (torch.cuda.Stream(device=self.device), torch.cuda.Event(), torch.cuda.Event())
         xs, ev_in, ev_fresh = self._copy
-        xs.wait_stream(cs)  # the device buffers are free once the previous step is done
+        if after is None:
+            xs.wait_stream(cs)  # the device buffers are free once the previous step is done
+        else:
+            xs.wait_event(after)
         with torch.cuda.stream(xs):
             for name, dst in (("k", self.kv.k), ("v", self.kv.v), ("q", self.q)):
                 dst.copy_(host[name], non_blocking=True)
@@ -252,6 +260,46 @@ class RefreshPipeline:
 
     def d2h_bytes(self) -> int:
         return self.idx.numel() * 4 + self.out.numel() * self.out.element_size()
+
+
+class DoubleBuffered:
+    """Two pipelines of one batch shape, stepped alternately from host buffers.
+
+    A step's host-to-device copies wait only for the previous step on the
+    same pipeline, so they run while the other pipeline's step computes, and
+    back-to-back steps are bound by the host link instead of by copies and
+    kernels in series. Both pipelines' kernels run on the current stream, in
+    call order, and each step's device-to-host copies complete before the
+    next step's kernels start.
+    """
+
+    def __init__(self, first: RefreshPipeline, second: RefreshPipeline):
+        if first.kv.k.shape != second.kv.k.shape or first.budgets != second.budgets:
+            raise ValueError("DoubleBuffered needs two pipelines of the same batch shape")
+        # a pipeline keeps the tensors it was built on; the copies of one step
+        # would overwrite what the other pipeline's step is reading
+        bufs = lambda p: {t.data_ptr() for t in (p.kv.k, p.kv.v, p.q, p.q_rows, p.k_rows, p.v_rows)}
+        if bufs(first) & bufs(second):
+            raise ValueError("DoubleBuffered needs two pipelines over separate device buffers")
+        self.pipes = (first, second)
+        self._done = [None, None]
+        self._next = 0
+
+    def start_after(self, event: torch.cuda.Event):
+        """Order the next copies of both pipelines after ``event`` (and after
+        every earlier step, which it must follow)."""
+        self._done = [event, event]
+
+    def step_from_host(self, host: dict) -> RefreshPipeline:
+        """One step on the next pipeline; returns the pipeline that ran it."""
+        i = self._next
+        p = self.pipes[i]
+        p.step_from_host(host, after=self._done[i])
+        ev = torch.cuda.Event()
+        ev.record(torch.cuda.current_stream(p.device))
+        self._done[i] = ev
+        self._next = i ^ 1
+        return p
 
 
 def from_inputs(inputs: dict, lam: float = 1.0, paged: Optional[bool] = None,

@@ -365,6 +365,62 @@ def test_step_from_host_equals_step(C, P):
     assert torch.equal(a.kv.k, b.kv.k) and torch.equal(a.kv.v, b.kv.v)
 
 
+def test_double_buffered_steps_equal_plain_steps(C, P):
+    """Two pipelines stepped alternately, back to back, from two different
+    host batches: every step's selection, output and patched cache are
+    bitwise those of a plain step on a fresh pipeline over that batch."""
+    from paper_2609_05821_gb300 import synth
+    w = synth.workload("multi", num_layers=3, tokens_per_image=128, images_per_request=4)
+    batches = [synth.make_inputs(w, device="cuda", seed=s) for s in (21, 22)]
+    fresh = [synth.make_fresh_rows(w, 51, device="cuda", seed=s) for s in (31, 32)]
+    own = lambda x: {n: t.clone() if torch.is_tensor(t) else t for n, t in x.items()}
+    # a pipeline keeps the tensors it is given (q, fresh rows), so each gets copies
+    pipes = [P.from_inputs(own(x), fresh=own(f), budgets=[51]) for x, f in zip(batches, fresh)]
+    hosts = [p.host_buffers() for p in pipes]  # each batch's cache before any step
+    for p in pipes:
+        p.capture()
+    stepper = P.DoubleBuffered(*pipes)
+    order = [0, 1, 0, 1, 1, 0]
+    outs = []
+    for j in order:
+        ran = stepper.step_from_host(hosts[j])
+        host_copy = {"idx": torch.empty_like(hosts[j]["idx"]), "out": torch.empty_like(hosts[j]["out"])}
+        torch.cuda.current_stream().synchronize()
+        host_copy["idx"].copy_(hosts[j]["idx"])
+        host_copy["out"].copy_(hosts[j]["out"])
+        outs.append((j, host_copy, ran.kv.k.clone(), ran.kv.v.clone()))
+    for j, got, k_now, v_now in outs:
+        ref = P.from_inputs(own(batches[j]), fresh=own(fresh[j]), budgets=[51])
+        ref.step()
+        torch.cuda.synchronize()
+        assert torch.equal(got["idx"].cuda(), ref.idx)
+        assert torch.equal(got["out"].cuda(), ref.out)
+        assert torch.equal(k_now, ref.kv.k) and torch.equal(v_now, ref.kv.v)
+
+
+def test_double_buffered_back_to_back_equals_plain(C, P):
+    """Back to back with no synchronisation between steps (each step's copies
+    overlapping the previous step's kernels), the last step's results are
+    bitwise those of a plain step."""
+    inputs = _small_multi(num_layers=3)
+    own = lambda x: {n: t.clone() if torch.is_tensor(t) else t for n, t in x.items()}
+    pipes = [P.from_inputs(own(inputs)) for _ in range(2)]
+    host = pipes[0].host_buffers()
+    for p in pipes:
+        p.capture()
+    stepper = P.DoubleBuffered(*pipes)
+    last = None
+    for _ in range(5):
+        last = stepper.step_from_host(host)
+    torch.cuda.synchronize()
+    ref = P.from_inputs(own(inputs))
+    ref.step()
+    torch.cuda.synchronize()
+    assert torch.equal(host["idx"].cuda(), ref.idx)
+    assert torch.equal(host["out"].cuda(), ref.out)
+    assert torch.equal(last.kv.k, ref.kv.k)
+
+
 @pytest.mark.parametrize("page_size,tokens_per_image", [(8, 208), (32, 208), (64, 224), (128, 192)])
 def test_paged_caches_of_every_page_size_equal_contiguous(C, P, page_size, tokens_per_image):
     """Scoring, selection, exchange and refresh over a paged cache (pages in a
