@@ -42,7 +42,7 @@ typedef int32_t conduit_status;
 enum {
   CONDUIT_OK = 0,
   CONDUIT_ERR_INVALID_ARG = 1, /* a pointer, size, span or budget is wrong */
-  CONDUIT_ERR_UNSUPPORTED = 2, /* valid, but a shape or dtype this build lacks */
+  CONDUIT_ERR_UNSUPPORTED = 2, /* valid, but a shape or dtype the library does not implement */
   CONDUIT_ERR_CUDA = 3,        /* a CUDA runtime call failed */
   CONDUIT_ERR_NONFINITE = 4,   /* device found a NaN / Inf score (status word) */
   CONDUIT_ERR_TIMEOUT = 5,     /* a bounded device wait ran out (status word) */
