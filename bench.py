@@ -529,7 +529,21 @@ def cpu_baseline(cfg: str, seconds: float, ratio=None) -> dict:
     est = statistics.median(ests)
     return {"value": round(n_tok / est, 2), "unit": UNIT, "cores": _CORES, "kind": "oracle",
             "sample": f"{len(ests)} repetition(s) of: {desc}", "sample_seconds": round(spent, 1),
+            "cpu": _cpu_model(),
             "threads_note": f"numpy BLAS threads = {_CORES}; elementwise numpy is single-threaded"}
+
+
+def _cpu_model() -> str:
+    """The host CPU's model name (lscpu), else the machine type."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.strip().startswith("Model name:"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    import platform
+    return platform.machine()
 
 
 def _workload_tokens(cfg: str) -> int:
@@ -563,7 +577,7 @@ def run_reference(args):
         "config": {"workload": DESCR[args.config], "name": args.config, "tokens_per_step": n_tok,
                    "ratio_override": args.ratio},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": _CORES, "kind": "oracle",
-                         "sample": desc},
+                         "sample": desc, "cpu": _cpu_model()},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(out), flush=True)
