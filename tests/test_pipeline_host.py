@@ -54,3 +54,29 @@ def test_pipelines_of_different_shapes_are_refused(P):
         P.DoubleBuffered(a, P.from_inputs(_inputs(tokens_per_image=48)))
     with pytest.raises(ValueError, match="same batch shape"):
         P.DoubleBuffered(a, P.from_inputs(_inputs(), budgets=[5]))
+
+
+def test_bench_work_model_matches_closed_forms(P):
+    """The algorithmic bytes and FLOPs behind bench.py's roofline figures, on
+    a hand-fixed selection: scoring reads K, V and Q once and writes s, A, g;
+    the exchange reads and writes K and V rows twice (gather, scatter);
+    refresh reads its query rows, writes its output and reads the K/V prefix
+    up to the largest selected position, with causal FLOPs 4 Hq d (p + 1)."""
+    import bench
+    x = _inputs(num_layers=2)
+    k = 5
+    pipe = P.from_inputs(_own(x), budgets=[k])
+    sel = [1, 7, 20, 33, 60]
+    pipe.idx[:k] = torch.tensor(sel, dtype=torch.int32)
+    m = bench.work_model(pipe)
+    L, Hq, Hkv, d, b = 2, 28, 4, 128, 2
+    N, nq, K = 64, 4, 2
+    assert m["score"]["bytes"] == 2 * L * Hkv * N * d * b + L * Hq * nq * d * b + 8 * N + 4 * K
+    assert m["score"]["flops"] == 2 * L * Hq * nq * N * d
+    assert m["exchange"]["bytes"] == 8 * L * k * Hkv * d * b
+    assert m["refresh"]["flops"] == L * sum(4 * Hq * d * (p + 1) for p in sel)
+    assert m["refresh"]["bytes"] == 2 * L * k * Hq * d * b + 2 * L * Hkv * (max(sel) + 1) * d * b
+    # scoring by attention alone drops the V read
+    alone = P.from_inputs(_own(x), budgets=[k], value_norm="none")
+    alone.idx[:k] = torch.tensor(sel, dtype=torch.int32)
+    assert m["score"]["bytes"] - bench.work_model(alone)["score"]["bytes"] == L * Hkv * N * d * b
