@@ -47,3 +47,31 @@ def test_reduce_max_over_two_gloo_ranks():
 def test_single_rank_is_identity():
     import bench
     assert bench.reduce_max(4.25, 1) == 4.25
+
+
+def _reference_run(rank: int, world: int):
+    import json
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    env = {**os.environ, "RANK": str(rank), "WORLD_SIZE": str(world), "LOCAL_RANK": str(rank)}
+    p = subprocess.run([sys.executable, "bench.py", "--impl", "reference", "--config", "tiny", "--steps", "2",
+                        "--warmup", "0", "--reference-step-seconds", "0.3"],
+                       cwd=root, env=env, capture_output=True, text=True, timeout=600)
+    lines = [json.loads(x) for x in p.stdout.splitlines() if x.startswith("{")]
+    return p.returncode, lines
+
+
+def test_reference_arm_runs_on_rank_zero_only():
+    """Under two ranks the oracle arm runs once: rank 0 prints the line, the
+    other rank exits 0 without work; the oracle's throughput is its own
+    (tokens per step over seconds per step), not multiplied by the rank count."""
+    rc1, lines1 = _reference_run(1, 2)
+    assert rc1 == 0 and lines1 == []
+    rc0, lines0 = _reference_run(0, 2)
+    assert rc0 == 0 and len(lines0) == 1
+    line = lines0[0]
+    assert line["impl"] == "reference" and line["n_gpus"] == 2
+    assert line["value"] == line["cpu_baseline"]["value"] == line["e2e"]["value"]
+    per_step = line["config"]["tokens_per_step"] / (line["ms_per_step"] / 1e3)
+    assert abs(line["value"] - per_step) <= 0.01 * per_step
