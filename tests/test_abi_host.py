@@ -119,6 +119,27 @@ def test_score_rejects_bad_arguments(C):
     _expect(C, C.ERR_INVALID_ARG, C.conduit_score, kv, b, None)
 
 
+def test_batch_structure_is_checked(C):
+    """Reading c7: every request has visual tokens and images, images are
+    non-empty spans that tile their request, offsets start at 0."""
+    kv = _kv(C)
+    q = torch.zeros((2, 4, 8, 64), dtype=torch.bfloat16)
+    # a request with tokens but no images
+    bad = _batch(C, img=(0, 32, 64), rio=(0, 2, 2))
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_score, kv, bad, q, match="no images")
+    # the image count of the last request does not close the image list
+    bad = _batch(C, rio=(0, 2, 2))
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_score, kv, bad, q, match="num_images")
+    # offsets that do not start at 0
+    bad = _batch(C, tok=(1, 64, 128), img=(1, 32, 64, 128))
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_score, kv, bad, q, match="start at 0")
+    # more images in one request than the selection keeps in shared memory
+    n = 4097
+    many = C.Batch([0, n], list(range(n + 1)), [0, n], [0, 4], device="cpu")
+    _expect(C, C.ERR_UNSUPPORTED, C.conduit_score, _kv(C, n=n), many,
+            torch.zeros((2, 4, 4, 64), dtype=torch.bfloat16), match="more than 4096 images")
+
+
 def test_select_rejects_bad_budgets_and_lambda(C):
     b = _batch(C)
     s = torch.zeros(128)
