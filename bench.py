@@ -6,7 +6,9 @@ gather, scatter and refresh attention over one batch of a synthetic workload.
 
 Prints one JSON line. ``value`` is cached visual tokens passed through the
 whole step per second (device time, inputs resident in HBM, L2 flushed
-between steps); ``e2e`` is the same through the public step with the cache,
+between steps); ``metric_parts`` splits it into the metric's two halves
+(tokens scored and selected per second, refresh-pass µs) from per-call
+times; ``e2e`` is the same through the public step with the cache,
 queries and fresh rows copied from pinned host memory each step and the
 selection and refresh output copied back, over back-to-back steps of two
 pipelines that alternate (one step's copies overlap the previous step's
@@ -434,6 +436,14 @@ def run_conduit(args):
         "refresh_pass_us": round((call_ms["exchange"] + call_ms.get("norm_update", 0.0)
                                   + call_ms["refresh"]) * 1e3, 2),
         "breakdown": breakdown,
+        # the metric's two halves from the eager per-call times: tokens scored and
+        # selected per second, and the refresh pass (K/V exchange, the norm update
+        # when the side cache is kept, refresh attention)
+        "metric_parts": {
+            "scored_selected_tokens_per_s": round(world * n_tok / ((call_ms["score"] + call_ms["select"]) / 1e3), 1),
+            "refresh_pass_us": round(1e3 * sum(call_ms[k] for k in ("exchange", "norm_update", "refresh")
+                                               if k in call_ms), 2),
+        },
         **({"side_cache_build": side_cache} if side_cache else {}),
         "roofline": roofline,
         "e2e": {"value": round(world * n_tok / (e2e_mean / 1e3), 1), "unit": UNIT,
