@@ -1,0 +1,34 @@
+"""Host logic of bench.py that needs no GPU: the clock record of the timed
+region (median SM clock, maximum clock, throttle reasons seen)."""
+
+import bench
+
+
+def _sampler(lines):
+    c = bench.ClockSampler(0)
+    c.lines = list(lines)
+    return c.summary()
+
+
+def test_clock_summary_median_max_and_reasons():
+    na, act = "Not Active", "Active"
+    lines = [
+        f"0, 2070, 2070, 900.1, 0x0, {na}, {na}, {na}, {na}",
+        f"0, 1980, 2070, 1400.0, 0x4, {na}, {na}, {na}, {act}",
+        f"0, 2070, 2070, 1390.5, 0x0, {na}, {na}, {na}, {na}",
+        "garbled line",
+        "0, [N/A], 2070, 1.0, 0x0, x, x, x, x",
+    ]
+    s = _sampler(lines)
+    assert s == {"sm_mhz": 2070.0, "sm_max_mhz": 2070.0, "reasons": ["sw_power_cap"], "samples": 3}
+
+
+def test_clock_summary_flags_every_slowdown_kind():
+    act = "Active"
+    s = _sampler([f"0, 1200, 2070, 700, 0x68, {act}, {act}, {act}, Not Active"])
+    assert s["reasons"] == ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown"]
+    assert s["sm_mhz"] == 1200.0
+
+
+def test_clock_summary_without_samples():
+    assert _sampler([]) == {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
