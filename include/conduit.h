@@ -300,6 +300,12 @@ conduit_status conduit_select_quota(const conduit_batch* batch, const float* s, 
  *    (tok_off[R]) is rejected with CONDUIT_ERR_UNSUPPORTED.
  *  - The first call on a device looks up the array's device address with
  *    that device current; make that first call before any stream capture.
+ *    The CUDA runtime may load the library's device code onto a device only
+ *    at that lookup (or at the library's first launch there), so that first
+ *    use needs about 4 MiB of free device memory; a caller that hands all
+ *    free memory to its KV pool should make one call (or any other library
+ *    call) first. If the lookup fails, for lack of memory or otherwise, the
+ *    call returns CONDUIT_ERR_CUDA with the runtime's message.
  *  - The call allocates nothing: no cudaMalloc, cudaFree or other
  *    allocating routine.
  *  - All calls share the array and it keeps the last call's contents. Each

@@ -60,7 +60,6 @@ __all__ = [
     "image_coefficients",
     "composite_score",
     "topk_select",
-    "image_coefficients_f32",
     "image_quotas",
     "quota_select",
     "refresh_mask",
@@ -246,29 +245,6 @@ def topk_select(s_hat: np.ndarray, k: int) -> np.ndarray:
 # App. D.3 ("explicit" cross-image variant): quotas k_j proportional to
 # c_j n_j, then a top-k_j inside each image.
 # --------------------------------------------------------------------------
-def image_coefficients_f32(g: np.ndarray, lam: float) -> np.ndarray:
-    """Eq. 9 evaluated in binary32, one rounding per operation, for decisions
-    that turn c_j into integers (the quotas below) in the kernel's precision:
-    g_bar = (((g_0 + g_1) + g_2) + ...) / K, c_j = (1 - lambda) + lambda * (g_j / g_bar),
-    c = 1 for K == 1 or g_bar == 0.
-    """
-    f = np.float32
-    g = np.asarray(g, dtype=np.float32)
-    k_img = g.shape[0]
-    lam32 = f(lam)
-    if k_img == 1:
-        return np.ones(1, dtype=np.float32)
-    total = f(0.0)
-    for j in range(k_img):
-        total = f(total + g[j])
-    g_bar = f(total / f(k_img))
-    if g_bar == 0:
-        return np.ones(k_img, dtype=np.float32)
-    one_minus = f(f(1.0) - lam32)
-    return np.array([f(one_minus + f(lam32 * f(g[j] / g_bar))) for j in range(k_img)],
-                    dtype=np.float32)
-
-
 def image_quotas(c: np.ndarray, n: Sequence[int], k: int) -> np.ndarray:
     """k_j proportional to c_j n_j with sum_j k_j = k and 0 <= k_j <= n_j.
 

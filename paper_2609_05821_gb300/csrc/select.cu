@@ -387,10 +387,10 @@ __global__ void __launch_bounds__(kQuotaThreads) quota_kernel(BatchDev b, const 
 }
 
 // Scratch of conduit_select_topk_noalloc: the sortable keys of up to
-// kNoAllocMaxTokens tokens (4 MiB), resident on every device that loads the
-// library until the process exits. Each call overwrites the keys of its own
-// tokens before reading them, so nothing needs clearing between calls.
-constexpr int64_t kNoAllocMaxTokens = int64_t(1) << 20;
+// CONDUIT_NOALLOC_MAX_TOKENS tokens (4 MiB), resident on every device that
+// loads the library until the process exits. Each call overwrites the keys of
+// its own tokens before reading them, so nothing needs clearing between calls.
+constexpr int64_t kNoAllocMaxTokens = CONDUIT_NOALLOC_MAX_TOKENS;
 static __device__ __align__(256) uint32_t g_noalloc_keys[kNoAllocMaxTokens];
 
 constexpr int kMaxDevices = 64;

@@ -310,3 +310,13 @@ def test_last_error_is_thread_local(C):
     t.start()
     t.join()
     assert seen == [""] and "out of range" in main_msg
+
+
+def test_noalloc_limit_is_the_header_value(C):
+    """The binding's limit of conduit_select_topk_noalloc is the header's
+    CONDUIT_NOALLOC_MAX_TOKENS (the library sizes its static array from it)."""
+    m = re.search(r"#define\s+CONDUIT_NOALLOC_MAX_TOKENS\s+\(1\s*<<\s*(\d+)\)", open(HEADER).read())
+    assert m is not None
+    assert C.NOALLOC_MAX_TOKENS == 1 << int(m.group(1))
+    src = open(os.path.join(ROOT, "paper_2609_05821_gb300", "csrc", "select.cu")).read()
+    assert re.search(r"kNoAllocMaxTokens\s*=\s*CONDUIT_NOALLOC_MAX_TOKENS\s*;", src)

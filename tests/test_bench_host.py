@@ -32,3 +32,20 @@ def test_clock_summary_flags_every_slowdown_kind():
 
 def test_clock_summary_without_samples():
     assert _sampler([]) == {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+
+
+def test_reference_arm_line_on_the_cpu(capsys):
+    """The reference arm (the CPU oracle) on the tiny workload: it prints the
+    GPU arm's config dict, a measured per-step sample time, and marks the
+    extrapolation to the whole step."""
+    import argparse
+    import json
+    args = argparse.Namespace(config="tiny", steps=2, warmup=0, ratio=None, no_graph=False,
+                              statistic="mean", value_norm="v", full_context=False,
+                              selection="global", reference_step_seconds=0.2)
+    bench.run_reference(args)
+    line = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
+    assert line["impl"] == "reference" and line["extrapolated"] is True
+    assert line["config"] == bench.run_config(args, 256, 25, 1)
+    assert 0 < line["ms_per_step"] <= line["extrapolated_full_step_ms"] * 1.5
+    assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["value"] > 0

@@ -64,6 +64,6 @@ def test_fuzzed_shapes(C, P, case):
     ref = _oracle(inputs, budgets=budgets)
     rtol = PT.RTOL[torch.float32 if dtype == "f32" else torch.bfloat16]
     PT.compare_score_select(pipe, inputs, ref, rtol)
-    _check_refresh(pipe, inputs, ref, 1e-5 if dtype == "f32" else None)
+    _check_refresh(P, pipe, inputs, ref, 1e-5 if dtype == "f32" else None)
     _patched_equals_scatter(C, pipe, inputs)
     assert C.conduit_read_status(pipe.status) == C.OK

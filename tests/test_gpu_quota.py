@@ -1,11 +1,14 @@
 """GPU parity of the explicit per-image quota selection (App. D.3).
 
-Integer work, so the bar is bitwise: on the same fp32 scores s and image
-means g, conduit_select_quota must return
-  coeff  bitwise the oracle's binary32 restatement of Eq. 9,
-  quota  exactly the oracle's largest-remainder quotas for those coefficients,
-  idx    exactly the oracle's per-image top-k_j of s (ties to the lowest index),
-  mask / s_hat consistent with idx and s * c.
+On the same fp32 scores s and image means g, conduit_select_quota must return
+  coeff  Eq. 9 in fp64 (the oracle) within 1e-5 relative (the kernel
+         evaluates it in binary32),
+  quota  the oracle's fp64 largest-remainder quotas, differing by one unit
+         only for an image whose fp64 decision lay within the coefficients'
+         tolerance of flipping (tests/parity.py, assert_quotas_in_band),
+  idx    exactly the per-image top-k_j of s at the kernel's quotas (integer
+         work on the same fp32 s: bitwise, ties to the lowest index),
+  mask / s_hat consistent with idx and with s times the kernel's own c.
 The crafted batches cover unequal image sizes, a cap (an image whose share
 exceeds its size), all-zero weights, lambda 0 / 0.5 / 1, budgets 0 and N_r,
 and tied scores. On the full multi-image and long-document workloads the
@@ -23,6 +26,10 @@ from paper_2609_05821_gb300 import synth
 from tests import parity as PT
 
 pytestmark = pytest.mark.gpu
+
+# relative error bound of the binary32 c_j of the kernel against Eq. 9 in fp64
+# (a sum of up to 5 fp32 means, one division, one fused step: a few ulps)
+C_RTOL = 1e-5
 
 
 @pytest.fixture(scope="module")
@@ -72,7 +79,7 @@ def _crafted(C, seed, g_mode):
 
 @pytest.mark.parametrize("lam", [0.0, 0.5, 1.0])
 @pytest.mark.parametrize("g_mode", ["random", "dominant", "zeros"])
-def test_quota_selection_bitwise(C, lam, g_mode):
+def test_quota_selection_crafted(C, lam, g_mode):
     s, g, batch, budgets, tok, img, rio = _crafted(C, 11, g_mode)
     off, off_d = C.idx_offsets(budgets, "cuda")
     n_tot, K = tok[-1], len(img) - 1
@@ -91,22 +98,26 @@ def test_quota_selection_bitwise(C, lam, g_mode):
     o = off.tolist()
     for r in range(len(CRAFTED)):
         j0, j1, t0, t1 = rio[r], rio[r + 1], tok[r], tok[r + 1]
-        c32 = O.image_coefficients_f32(g32[j0:j1], lam)
-        assert np.array_equal(coeff[j0:j1], c32), r
+        c64 = O.image_coefficients(g32[j0:j1].astype(np.float64), lam)
+        PT.assert_scores_close(coeff[j0:j1], c64, C_RTOL, f"c (request {r})")
         spans = [x - t0 for x in img[j0:j1 + 1]]
-        want = O.quota_select(s32[t0:t1].astype(np.float64), c32, spans, budgets[r])
-        assert quota[j0:j1].tolist() == want["quota"].tolist(), (r, quota[j0:j1], want["quota"])
-        assert idx[o[r]:o[r + 1]].tolist() == want["idx"].tolist(), r
-        m = np.zeros(t1 - t0, dtype=np.uint8)
-        m[want["idx"]] = 1
-        assert np.array_equal(mask[t0:t1], m)
         n = np.diff(spans)
-        assert np.array_equal(s_hat[t0:t1], s32[t0:t1] * np.repeat(c32, n))
+        PT.assert_quotas_in_band(quota[j0:j1], c64, n, budgets[r], C_RTOL)
+        want = []
+        for j in range(j1 - j0):  # the per-image top-k_j at the kernel's quotas
+            lo, hi = spans[j], spans[j + 1]
+            want.extend((lo + O.topk_select(s32[t0 + lo:t0 + hi].astype(np.float64), int(quota[j0 + j]))).tolist())
+        assert idx[o[r]:o[r + 1]].tolist() == sorted(want), r
+        m = np.zeros(t1 - t0, dtype=np.uint8)
+        m[sorted(want)] = 1
+        assert np.array_equal(mask[t0:t1], m)
+        assert np.array_equal(s_hat[t0:t1], s32[t0:t1] * np.repeat(coeff[j0:j1], n))
     if g_mode == "dominant" and lam == 1.0:
         assert quota[rio[3]] == 5                          # capped at its 5 tokens
 
 
-def test_global_coefficients_are_the_binary32_restatement(C):
+def test_global_coefficients_follow_eq9(C):
+    """conduit_select_topk's c_j against Eq. 9 in fp64 (binary32 on the GPU)."""
     s, g, batch, budgets, tok, img, rio = _crafted(C, 12, "random")
     off, off_d = C.idx_offsets(budgets, "cuda")
     coeff = torch.empty(len(img) - 1, device="cuda")
@@ -114,14 +125,18 @@ def test_global_coefficients_are_the_binary32_restatement(C):
     torch.cuda.synchronize()
     got = coeff.cpu().numpy()
     for r in range(len(CRAFTED)):
-        assert np.array_equal(got[rio[r]:rio[r + 1]], O.image_coefficients_f32(g.numpy()[rio[r]:rio[r + 1]], 0.7))
+        want = O.image_coefficients(g.numpy()[rio[r]:rio[r + 1]].astype(np.float64), 0.7)
+        PT.assert_scores_close(got[rio[r]:rio[r + 1]], want, C_RTOL, f"c (request {r})")
+        if rio[r + 1] - rio[r] == 1:
+            assert got[rio[r]] == 1.0                      # K = 1: c = 1 exactly (Sec. 3.5)
 
 
 @pytest.mark.parametrize("name", ["multi", "longdoc"])
 def test_quota_selection_on_scored_workloads(C, name):
     """The GPU's own scoring pass feeds the quota rule; against the oracle's
-    scores: quotas within one unit of the oracle's, exact sums, and per image
-    the selection bar of tests/parity.py at the GPU's quota."""
+    scores: quotas within the band of the fp64 rule (one unit, only near a
+    tie, at the score tolerance), exact sums, and per image the selection bar
+    of tests/parity.py at the GPU's quota."""
     from paper_2609_05821_gb300 import pipeline
     inputs = synth.make_inputs(synth.workload(name), device="cuda")
     pipe = pipeline.from_inputs(inputs, selection="quota")
@@ -131,10 +146,10 @@ def test_quota_selection_on_scored_workloads(C, name):
     spans = inputs["img_off"].tolist()
     n = np.diff(spans)
     quota = pipe.quota.cpu().numpy()
-    c32 = O.image_coefficients_f32(ref["g"].astype(np.float32), pipe.lam)
-    want_q = O.image_quotas(c32, n, ref["k"])
-    assert quota.sum() == ref["k"] and np.all(quota <= n) and np.all(quota >= 0)
-    assert np.all(np.abs(quota - want_q) <= 1)
+    # the GPU's g is within the score tolerance of the oracle's, so its c (and
+    # with it each ideal share) within about twice that
+    c64 = O.image_coefficients(ref["g"], pipe.lam)
+    PT.assert_quotas_in_band(quota, c64, n, ref["k"], 2 * PT.RTOL[torch.bfloat16])
     idx = pipe.idx.cpu().numpy()[:ref["k"]]
     for j in range(len(n)):
         lo, hi = spans[j], spans[j + 1]

@@ -73,5 +73,8 @@ def test_reference_arm_runs_on_rank_zero_only():
     line = lines0[0]
     assert line["impl"] == "reference" and line["n_gpus"] == 2
     assert line["value"] == line["cpu_baseline"]["value"] == line["e2e"]["value"]
-    per_step = line["config"]["tokens_per_step"] / (line["ms_per_step"] / 1e3)
+    # value: the step's tokens over the step time extrapolated from the
+    # measured samples (ms_per_step is the measured sample time per step)
+    per_step = line["config"]["tokens_per_step"] / (line["extrapolated_full_step_ms"] / 1e3)
     assert abs(line["value"] - per_step) <= 0.01 * per_step
+    assert line["extrapolated"] is True and line["ms_per_step"] > 0

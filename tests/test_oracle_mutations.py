@@ -93,14 +93,6 @@ def _quotas_ties_high_free(w, K, k):
     return base
 
 
-def _coefficients_f32_mean_over_k_minus_1(g, lam):
-    g = np.asarray(g, dtype=np.float32)
-    if g.shape[0] == 1:
-        return np.ones(1, dtype=np.float32)
-    gbar = np.float32(g.sum() / np.float32(g.shape[0] - 1))
-    return (np.float32(1 - lam) + np.float32(lam) * (g / gbar)).astype(np.float32)
-
-
 _staleness_iso = O.staleness_iso  # the original, for the mutants that wrap it
 
 
@@ -192,7 +184,6 @@ MUTANTS = {
     "quotas floored, leftover dropped": ("image_quotas", _quotas_floor_only),
     "quota remainder ties to the higher index": ("image_quotas", _quotas_ties_high),
     "quotas ignore image sizes": ("image_quotas", _quotas_ignore_sizes),
-    "f32 coefficients divide by K - 1": ("image_coefficients_f32", _coefficients_f32_mean_over_k_minus_1),
     "outside keys dropped": ("softmax_with_outside_keys", _outside_keys_dropped),
     "outside keys counted twice": ("softmax_with_outside_keys", _outside_keys_twice),
     "RMS without the root": ("head_query_rms_attention", _rms_without_root),

@@ -398,17 +398,6 @@ def test_quotas_minimise_deviation_brute_force():
         assert abs(np.abs(got - ideal).sum() - best) < 1e-9
 
 
-def test_coefficients_f32_follow_eq9():
-    rng = np.random.default_rng(22)
-    for lam in (0.0, 0.3, 1.0):
-        g = rng.uniform(0.0, 0.01, size=7).astype(np.float32)
-        c32 = O.image_coefficients_f32(g, lam)
-        assert c32.dtype == np.float32
-        np.testing.assert_allclose(c32, O.image_coefficients(g.astype(np.float64), lam), rtol=2e-6)
-    assert O.image_coefficients_f32(np.array([0.2], dtype=np.float32), 0.7).tolist() == [1.0]
-    assert O.image_coefficients_f32(np.zeros(3, dtype=np.float32), 1.0).tolist() == [1.0] * 3
-
-
 def test_quota_select_per_image_top():
     rng = np.random.default_rng(23)
     s = rng.uniform(size=40)
