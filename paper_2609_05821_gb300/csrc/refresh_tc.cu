@@ -196,13 +196,26 @@ __device__ __forceinline__ void raise_abort(const RefArgs& a, const Smem& s, int
   *s.abort = 1;
 }
 
+// Page of the 128-key tile starting at request-local key j0 that lane
+// `lane` copies (page lane / 2 of the tile; 0 for a contiguous cache or a lane
+// without a copy). The loaders fetch it one tile ahead, so that the page-table
+// load overlaps the wait for a free stage.
+__device__ __forceinline__ int tile_page(const RefArgs& a, int r, int N, int j0, int lane) {
+  const KvDev& kv = a.kv;
+  if (kv.page_size == 0) return 0;
+  const int ps = kv.page_size, i = lane >> 1;
+  if (i >= kKT / ps) return 0;
+  const int lp = min((j0 + i * ps) / ps, (N - 1) / ps);  // tail pages repeat the last one (masked)
+  return __ldg(kv.page_table + int64_t(r) * kv.max_pages + lp);
+}
+
 // Warp-cooperative TMA of the 128-key tile starting at request-local key j0:
 // lane 0 posts the byte count, then copy c is issued by lane c. A copy is one
 // 64-dim half of the whole tile (contiguous cache: 2 copies) or of one page
-// (paged cache: 2 x 128/page copies, up to 32), so a paged tile costs one
-// round of parallel page-index loads and copy issues instead of a serial loop.
+// (paged cache: 2 x 128/page copies, up to 32; `page` from tile_page), so a
+// paged tile costs one round of parallel copy issues.
 __device__ __forceinline__ void load_tile(const RefArgs& a, const CUtensorMap* map, uint8_t* dst,
-                                          uint64_t* bar, int l, int g, int r, int t0, int N, int j0,
+                                          uint64_t* bar, int l, int g, int t0, int j0, int page,
                                           int lane) {
   const KvDev& kv = a.kv;
   if (lane == 0) tc::mbar_arrive_expect_tx(bar, kTileBytes);
@@ -217,8 +230,6 @@ __device__ __forceinline__ void load_tile(const RefArgs& a, const CUtensorMap* m
     const int ps = kv.page_size;
     const int i = lane >> 1;  // page of the tile
     if (i < kKT / ps) {
-      const int lp = min((j0 + i * ps) / ps, (N - 1) / ps);  // tail pages repeat the last one (masked)
-      const int page = kv.page_table[int64_t(r) * kv.max_pages + lp];
       const int32_t y = int32_t(((int64_t(l) * kv.num_pages + page) * kv.Hkv + g) * ps);
       tc::tma_load_2d(dst + hf * kTileHalf + i * ps * 128, map, bar, hf * 64, y);
     }
@@ -334,14 +345,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       if (u < 0) break;
+      int page = nt > 0 ? tile_page(a, it.r, N, 0, lane) : 0;
       for (int t = 0; t < nt; ++t, ++T) {
+        const int page_next = t + 1 < nt ? tile_page(a, it.r, N, (t + 1) * kKT, lane) : 0;
         const int sk = T % kKStages;
         if (!__all_sync(0xffffffffu, wait_or_abort(&s.kempty[sk], ((T / kKStages) & 1) ^ 1, s.abort))) {
           if (lane == 0) raise_abort(a, s, tc::kSiteLoad);
           ok = false;
           break;
         }
-        load_tile(a, &kmap, s.k + sk * kTileBytes, &s.kfull[sk], it.l, it.g, it.r, t0, N, t * kKT, lane);
+        load_tile(a, &kmap, s.k + sk * kTileBytes, &s.kfull[sk], it.l, it.g, t0, t * kKT, page, lane);
+        page = page_next;
         ++nk;
       }
     }
@@ -364,14 +378,17 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (lane == 0) tc::mbar_arrive(&s.qempty[qs]);  // this warp is done with the record
       if (u < 0) break;
       bool ok = true;
+      int page = nt > 0 ? tile_page(a, r, N, 0, lane) : 0;
       for (int t = 0; t < nt; ++t, ++T) {
+        const int page_next = t + 1 < nt ? tile_page(a, r, N, (t + 1) * kKT, lane) : 0;
         const int sv = T % kVStages;
         if (!__all_sync(0xffffffffu, wait_or_abort(&s.vempty[sv], ((T / kVStages) & 1) ^ 1, s.abort))) {
           if (lane == 0) raise_abort(a, s, tc::kSiteLoad);
           ok = false;
           break;
         }
-        load_tile(a, &vmap, s.v + sv * kTileBytes, &s.vfull[sv], l, g, r, t0, N, t * kKT, lane);
+        load_tile(a, &vmap, s.v + sv * kTileBytes, &s.vfull[sv], l, g, t0, t * kKT, page, lane);
+        page = page_next;
         ++nv;
       }
       if (!ok) break;

@@ -179,13 +179,26 @@ __device__ __forceinline__ void epi_barrier() {
   asm volatile("bar.sync 1, %0;" ::"n"(kEpiThreads) : "memory");
 }
 
+// Page of K (or V) tile `tile` of unit w that lane `lane` copies (page
+// lane / 2 of the tile; 0 for a contiguous cache or a lane without a copy).
+// The producers fetch it one tile ahead, so that the page-table load overlaps
+// the wait for a free buffer.
+__device__ __forceinline__ int tile_page(const TcArgs& a, const Unit& w, int tile, int lane) {
+  const KvDev& kv = a.kv;
+  if (kv.page_size == 0) return 0;
+  const int ps = kv.page_size, i = lane >> 1;
+  if (i >= kTile / ps) return 0;
+  const int lp = min((tile * kTile + i * ps) / ps, (w.N - 1) / ps);  // tail pages repeat the last one (masked)
+  return __ldg(kv.page_table + int64_t(w.r) * kv.max_pages + lp);
+}
+
 // Warp-cooperative TMA of K (or V) tile `tile` of unit w into `dst`: lane 0
 // posts the byte count, then copy c is issued by lane c. A copy is one 64-dim
 // half of the whole tile (contiguous cache: 2 copies) or of one page (paged
-// cache: 2 x 128/page copies, up to 32), so a paged tile costs one round of
-// parallel page-index loads and copy issues.
+// cache: 2 x 128/page copies, up to 32; `page` from tile_page), so a paged
+// tile costs one round of parallel copy issues.
 __device__ __forceinline__ void load_k_tile(const TcArgs& a, const CUtensorMap* kmap, const Unit& w,
-                                            uint8_t* dst, uint64_t* bar, int tile, int lane) {
+                                            uint8_t* dst, uint64_t* bar, int tile, int page, int lane) {
   if (lane == 0) tc::mbar_arrive_expect_tx(bar, kStageBytes);
   __syncwarp();
   const int tok = tile * kTile;
@@ -200,8 +213,6 @@ __device__ __forceinline__ void load_k_tile(const TcArgs& a, const CUtensorMap* 
     const int ps = kv.page_size;
     const int i = lane >> 1;  // page of the tile
     if (i < kTile / ps) {
-      const int lp = min((tok + i * ps) / ps, (w.N - 1) / ps);  // tail pages repeat the last one (masked)
-      const int page = kv.page_table[int64_t(w.r) * kv.max_pages + lp];
       const int32_t y = int32_t(((int64_t(w.l) * kv.num_pages + page) * kv.Hkv + w.g) * ps);
       tc::tma_load_2d(dst + hf * kHalfK + i * ps * 128, kmap, bar, hf * 64, y);
     }
@@ -350,14 +361,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int u = blockIdx.x; u < a.n_units && ok; u += gridDim.x) {
       Unit w;
       if (!decode_unit(a, u, w)) continue;
+      int page = tile_page(a, w, tile_of(w, 0), lane);
       for (int i = 0; i < 2 * w.tiles; ++i, ++seq) {
+        const int page_next = i + 1 < 2 * w.tiles ? tile_page(a, w, tile_of(w, i + 1), lane) : 0;
         const int st = seq % kStages;
         if (!__all_sync(0xffffffffu, wait_or_abort(&s.kempty[st], ((seq / kStages) & 1) ^ 1, s.abort))) {
           if (lane == 0 && !*s.abort) raise_abort(a, s, tc::kSiteLoad);
           ok = false;
           break;
         }
-        load_k_tile(a, &kmap, w, s.k + st * kStageBytes, &s.kfull[st], tile_of(w, i), lane);
+        load_k_tile(a, &kmap, w, s.k + st * kStageBytes, &s.kfull[st], tile_of(w, i), page, lane);
+        page = page_next;
       }
     }
     if (lane == 0) s.counters[0] = seq;
@@ -370,14 +384,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int u = blockIdx.x; u < a.n_units && ok; u += gridDim.x) {
       Unit w;
       if (!decode_unit(a, u, w) || w.rg != 0) continue;
+      int page = tile_page(a, w, 0, lane);
       for (int i = 0; i < w.tiles; ++i, ++vseq) {
+        const int page_next = i + 1 < w.tiles ? tile_page(a, w, i + 1, lane) : 0;
         const int vb = vseq % kVBufs;
         if (!__all_sync(0xffffffffu, wait_or_abort(&s.vempty[vb], ((vseq / kVBufs) & 1) ^ 1, s.abort))) {
           if (lane == 0 && !*s.abort) raise_abort(a, s, tc::kSiteLoad);
           ok = false;
           break;
         }
-        load_k_tile(a, &vmap, w, s.v + vb * kStageBytes, &s.vfull[vb], i, lane);
+        load_k_tile(a, &vmap, w, s.v + vb * kStageBytes, &s.vfull[vb], i, page, lane);
+        page = page_next;
       }
     }
     if (lane == 0) s.counters[2] = vseq;
