@@ -49,8 +49,19 @@ enum {
   CONDUIT_ERR_WORKSPACE = 6    /* workspace pointer missing, misaligned or short */
 };
 
-/* Bits of the device status word. */
-enum { CONDUIT_FLAG_NONFINITE = 1, CONDUIT_FLAG_TIMEOUT = 2 };
+/*
+ * Bits of the device status word. A bounded wait that ran out sets
+ * CONDUIT_FLAG_TIMEOUT together with one site bit naming what never arrived:
+ * a TMA tile (CONDUIT_SITE_LOAD), an MMA completion (CONDUIT_SITE_MMA) or an
+ * item's final MMA completion (CONDUIT_SITE_FINAL).
+ */
+enum {
+  CONDUIT_FLAG_NONFINITE = 1,
+  CONDUIT_FLAG_TIMEOUT = 2,
+  CONDUIT_SITE_LOAD = 1 << 8,
+  CONDUIT_SITE_MMA = 1 << 9,
+  CONDUIT_SITE_FINAL = 1 << 10
+};
 
 /* Element type of K, V, queries, fresh rows and refresh outputs. */
 enum { CONDUIT_F32 = 0, CONDUIT_BF16 = 1 };

@@ -35,15 +35,20 @@ def _headers_mtime() -> float:
     return max((os.path.getmtime(h) for h in hs), default=0.0)
 
 
-def build(verbose: bool = False, extra_flags=()) -> str:
-    """Compile every csrc/*.cu and link libconduit.so; returns its path."""
+def build(verbose: bool = False, extra_flags=(), variant: str = "") -> str:
+    """Compile every csrc/*.cu and link libconduit.so; returns its path.
+
+    A `variant` builds a separate library (libconduit_<variant>.so, objects in
+    _build_<variant>/) with `extra_flags`, for the test suite only."""
     nvcc = _nvcc()
-    os.makedirs(BUILD, exist_ok=True)
+    bdir = os.path.join(HERE, "_build_" + variant) if variant else BUILD
+    lib = os.path.join(HERE, f"libconduit_{variant}.so") if variant else LIB
+    os.makedirs(bdir, exist_ok=True)
     sources = sorted(glob.glob(os.path.join(CSRC, "*.cu")))
     hdr_t = _headers_mtime()
 
     def compile_one(src: str) -> str:
-        obj = os.path.join(BUILD, os.path.basename(src)[:-3] + ".o")
+        obj = os.path.join(bdir, os.path.basename(src)[:-3] + ".o")
         if os.path.exists(obj) and os.path.getmtime(obj) >= max(os.path.getmtime(src), hdr_t):
             return obj
         cmd = [nvcc, *ARCH, *FLAGS, *extra_flags, "-c", src, "-o", obj]
@@ -58,12 +63,20 @@ def build(verbose: bool = False, extra_flags=()) -> str:
 
     with cf.ThreadPoolExecutor(max_workers=min(8, os.cpu_count() or 1)) as ex:
         objs = list(ex.map(compile_one, sources))
-    if not os.path.exists(LIB) or os.path.getmtime(LIB) < max(os.path.getmtime(o) for o in objs):
-        cmd = [nvcc, *ARCH, "-shared", "-o", LIB, *objs]
+    if not os.path.exists(lib) or os.path.getmtime(lib) < max(os.path.getmtime(o) for o in objs):
+        cmd = [nvcc, *ARCH, "-shared", "-o", lib, *objs]
         res = subprocess.run(cmd, capture_output=True, text=True)
         if res.returncode != 0:
-            raise RuntimeError(f"link of libconduit.so failed:\n{res.stderr}")
-    return LIB
+            raise RuntimeError(f"link of {os.path.basename(lib)} failed:\n{res.stderr}")
+    return lib
+
+
+def build_test_hooks(verbose: bool = False) -> str:
+    """The test-only library libconduit_testhooks.so: bounded device waits give
+    up after 1 ms instead of 1 s, and conduit_test_withhold_v_tile(n) makes the
+    scoring kernel's V producer skip one tile (no copy, no arrive), so a test
+    can run the timeout path without a fault. Never loaded by the package."""
+    return build(verbose, ("-DCONDUIT_TEST_HOOKS", "-DCONDUIT_WAIT_NS=1000000ull"), "testhooks")
 
 
 if __name__ == "__main__":

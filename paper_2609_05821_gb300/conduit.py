@@ -20,6 +20,8 @@ LIB_PATH = os.path.join(_HERE, "libconduit.so")
 
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_CUDA, ERR_NONFINITE, ERR_TIMEOUT, ERR_WORKSPACE = range(7)
 FLAG_NONFINITE, FLAG_TIMEOUT = 1, 2
+# with FLAG_TIMEOUT, the wait that ran out: a TMA tile, an MMA completion, an item's final MMA
+SITE_LOAD, SITE_MMA, SITE_FINAL = 1 << 8, 1 << 9, 1 << 10
 F32, BF16 = 0, 1
 MAX_LAYERS = 512
 STAT_MEAN, STAT_RMS = 0, 1

@@ -69,6 +69,9 @@ struct TcArgs {
   const float* extra_lse;  // [L][Hq][q_tot] natural-log LSE of keys outside the visual span, or NULL
   int32_t* status;
   LayerList layers;
+#ifdef CONDUIT_TEST_HOOKS
+  int32_t withhold_v;  // test builds: the V producer skips this V tile of each CTA (-1: none)
+#endif
 };
 
 struct Unit {
@@ -133,7 +136,8 @@ struct Smem {
   uint64_t* mdone;     // [1]
   uint32_t* tmem_slot;
   volatile int* abort;
-  uint32_t* counters;  // [0] K loads issued, [1] K loads consumed, [2] V issued, [3] V consumed
+  uint32_t* counters;  // [0] K loads issued, [1] K loads consumed, [2] V issued, [3] V consumed,
+                       // [4] (test builds) 1 + the V tile withheld, else 0
   float* lse;          // [256]
 };
 
@@ -344,7 +348,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc::mbar_init(s.qready, 1);
     tc::mbar_init(s.mdone, 1);
     *s.abort = 0;
-    for (int i = 0; i < 4; ++i) s.counters[i] = 0;
+    for (int i = 0; i < 5; ++i) s.counters[i] = 0;
     tc::fence_barrier_init();
     tc::prefetch_tensormap(&kmap);
     tc::prefetch_tensormap(&vmap);
@@ -393,6 +397,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           ok = false;
           break;
         }
+#ifdef CONDUIT_TEST_HOOKS
+        if (int(vseq) == a.withhold_v) {  // neither copy nor arrive: the consumer's wait runs out
+          if (lane == 0) s.counters[4] = vseq + 1;
+          page = page_next;
+          continue;
+        }
+#endif
         load_k_tile(a, &vmap, w, s.v + vb * kStageBytes, &s.vfull[vb], i, page, lane);
         page = page_next;
       }
@@ -620,7 +631,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (uint32_t n = s.counters[1]; n < s.counters[0]; ++n)
       tc::mbar_wait(&s.kfull[n % kStages], (n / kStages) & 1);
     for (uint32_t n = s.counters[3]; n < s.counters[2]; ++n)
-      tc::mbar_wait(&s.vfull[n % kVBufs], (n / kVBufs) & 1);
+      if (n + 1 != s.counters[4])  // (test builds) a withheld V tile has nothing in flight
+        tc::mbar_wait(&s.vfull[n % kVBufs], (n / kVBufs) & 1);
   }
   tc::tc_fence_before();
   __syncthreads();
@@ -646,6 +658,14 @@ EncodeTiledFn encode_fn() {
 }
 
 }  // namespace
+
+#ifdef CONDUIT_TEST_HOOKS
+// Test builds only (never in libconduit.so): the next scoring launches
+// withhold V tile n of each CTA (n < 0: none), so that the epilogue's bounded
+// wait for it runs out and the kernel takes its timeout path.
+int32_t g_test_withhold_v = -1;
+extern "C" void conduit_test_withhold_v_tile(int32_t n) { g_test_withhold_v = n; }
+#endif
 
 bool score_tc_supported(const KvDev& kv) {
   if (kv.dtype != CONDUIT_BF16 || kv.d != kD) return false;
@@ -699,6 +719,9 @@ cudaError_t launch_score_tc(const KvDev& kv, const BatchDev& b, const int32_t* q
   a.extra_lse = extra_lse;
   a.status = status;
   a.layers = layers;
+#ifdef CONDUIT_TEST_HOOKS
+  a.withhold_v = g_test_withhold_v;
+#endif
   if (units == 0) return cudaSuccess;
 
   int dev = 0, sms = 0;

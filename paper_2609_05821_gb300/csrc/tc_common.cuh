@@ -8,6 +8,8 @@
 #include <cuda.h>
 #include <stdint.h>
 
+#include "conduit.h"
+
 namespace conduit {
 namespace tc {
 
@@ -20,9 +22,9 @@ constexpr uint64_t kWaitNs = CONDUIT_WAIT_NS;    // polling time before a wait g
 
 // Diagnostic bits of the status word, set next to CONDUIT_FLAG_TIMEOUT to
 // name the wait that ran out.
-constexpr int32_t kSiteLoad = 1 << 8;    // a TMA tile never arrived
-constexpr int32_t kSiteMma = 1 << 9;     // an MMA commit never arrived
-constexpr int32_t kSiteFinal = 1 << 10;  // the final commit of an item (or CTA) never arrived
+constexpr int32_t kSiteLoad = CONDUIT_SITE_LOAD;    // a TMA tile never arrived
+constexpr int32_t kSiteMma = CONDUIT_SITE_MMA;      // an MMA commit never arrived
+constexpr int32_t kSiteFinal = CONDUIT_SITE_FINAL;  // the final commit of an item (or CTA) never arrived
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));

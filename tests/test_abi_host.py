@@ -320,3 +320,18 @@ def test_noalloc_limit_is_the_header_value(C):
     assert C.NOALLOC_MAX_TOKENS == 1 << int(m.group(1))
     src = open(os.path.join(ROOT, "paper_2609_05821_gb300", "csrc", "select.cu")).read()
     assert re.search(r"kNoAllocMaxTokens\s*=\s*CONDUIT_NOALLOC_MAX_TOKENS\s*;", src)
+
+
+def test_status_bits_are_the_header_values(C):
+    text = open(HEADER).read()
+    for name, val in (("CONDUIT_FLAG_NONFINITE", C.FLAG_NONFINITE), ("CONDUIT_FLAG_TIMEOUT", C.FLAG_TIMEOUT),
+                      ("CONDUIT_SITE_LOAD", C.SITE_LOAD), ("CONDUIT_SITE_MMA", C.SITE_MMA),
+                      ("CONDUIT_SITE_FINAL", C.SITE_FINAL)):
+        m = re.search(name + r"\s*=\s*([0-9]+)(?:\s*<<\s*([0-9]+))?", text)
+        assert m is not None, name
+        assert val == int(m.group(1)) << int(m.group(2) or 0), name
+
+
+def test_product_library_has_no_test_hooks(C):
+    lib = ctypes.CDLL(C.LIB_PATH)
+    assert not hasattr(lib, "conduit_test_withhold_v_tile")
