@@ -52,6 +52,7 @@ constexpr int kSoftThreads = 256;
 constexpr int kVWarp = 10;                       // after the loader, MMA and eight softmax warps
 constexpr int kThreads = 64 + kSoftThreads + 32;
 constexpr int kKStages = 2;
+constexpr int kPageAhead = 4;                    // paged caches: tiles whose page indices load ahead
 constexpr int kVStages = 2;
 constexpr int kQBufs = 2;
 constexpr uint32_t kQHalf = kRows * 128;         // 16 KB: one 64-dim half of the query tile
@@ -198,8 +199,9 @@ __device__ __forceinline__ void raise_abort(const RefArgs& a, const Smem& s, int
 
 // Page of the 128-key tile starting at request-local key j0 that lane
 // `lane` copies (page lane / 2 of the tile; 0 for a contiguous cache or a lane
-// without a copy). The loaders fetch it one tile ahead, so that the page-table
-// load overlaps the wait for a free stage.
+// without a copy). The loaders fetch the pages of a group of tiles while they
+// issue the previous group's copies, so the page-table loads never hold back
+// a copy.
 __device__ __forceinline__ int tile_page(const RefArgs& a, int r, int N, int j0, int lane) {
   const KvDev& kv = a.kv;
   if (kv.page_size == 0) return 0;
@@ -345,9 +347,25 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       if (u < 0) break;
-      int page = nt > 0 ? tile_page(a, it.r, N, 0, lane) : 0;
+      // page indices go out a group of kPageAhead tiles ahead of their copies
+      int pg[kPageAhead], pg_next[kPageAhead];
+#pragma unroll
+      for (int j = 0; j < kPageAhead; ++j) pg[j] = j < nt ? tile_page(a, it.r, N, j * kKT, lane) : 0;
       for (int t = 0; t < nt; ++t, ++T) {
-        const int page_next = t + 1 < nt ? tile_page(a, it.r, N, (t + 1) * kKT, lane) : 0;
+        const int jj = t % kPageAhead;
+        if (jj == 0) {
+#pragma unroll
+          for (int j = 0; j < kPageAhead; ++j)
+            pg_next[j] = t + kPageAhead + j < nt ? tile_page(a, it.r, N, (t + kPageAhead + j) * kKT, lane) : 0;
+        }
+        int page = pg[0];
+#pragma unroll
+        for (int j = 1; j < kPageAhead; ++j)
+          if (jj == j) page = pg[j];
+        if (jj == kPageAhead - 1) {
+#pragma unroll
+          for (int j = 0; j < kPageAhead; ++j) pg[j] = pg_next[j];
+        }
         const int sk = T % kKStages;
         if (!__all_sync(0xffffffffu, wait_or_abort(&s.kempty[sk], ((T / kKStages) & 1) ^ 1, s.abort))) {
           if (lane == 0) raise_abort(a, s, tc::kSiteLoad);
@@ -355,7 +373,6 @@ __global__ void __launch_bounds__(kThreads, 1)
           break;
         }
         load_tile(a, &kmap, s.k + sk * kTileBytes, &s.kfull[sk], it.l, it.g, t0, t * kKT, page, lane);
-        page = page_next;
         ++nk;
       }
     }
@@ -378,9 +395,24 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (lane == 0) tc::mbar_arrive(&s.qempty[qs]);  // this warp is done with the record
       if (u < 0) break;
       bool ok = true;
-      int page = nt > 0 ? tile_page(a, r, N, 0, lane) : 0;
+      int pg[kPageAhead], pg_next[kPageAhead];
+#pragma unroll
+      for (int j = 0; j < kPageAhead; ++j) pg[j] = j < nt ? tile_page(a, r, N, j * kKT, lane) : 0;
       for (int t = 0; t < nt; ++t, ++T) {
-        const int page_next = t + 1 < nt ? tile_page(a, r, N, (t + 1) * kKT, lane) : 0;
+        const int jj = t % kPageAhead;
+        if (jj == 0) {
+#pragma unroll
+          for (int j = 0; j < kPageAhead; ++j)
+            pg_next[j] = t + kPageAhead + j < nt ? tile_page(a, r, N, (t + kPageAhead + j) * kKT, lane) : 0;
+        }
+        int page = pg[0];
+#pragma unroll
+        for (int j = 1; j < kPageAhead; ++j)
+          if (jj == j) page = pg[j];
+        if (jj == kPageAhead - 1) {
+#pragma unroll
+          for (int j = 0; j < kPageAhead; ++j) pg[j] = pg_next[j];
+        }
         const int sv = T % kVStages;
         if (!__all_sync(0xffffffffu, wait_or_abort(&s.vempty[sv], ((T / kVStages) & 1) ^ 1, s.abort))) {
           if (lane == 0) raise_abort(a, s, tc::kSiteLoad);
@@ -388,7 +420,6 @@ __global__ void __launch_bounds__(kThreads, 1)
           break;
         }
         load_tile(a, &vmap, s.v + sv * kTileBytes, &s.vfull[sv], l, g, t0, t * kKT, page, lane);
-        page = page_next;
         ++nv;
       }
       if (!ok) break;
