@@ -176,11 +176,14 @@ cudaError_t launch_staleness_iso(const KvDev& kv, const BatchDev& b, const int32
                                  int32_t q_tot, const void* q, const uint8_t* refreshed,
                                  const void* z, int M, float kappa, double* err, double* err_rl,
                                  void* workspace, int32_t* status, cudaStream_t stream);
-// max_tokens: the largest request (picks how many keys a thread keeps in registers).
+// max_tokens: the largest request (picks how many keys a thread keeps in
+// registers). Requests of more than 8 x 1024 tokens take one cluster of CTAs
+// each (keys in registers) when cluster_ok, else one CTA with its keys in
+// `keys`.
 cudaError_t launch_select(const BatchDev& b, int max_tokens, const float* s, const float* g,
                           float lambda, const int32_t* idx_off_dev, int32_t* idx, uint8_t* mask,
                           float* s_hat, float* coeff, uint32_t* keys, int32_t* status,
-                          cudaStream_t stream);
+                          cudaStream_t stream, bool cluster_ok = true);
 // Explicit per-image quotas (App. D.3): quota_kernel per request, then one
 // selection CTA per image. scratch holds quota_scratch_bytes(K) bytes.
 size_t quota_scratch_bytes(int total_images);

@@ -266,6 +266,201 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(BatchDev b, const f
   }
 }
 
+// ------------------------------------------------ one cluster per request
+// Requests too large for one CTA's registers (more than 8 x 1024 tokens) take
+// a cluster of kClusterCtas CTAs: CTA c of the cluster owns the c-th
+// contiguous chunk of the request's tokens and keeps its keys in registers.
+// Each radix pass builds a 256-bin histogram per CTA in shared memory; after a
+// cluster barrier every CTA sums the kClusterCtas histograms through
+// distributed shared memory and takes the same digit decision. The selected
+// indices go out in ascending order: each CTA's count of keys above the k-th
+// and of keys equal to it are exchanged the same way, ties go to the lowest
+// tokens. Histograms alternate between two buffers, so one cluster barrier per
+// pass suffices (a CTA rewrites a buffer only after every CTA has passed the
+// barrier that follows the reads of it).
+constexpr int kClusterCtas = 8;
+
+__device__ __forceinline__ void cluster_barrier() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+
+// 32-bit word at the same shared-memory offset in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t dsmem_ld(const void* local, uint32_t rank) {
+  const uint32_t a = static_cast<uint32_t>(__cvta_generic_to_shared(local));
+  uint32_t ra, v;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(ra) : "r"(a), "r"(rank));
+  asm volatile("ld.shared::cluster.u32 %0, [%1];" : "=r"(v) : "r"(ra) : "memory");
+  return v;
+}
+
+template <int kRegKeys>
+__global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kSelThreads)
+    select_cluster_kernel(BatchDev b, const float* s, const float* g, float lambda,
+                          const int32_t* idx_off, int32_t* idx, uint8_t* mask, float* s_hat,
+                          float* coeff, int32_t* status) {
+  __shared__ float c_s[kMaxImagesPerRequest];
+  __shared__ int img_s[kMaxImagesPerRequest + 1];
+  __shared__ unsigned hist[2][256];
+  __shared__ unsigned tot[256];
+  __shared__ int warp_s[32];
+  __shared__ uint32_t prefix_s;
+  __shared__ int remaining_s;
+  __shared__ float gbar_s;
+  __shared__ int counts_s[2];  // this CTA's keys above the k-th, equal to it
+
+  const uint32_t crank = cluster_rank();
+  const int r = blockIdx.x / kClusterCtas;
+  const int t0 = b.tok_off[r], N = b.tok_off[r + 1] - t0;
+  const int j0 = b.req_img_off[r], K = b.req_img_off[r + 1] - j0;
+  const int k = idx_off[r + 1] - idx_off[r];
+  int32_t* out = idx + idx_off[r];
+  for (int j = threadIdx.x; j <= K; j += blockDim.x) img_s[j] = b.img_off[j0 + j] - t0;
+  if (threadIdx.x == 0) gbar_s = image_mean_f32(g + j0, K);
+  __syncthreads();
+  for (int j = threadIdx.x; j < K; j += blockDim.x) {
+    const float c = image_coefficient(g[j0 + j], gbar_s, lambda, K);
+    c_s[j] = c;
+    if (coeff && crank == 0) coeff[j0 + j] = c;
+  }
+  __syncthreads();
+
+  // this CTA's chunk [c_lo, c_hi), then each thread's contiguous tokens
+  const int chunk = (N + kClusterCtas - 1) / kClusterCtas;
+  const int c_lo = min(N, int(crank) * chunk), c_hi = min(N, c_lo + chunk);
+  const int per = (c_hi - c_lo + kSelThreads - 1) / kSelThreads;
+  const int lo = min(c_hi, c_lo + int(threadIdx.x) * per), hi = min(c_hi, lo + per);
+  uint32_t kr[kRegKeys];
+  bool bad = false;
+  {
+    int a0 = 0, a1 = K - 1;  // image of token lo
+    while (a0 < a1) {
+      const int mid = (a0 + a1 + 1) >> 1;
+      if (img_s[mid] <= lo) a0 = mid; else a1 = mid - 1;
+    }
+    int img = a0;
+#pragma unroll
+    for (int j = 0; j < kRegKeys; ++j) {
+      kr[j] = 0u;
+      const int t = lo + j;
+      if (t < hi) {
+        while (img + 1 < K && img_s[img + 1] <= t) ++img;
+        float key = s[t0 + t] * c_s[img];
+        if (!isfinite(key) || key < 0.f) bad = true;
+        if (s_hat) s_hat[t0 + t] = key == 0.f ? 0.f : key;
+        if (key == 0.f) key = 0.f;  // -0 -> +0
+        kr[j] = __float_as_uint(key);
+      }
+    }
+  }
+  if (bad) flag_status(status, CONDUIT_FLAG_NONFINITE);
+  if (k == 0) {  // the same for every CTA of the cluster: none touches another's memory
+    if (mask)
+      for (int t = c_lo + int(threadIdx.x); t < c_hi; t += blockDim.x) mask[t0 + t] = 0;
+    return;
+  }
+
+  if (threadIdx.x == 0) {
+    prefix_s = 0u;
+    remaining_s = k;
+  }
+  uint32_t pmask = 0u;
+  int pass = 0;
+  for (int shift = 24; shift >= 0; shift -= 8, ++pass) {
+    unsigned* h = hist[pass & 1];
+    for (int i = threadIdx.x; i < 256; i += blockDim.x) h[i] = 0u;
+    __syncthreads();
+    const uint32_t prefix = prefix_s;
+#pragma unroll
+    for (int j = 0; j < kRegKeys; ++j)
+      if (lo + j < hi && (kr[j] & pmask) == prefix) atomicAdd(&h[(kr[j] >> shift) & 255u], 1u);
+    cluster_barrier();  // every CTA's histogram of this pass is complete
+    for (int i = threadIdx.x; i < 256; i += blockDim.x) {
+      unsigned t = 0u;
+      for (uint32_t c = 0; c < kClusterCtas; ++c) t += dsmem_ld(&h[i], c);  // fixed order
+      tot[i] = t;
+    }
+    __syncthreads();
+    if (threadIdx.x < 32) {  // the digit holding the remaining rank, as in select_kernel
+      const int lane = threadIdx.x;
+      int cnt[8], lsum = 0;
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        cnt[q] = int(tot[255 - 8 * lane - q]);
+        lsum += cnt[q];
+      }
+      int incl = lsum;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+      }
+      const int rem = remaining_s, excl = incl - lsum;
+      const unsigned hit = __ballot_sync(0xffffffffu, excl < rem && rem <= incl);
+      if (lane == __ffs(hit) - 1) {
+        int r2 = rem - excl, q = 0;
+        for (; q < 7; ++q) {
+          if (cnt[q] >= r2) break;
+          r2 -= cnt[q];
+        }
+        remaining_s = r2;
+        prefix_s = prefix | (uint32_t(255 - 8 * lane - q) << shift);
+      }
+    }
+    pmask |= 255u << shift;
+    __syncthreads();
+  }
+  const uint32_t kth = prefix_s;
+  const int need = remaining_s;  // keys equal to kth still to take over the request, >= 1
+
+  int gt = 0, eq = 0;
+#pragma unroll
+  for (int j = 0; j < kRegKeys; ++j)
+    if (lo + j < hi) {
+      gt += kr[j] > kth;
+      eq += kr[j] == kth;
+    }
+  int cta_gt = 0, cta_eq = 0;
+  const int eq_base_local = block_exclusive_scan(eq, warp_s, &cta_eq);
+  block_exclusive_scan(gt, warp_s, &cta_gt);
+  if (threadIdx.x == 0) {
+    counts_s[0] = cta_gt;
+    counts_s[1] = cta_eq;
+  }
+  cluster_barrier();  // every CTA's counts are published
+  // ties and output slots before this CTA's chunk (lower tokens)
+  int eq_before = 0, gt_before = 0;
+  for (uint32_t c = 0; c < crank; ++c) {
+    gt_before += int(dsmem_ld(&counts_s[0], c));
+    eq_before += int(dsmem_ld(&counts_s[1], c));
+  }
+  const int take_cta = max(0, min(cta_eq, need - eq_before));
+  const int out0 = gt_before + min(eq_before, need);
+  const int take_eq = max(0, min(eq, take_cta - eq_base_local));
+  const int pos0 = out0 + block_exclusive_scan(gt + take_eq, warp_s, nullptr);
+  int pos = pos0, seen_eq = 0;
+#pragma unroll
+  for (int j = 0; j < kRegKeys; ++j) {
+    const int t = lo + j;
+    if (t < hi) {
+      const uint32_t key = kr[j];
+      bool sel = key > kth;
+      if (key == kth) {
+        sel = seen_eq < take_eq;
+        ++seen_eq;
+      }
+      if (sel) out[pos++] = t;
+      if (mask) mask[t0 + t] = sel ? 1 : 0;
+    }
+  }
+  cluster_barrier();  // no CTA leaves while another may still read its counts
+}
+
 // Quotas of one request (App. D.3): c_j as the global rule computes it, then
 // k_j proportional to c_j n_j with sum k_j = k_r and k_j <= n_j, by the largest
 // remainder in float64 (w_j = c_j n_j, W summed left to right over the open
@@ -424,13 +619,13 @@ cudaError_t launch_select_noalloc(const BatchDev& b, int max_tokens, const float
     keys = g_noalloc_ptr[dev];
   }
   return launch_select(b, max_tokens, s, g, lambda, idx_off_dev, idx, mask, s_hat, coeff, keys,
-                       status, stream);
+                       status, stream, /*cluster_ok=*/false);
 }
 
 cudaError_t launch_select(const BatchDev& b, int max_tokens, const float* s, const float* g,
                           float lambda, const int32_t* idx_off_dev, int32_t* idx, uint8_t* mask,
                           float* s_hat, float* coeff, uint32_t* keys, int32_t* status,
-                          cudaStream_t stream) {
+                          cudaStream_t stream, bool cluster_ok) {
   // the smallest register budget that holds every request's keys
   if (max_tokens <= kSelThreads)
     select_kernel<1, false><<<b.R, kSelThreads, 0, stream>>>(
@@ -438,6 +633,9 @@ cudaError_t launch_select(const BatchDev& b, int max_tokens, const float* s, con
   else if (max_tokens <= 8 * kSelThreads)
     select_kernel<8, false><<<b.R, kSelThreads, 0, stream>>>(
         b, s, g, lambda, idx_off_dev, idx, mask, s_hat, coeff, keys, status, nullptr, nullptr, nullptr);
+  else if (cluster_ok && max_tokens <= kClusterCtas * 8 * kSelThreads)
+    select_cluster_kernel<8><<<b.R * kClusterCtas, kSelThreads, 0, stream>>>(
+        b, s, g, lambda, idx_off_dev, idx, mask, s_hat, coeff, status);
   else
     select_kernel<0, false><<<b.R, kSelThreads, 0, stream>>>(
         b, s, g, lambda, idx_off_dev, idx, mask, s_hat, coeff, keys, status, nullptr, nullptr, nullptr);
