@@ -147,8 +147,7 @@ struct ScoreLayout {
   bool tc;     // tensor-core kernel (bf16, head_dim 128) or the CUDA-core ones
   int rg_max;  // row groups per slab (column-sum partials per KV head)
   int group_rows;
-  int parts;     // partials per row group (4 for the tensor-core kernel)
-  int parts_ss;  // partials per value norm and KV head (2 for the tensor-core kernel)
+  int parts;   // partials per row group and per value norm (2 for the tensor-core kernel)
   size_t stats, pa, pa2, ss, attn, total;
 };
 
@@ -187,8 +186,7 @@ ScoreLayout score_layout(const conduit_kv* kv, const conduit_batch* b, int n_lay
   ScoreLayout s{};
   s.tc = score_tc_supported(make_kv(kv, b));
   s.rg_max = 1;
-  s.parts = s.tc ? 4 : 1;
-  s.parts_ss = s.tc ? 2 : 1;
+  s.parts = s.tc ? 2 : 1;
   if (s.tc) {
     s.group_rows = kScoreGroupRows;
     const int G = kv->num_q_heads / kv->num_kv_heads;
@@ -206,7 +204,7 @@ ScoreLayout score_layout(const conduit_kv* kv, const conduit_batch* b, int n_lay
   s.pa2 = off;
   if (mode.rms) off += pa_bytes;
   s.ss = off;
-  if (!normed) off += align_up(size_t(n_layers) * kv->num_kv_heads * s.parts_ss * n_tot * sizeof(float));
+  if (!normed) off += align_up(size_t(n_layers) * kv->num_kv_heads * s.parts * n_tot * sizeof(float));
   s.attn = off;
   off += align_up(n_tot * sizeof(float));
   s.total = off;
@@ -305,7 +303,7 @@ conduit_status score_impl(const conduit_kv* kv, const conduit_batch* batch, cons
   }
   if (err) return cuda_fail(err, "score");
   if ((err = launch_finalize(pa, pa2, ss, mode.vnorm, mode.vmode, ll, bd, ll.n, kd.Hkv, kd.Hq,
-                             lay.rg_max, lay.group_rows, lay.parts, lay.parts_ss, kd.n_tot, s, attn, g, status, cs)))
+                             lay.rg_max, lay.group_rows, lay.parts, kd.n_tot, s, attn, g, status, cs)))
     return cuda_fail(err, "finalize");
   return CONDUIT_OK;
 }

@@ -25,7 +25,7 @@ __global__ void __launch_bounds__(1024) finalize_tokens_kernel(const float* pa, 
                                                                const __grid_constant__ LayerList layers,
                                                                BatchDev b, int n_layers, int Hkv,
                                                                int Hq, int rg_max, int group_rows,
-                                                               int parts, int parts_ss, int64_t n_tot, float* s,
+                                                               int parts, int64_t n_tot, float* s,
                                                                float* attn_sum, int32_t* status) {
   __shared__ float part_s[kLayerSlots][33];
   __shared__ float part_a[kLayerSlots][33];
@@ -38,7 +38,7 @@ __global__ void __launch_bounds__(1024) finalize_tokens_kernel(const float* pa, 
     const float denom = float(nq * Hq);
     const int rows = (Hq / Hkv) * nq;
     const int n_sl = (group_rows ? (rows + group_rows - 1) / group_rows : 1) * parts;
-    const int npa = Hkv * n_sl, nss = Hkv * parts_ss;  // partials of one layer
+    const int npa = Hkv * n_sl, nss = Hkv * parts;  // partials of one layer
     for (int li = slot; li < n_layers; li += kLayerSlots) {
       // loads go out in batches of eight, so their latencies overlap
       const float* pa_l = pa + int64_t(li) * Hkv * rg_max * parts * n_tot + tg;
@@ -131,12 +131,12 @@ __global__ void __launch_bounds__(256) image_means_kernel(const float* attn_sum,
 
 cudaError_t launch_finalize(const float* pa, const float* pa2, const float* ss, const float* vnorm,
                             int vmode, const LayerList& layers, const BatchDev& b, int n_layers, int Hkv,
-                            int Hq, int rg_max, int group_rows, int parts, int parts_ss, int64_t n_tot,
-                            float* s, float* attn_sum, float* g, int32_t* status, cudaStream_t stream) {
+                            int Hq, int rg_max, int group_rows, int parts, int64_t n_tot, float* s,
+                            float* attn_sum, float* g, int32_t* status, cudaStream_t stream) {
   if (n_tot == 0) return cudaSuccess;
   const int threads = 32 * std::min(kLayerSlots, n_layers);
   finalize_tokens_kernel<<<unsigned((n_tot + 31) / 32), threads, 0, stream>>>(
-      pa, pa2, ss, vnorm, vmode, layers, b, n_layers, Hkv, Hq, rg_max, group_rows, parts, parts_ss, n_tot, s, attn_sum,
+      pa, pa2, ss, vnorm, vmode, layers, b, n_layers, Hkv, Hq, rg_max, group_rows, parts, n_tot, s, attn_sum,
       status);
   cudaError_t err = cudaGetLastError();
   if (err) return err;

@@ -137,7 +137,7 @@ cudaError_t launch_score_simt(const KvDev& kv, const BatchDev& b, const void* q,
                               float2* stats, float* pa, float* pa2, const float* extra_lse,
                               cudaStream_t stream);
 // Tensor-core scoring (bf16, head_dim 128): one kernel, row statistics then
-// column sums per (slab, group of at most 256 scoring rows); it writes four
+// column sums per (slab, group of at most 256 scoring rows); it writes two
 // partials per row group into pa and two half-row partials into ss (ss NULL:
 // V is not read, the norms come from the side cache).
 constexpr int kScoreGroupRows = 256;
@@ -147,7 +147,7 @@ cudaError_t launch_score_tc(const KvDev& kv, const BatchDev& b, const int32_t* q
                             const void* q, int32_t q_tot, const LayerList& layers, int rg_max,
                             float* pa, float* ss, float* pa2, const float* extra_lse,
                             int32_t* status, cudaStream_t stream);
-// pa is [n_layers][Hkv][rg_max][parts][n_tot] and ss [n_layers][Hkv][parts_ss][n_tot]
+// pa is [n_layers][Hkv][rg_max][parts][n_tot] and ss [n_layers][Hkv][parts][n_tot]
 // (partial sums of squares of V per KV head); request r contributes
 // ceil(G n_q_r / group_rows) row groups (one when group_rows == 0).
 // Value norms: vmode 0 from ss, 1 from the side cache vnorm [L][n_tot] (read
@@ -156,8 +156,7 @@ cudaError_t launch_score_tc(const KvDev& kv, const BatchDev& b, const int32_t* q
 // and g always take the mean of Eq. 6.
 cudaError_t launch_finalize(const float* pa, const float* pa2, const float* ss, const float* vnorm,
                             int vmode, const LayerList& layers, const BatchDev& b, int n_layers, int Hkv,
-                            int Hq, int rg_max, int group_rows, int parts, int parts_ss, int64_t n_tot,
-                            float* s,
+                            int Hq, int rg_max, int group_rows, int parts, int64_t n_tot, float* s,
                             float* attn_sum, float* g, int32_t* status, cudaStream_t stream);
 // Value-norm side cache: vnorm[l][tg] for every layer and for rows i < n_rows,
 // row i being global token i (idx == NULL) or request r's selected token

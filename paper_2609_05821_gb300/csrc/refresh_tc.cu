@@ -52,7 +52,6 @@ constexpr int kSoftThreads = 256;
 constexpr int kVWarp = 10;                       // after the loader, MMA and eight softmax warps
 constexpr int kThreads = 64 + kSoftThreads + 32;
 constexpr int kKStages = 2;
-constexpr int kPageAhead = 4;                    // paged caches: tiles whose page indices load ahead
 constexpr int kVStages = 2;
 constexpr int kQBufs = 2;
 constexpr uint32_t kQHalf = kRows * 128;         // 16 KB: one 64-dim half of the query tile
@@ -197,27 +196,13 @@ __device__ __forceinline__ void raise_abort(const RefArgs& a, const Smem& s, int
   *s.abort = 1;
 }
 
-// Page of the 128-key tile starting at request-local key j0 that lane
-// `lane` copies (page lane / 2 of the tile; 0 for a contiguous cache or a lane
-// without a copy). The loaders fetch the pages of a group of tiles while they
-// issue the previous group's copies, so the page-table loads never hold back
-// a copy.
-__device__ __forceinline__ int tile_page(const RefArgs& a, int r, int N, int j0, int lane) {
-  const KvDev& kv = a.kv;
-  if (kv.page_size == 0) return 0;
-  const int ps = kv.page_size, i = lane >> 1;
-  if (i >= kKT / ps) return 0;
-  const int lp = min((j0 + i * ps) / ps, (N - 1) / ps);  // tail pages repeat the last one (masked)
-  return __ldg(kv.page_table + int64_t(r) * kv.max_pages + lp);
-}
-
 // Warp-cooperative TMA of the 128-key tile starting at request-local key j0:
 // lane 0 posts the byte count, then copy c is issued by lane c. A copy is one
 // 64-dim half of the whole tile (contiguous cache: 2 copies) or of one page
-// (paged cache: 2 x 128/page copies, up to 32; `page` from tile_page), so a
-// paged tile costs one round of parallel copy issues.
+// (paged cache: 2 x 128/page copies, up to 32), so a paged tile costs one
+// round of parallel page-index loads and copy issues instead of a serial loop.
 __device__ __forceinline__ void load_tile(const RefArgs& a, const CUtensorMap* map, uint8_t* dst,
-                                          uint64_t* bar, int l, int g, int t0, int j0, int page,
+                                          uint64_t* bar, int l, int g, int r, int t0, int N, int j0,
                                           int lane) {
   const KvDev& kv = a.kv;
   if (lane == 0) tc::mbar_arrive_expect_tx(bar, kTileBytes);
@@ -232,6 +217,8 @@ __device__ __forceinline__ void load_tile(const RefArgs& a, const CUtensorMap* m
     const int ps = kv.page_size;
     const int i = lane >> 1;  // page of the tile
     if (i < kKT / ps) {
+      const int lp = min((j0 + i * ps) / ps, (N - 1) / ps);  // tail pages repeat the last one (masked)
+      const int page = kv.page_table[int64_t(r) * kv.max_pages + lp];
       const int32_t y = int32_t(((int64_t(l) * kv.num_pages + page) * kv.Hkv + g) * ps);
       tc::tma_load_2d(dst + hf * kTileHalf + i * ps * 128, map, bar, hf * 64, y);
     }
@@ -347,32 +334,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       if (u < 0) break;
-      // page indices go out a group of kPageAhead tiles ahead of their copies
-      int pg[kPageAhead], pg_next[kPageAhead];
-#pragma unroll
-      for (int j = 0; j < kPageAhead; ++j) pg[j] = j < nt ? tile_page(a, it.r, N, j * kKT, lane) : 0;
       for (int t = 0; t < nt; ++t, ++T) {
-        const int jj = t % kPageAhead;
-        if (jj == 0) {
-#pragma unroll
-          for (int j = 0; j < kPageAhead; ++j)
-            pg_next[j] = t + kPageAhead + j < nt ? tile_page(a, it.r, N, (t + kPageAhead + j) * kKT, lane) : 0;
-        }
-        int page = pg[0];
-#pragma unroll
-        for (int j = 1; j < kPageAhead; ++j)
-          if (jj == j) page = pg[j];
-        if (jj == kPageAhead - 1) {
-#pragma unroll
-          for (int j = 0; j < kPageAhead; ++j) pg[j] = pg_next[j];
-        }
         const int sk = T % kKStages;
         if (!__all_sync(0xffffffffu, wait_or_abort(&s.kempty[sk], ((T / kKStages) & 1) ^ 1, s.abort))) {
           if (lane == 0) raise_abort(a, s, tc::kSiteLoad);
           ok = false;
           break;
         }
-        load_tile(a, &kmap, s.k + sk * kTileBytes, &s.kfull[sk], it.l, it.g, t0, t * kKT, page, lane);
+        load_tile(a, &kmap, s.k + sk * kTileBytes, &s.kfull[sk], it.l, it.g, it.r, t0, N, t * kKT, lane);
         ++nk;
       }
     }
@@ -395,31 +364,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (lane == 0) tc::mbar_arrive(&s.qempty[qs]);  // this warp is done with the record
       if (u < 0) break;
       bool ok = true;
-      int pg[kPageAhead], pg_next[kPageAhead];
-#pragma unroll
-      for (int j = 0; j < kPageAhead; ++j) pg[j] = j < nt ? tile_page(a, r, N, j * kKT, lane) : 0;
       for (int t = 0; t < nt; ++t, ++T) {
-        const int jj = t % kPageAhead;
-        if (jj == 0) {
-#pragma unroll
-          for (int j = 0; j < kPageAhead; ++j)
-            pg_next[j] = t + kPageAhead + j < nt ? tile_page(a, r, N, (t + kPageAhead + j) * kKT, lane) : 0;
-        }
-        int page = pg[0];
-#pragma unroll
-        for (int j = 1; j < kPageAhead; ++j)
-          if (jj == j) page = pg[j];
-        if (jj == kPageAhead - 1) {
-#pragma unroll
-          for (int j = 0; j < kPageAhead; ++j) pg[j] = pg_next[j];
-        }
         const int sv = T % kVStages;
         if (!__all_sync(0xffffffffu, wait_or_abort(&s.vempty[sv], ((T / kVStages) & 1) ^ 1, s.abort))) {
           if (lane == 0) raise_abort(a, s, tc::kSiteLoad);
           ok = false;
           break;
         }
-        load_tile(a, &vmap, s.v + sv * kTileBytes, &s.vfull[sv], l, g, t0, t * kKT, page, lane);
+        load_tile(a, &vmap, s.v + sv * kTileBytes, &s.vfull[sv], l, g, r, t0, N, t * kKT, lane);
         ++nv;
       }
       if (!ok) break;

@@ -43,13 +43,11 @@ namespace {
 constexpr int kD = 128;
 constexpr int kTile = 128;
 constexpr int kStages = 3;                     // K ring
-constexpr int kPageAhead = 4;                  // paged caches: tiles whose page indices load ahead
 constexpr int kVBufs = 2;                      // V tiles (value norms, pass A)
 constexpr int kGroupRows = 256;
-constexpr int kThreads = 608;
-constexpr int kEpiThreads = 512;
-constexpr int kNormThreads = 256;              // epilogue threads that also take value norms
-constexpr int kVWarp = 18;                     // warps 2-17 are the epilogue
+constexpr int kThreads = 352;
+constexpr int kEpiThreads = 256;
+constexpr int kVWarp = 10;                     // warps 2-9 are the epilogue
 constexpr uint32_t kHalfQ = kGroupRows * 128;  // 32 KB: one 64-dim half of the row tile
 constexpr uint32_t kHalfK = kTile * 128;       // 16 KB
 constexpr uint32_t kStageBytes = 2 * kHalfK;   // 32 KB per K tile
@@ -64,7 +62,7 @@ struct TcArgs {
   int32_t n_units;
   int32_t rg_max;      // row groups per slab, maximum over requests (pa stride)
   float scale_log2;    // log2(e) / sqrt(d)
-  float* pa;           // [n_layers][Hkv][rg_max][4][n_tot] (four warp groups' column shares)
+  float* pa;           // [n_layers][Hkv][rg_max][2][n_tot]
   float* ss;           // [n_layers][Hkv][2][n_tot] sum of squares of V, per half of the head;
                        // NULL when the norms come from the side cache (V is not read)
   float* pa2;          // like pa, sums of alpha^2 (RMS statistic, Eq. 4), or NULL
@@ -185,26 +183,13 @@ __device__ __forceinline__ void epi_barrier() {
   asm volatile("bar.sync 1, %0;" ::"n"(kEpiThreads) : "memory");
 }
 
-// Page of K (or V) tile `tile` of unit w that lane `lane` copies (page
-// lane / 2 of the tile; 0 for a contiguous cache or a lane without a copy).
-// The producers fetch the pages of a group of tiles while they issue the
-// previous group's copies, so the page-table loads never hold back a copy.
-__device__ __forceinline__ int tile_page(const TcArgs& a, const Unit& w, int tile, int lane) {
-  const KvDev& kv = a.kv;
-  if (kv.page_size == 0) return 0;
-  const int ps = kv.page_size, i = lane >> 1;
-  if (i >= kTile / ps) return 0;
-  const int lp = min((tile * kTile + i * ps) / ps, (w.N - 1) / ps);  // tail pages repeat the last one (masked)
-  return __ldg(kv.page_table + int64_t(w.r) * kv.max_pages + lp);
-}
-
 // Warp-cooperative TMA of K (or V) tile `tile` of unit w into `dst`: lane 0
 // posts the byte count, then copy c is issued by lane c. A copy is one 64-dim
 // half of the whole tile (contiguous cache: 2 copies) or of one page (paged
-// cache: 2 x 128/page copies, up to 32; `page` from tile_page), so a paged
-// tile costs one round of parallel copy issues.
+// cache: 2 x 128/page copies, up to 32), so a paged tile costs one round of
+// parallel page-index loads and copy issues.
 __device__ __forceinline__ void load_k_tile(const TcArgs& a, const CUtensorMap* kmap, const Unit& w,
-                                            uint8_t* dst, uint64_t* bar, int tile, int page, int lane) {
+                                            uint8_t* dst, uint64_t* bar, int tile, int lane) {
   if (lane == 0) tc::mbar_arrive_expect_tx(bar, kStageBytes);
   __syncwarp();
   const int tok = tile * kTile;
@@ -219,6 +204,8 @@ __device__ __forceinline__ void load_k_tile(const TcArgs& a, const CUtensorMap* 
     const int ps = kv.page_size;
     const int i = lane >> 1;  // page of the tile
     if (i < kTile / ps) {
+      const int lp = min((tok + i * ps) / ps, (w.N - 1) / ps);  // tail pages repeat the last one (masked)
+      const int page = kv.page_table[int64_t(w.r) * kv.max_pages + lp];
       const int32_t y = int32_t(((int64_t(w.l) * kv.num_pages + page) * kv.Hkv + w.g) * ps);
       tc::tma_load_2d(dst + hf * kHalfK + i * ps * 128, kmap, bar, hf * 64, y);
     }
@@ -341,7 +328,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int i = 0; i < kVBufs; ++i) {
       tc::mbar_init(&s.vfull[i], 1);
-      tc::mbar_init(&s.vempty[i], kNormThreads);
+      tc::mbar_init(&s.vempty[i], kEpiThreads);
     }
     for (int i = 0; i < 2; ++i) {
       tc::mbar_init(&s.tfull[i], 1);
@@ -367,30 +354,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int u = blockIdx.x; u < a.n_units && ok; u += gridDim.x) {
       Unit w;
       if (!decode_unit(a, u, w)) continue;
-      // page indices go out a group of kPageAhead tiles ahead of their copies
-      const int n = 2 * w.tiles;
-      int pg[kPageAhead], pg_next[kPageAhead];
-#pragma unroll
-      for (int j = 0; j < kPageAhead; ++j) pg[j] = j < n ? tile_page(a, w, tile_of(w, j), lane) : 0;
-      for (int i0 = 0; i0 < n && ok; i0 += kPageAhead) {
-#pragma unroll
-        for (int j = 0; j < kPageAhead; ++j)
-          pg_next[j] = i0 + kPageAhead + j < n ? tile_page(a, w, tile_of(w, i0 + kPageAhead + j), lane) : 0;
-#pragma unroll
-        for (int j = 0; j < kPageAhead; ++j) {
-          const int i = i0 + j;
-          if (i >= n) break;
-          const int st = seq % kStages;
-          if (!__all_sync(0xffffffffu, wait_or_abort(&s.kempty[st], ((seq / kStages) & 1) ^ 1, s.abort))) {
-            if (lane == 0 && !*s.abort) raise_abort(a, s, tc::kSiteLoad);
-            ok = false;
-            break;
-          }
-          load_k_tile(a, &kmap, w, s.k + st * kStageBytes, &s.kfull[st], tile_of(w, i), pg[j], lane);
-          ++seq;
+      for (int i = 0; i < 2 * w.tiles; ++i, ++seq) {
+        const int st = seq % kStages;
+        if (!__all_sync(0xffffffffu, wait_or_abort(&s.kempty[st], ((seq / kStages) & 1) ^ 1, s.abort))) {
+          if (lane == 0 && !*s.abort) raise_abort(a, s, tc::kSiteLoad);
+          ok = false;
+          break;
         }
-#pragma unroll
-        for (int j = 0; j < kPageAhead; ++j) pg[j] = pg_next[j];
+        load_k_tile(a, &kmap, w, s.k + st * kStageBytes, &s.kfull[st], tile_of(w, i), lane);
       }
     }
     if (lane == 0) s.counters[0] = seq;
@@ -403,24 +374,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int u = blockIdx.x; u < a.n_units && ok; u += gridDim.x) {
       Unit w;
       if (!decode_unit(a, u, w) || w.rg != 0) continue;
-      int pg[kPageAhead], pg_next[kPageAhead];
-#pragma unroll
-      for (int j = 0; j < kPageAhead; ++j) pg[j] = j < w.tiles ? tile_page(a, w, j, lane) : 0;
       for (int i = 0; i < w.tiles; ++i, ++vseq) {
-        const int jj = i % kPageAhead;
-        if (jj == 0) {  // page indices of the next group of tiles go out now
-#pragma unroll
-          for (int j = 0; j < kPageAhead; ++j)
-            pg_next[j] = i + kPageAhead + j < w.tiles ? tile_page(a, w, i + kPageAhead + j, lane) : 0;
-        }
-        int page = pg[0];
-#pragma unroll
-        for (int j = 1; j < kPageAhead; ++j)
-          if (jj == j) page = pg[j];
-        if (jj == kPageAhead - 1) {
-#pragma unroll
-          for (int j = 0; j < kPageAhead; ++j) pg[j] = pg_next[j];
-        }
         const int vb = vseq % kVBufs;
         if (!__all_sync(0xffffffffu, wait_or_abort(&s.vempty[vb], ((vseq / kVBufs) & 1) ^ 1, s.abort))) {
           if (lane == 0 && !*s.abort) raise_abort(a, s, tc::kSiteLoad);
@@ -433,7 +387,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           continue;
         }
 #endif
-        load_k_tile(a, &vmap, w, s.v + vb * kStageBytes, &s.vfull[vb], i, page, lane);
+        load_k_tile(a, &vmap, w, s.v + vb * kStageBytes, &s.vfull[vb], i, lane);
       }
     }
     if (lane == 0) s.counters[2] = vseq;
@@ -501,8 +455,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------------------ epilogue
     // After an abort the epilogue keeps walking its units (skipping the work)
     // so that every thread reaches every named barrier.
-    const int et = tid - 64;                       // 0..511
-    const int grp = et >> 7;                       // warp group 0..3 (four warps per lane quarter)
+    const int et = tid - 64;                       // 0..255
+    const int h = et >> 7;                         // warp group: column half or row block
     const int quarter = warp & 3;                  // TMEM lanes 32*quarter .. +31
     const int lrow = quarter * 32 + lane;          // row (pass A) / token (pass B) in the tile
     const uint32_t lane_base = uint32_t(quarter * 32) << 16;
@@ -513,10 +467,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t zero[64];
 #pragma unroll
       for (int i = 0; i < 64; ++i) zero[i] = 0u;
-      for (int c = grp * 128; c < grp * 128 + 128; c += 64) tc::tmem_st64(tmem + lane_base + c, zero);
+      for (int c = h * 256; c < h * 256 + 256; c += 64) tc::tmem_st64(tmem + lane_base + c, zero);
       tc::tc_fence_before();
     }
-    float2* xch = reinterpret_cast<float2*>(s.lse);  // 128 (m, z) pairs while pass A's parts merge
     for (int u = blockIdx.x; u < a.n_units; u += gridDim.x) {
       Unit w;
       if (!decode_unit(a, u, w)) continue;
@@ -525,17 +478,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::fence_proxy_async_smem();
       epi_barrier();
       if (et == 0) tc::mbar_arrive(s.qready);
-      // pass A share: two row blocks -> block grp / 2, keys [64 (grp % 2), +64)
-      // of each tile; one row block -> keys [32 grp, +32). Groups 0 and 1 also
-      // take half grp of each V row of the tile for the value norms.
-      const int rb = nrb == 2 ? grp >> 1 : 0;
-      const int kc0 = nrb == 2 ? (grp & 1) * 64 : grp * 32;
-      const int nkc = nrb == 2 ? 2 : 1;  // 32-key chunks per tile
-      const int row = rb * 128 + lrow;
-      const bool live = __any_sync(0xffffffffu, row < w.rows);  // warps of padding rows skip the stats
-      const bool do_norm = grp < 2 && w.rg == 0 && a.ss != nullptr;  // one row group of each slab also streams V
+      // pass A share: row block rb (with one row block the second warp group
+      // only does value norms) and this thread's half of each V row
+      const bool do_rows = nrb == 2 || h == 0;
+      const int rb = nrb == 2 ? h : 0;
+      const bool do_norm = w.rg == 0 && a.ss != nullptr;  // one row group of each slab also streams V
       const int64_t lg = int64_t(w.li) * a.kv.Hkv + w.g;
-      float* ss_out = do_norm ? a.ss + (lg * 2 + grp) * n_tot + w.t0 : nullptr;
+      float* ss_out = do_norm ? a.ss + (lg * 2 + h) * n_tot + w.t0 : nullptr;
       float m = -INFINITY, z = 0.f;
       for (int i = 0; i < w.tiles; ++i) {            // pass A
         const int slot = tseq & 1;
@@ -548,22 +497,16 @@ __global__ void __launch_bounds__(kThreads, 1)
           continue;
         }
         tc::tc_fence_after();
-        const uint32_t col0 = uint32_t(slot) * kSlotCols + rb * 128 + kc0;
-        const int valid = w.N - i * kTile - kc0;
-        if (live) {  // the slot is free again after this thread's last load
-          float v[32];
-          tc::tmem_ld32(tmem + lane_base + col0, v);
-          if (nkc == 1) {
-            tc::tc_fence_before();
-            tc::mbar_arrive(&s.tempty[slot]);
-          }
-          row_stats<32>(v, valid, a.scale_log2, m, z);
-          if (nkc == 2) {
-            tc::tmem_ld32(tmem + lane_base + col0 + 32, v);
-            tc::tc_fence_before();
-            tc::mbar_arrive(&s.tempty[slot]);
-            row_stats<32>(v, valid - 32, a.scale_log2, m, z);
-          }
+        const uint32_t col0 = uint32_t(slot) * kSlotCols + rb * 128;
+        const int valid = w.N - i * kTile;
+        if (do_rows) {  // 128 columns in two loads; the slot is free again after the second
+          float v[64];
+          tc::tmem_ld64(tmem + lane_base + col0, v);
+          row_stats<64>(v, valid, a.scale_log2, m, z);
+          tc::tmem_ld64(tmem + lane_base + col0 + 64, v);
+          tc::tc_fence_before();
+          tc::mbar_arrive(&s.tempty[slot]);
+          row_stats<64>(v, valid - 64, a.scale_log2, m, z);
         } else {
           tc::tc_fence_before();
           tc::mbar_arrive(&s.tempty[slot]);
@@ -576,7 +519,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             continue;
           }
           ++vcons;
-          const uint8_t* vh = s.v + vb * kStageBytes + grp * kHalfK;
+          const uint8_t* vh = s.v + vb * kStageBytes + h * kHalfK;
           float sq[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
           for (int c = 0; c < 8; ++c)
@@ -586,47 +529,26 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (tok < w.N) ss_out[tok] = sumsq_combine(sq);
         }
       }
-      // each row's parts (two with two row blocks, four with one) merge, in a
-      // fixed order, into the group that holds the row's first keys, one part
-      // at a time through the 1 KB row buffer
-      epi_barrier();
-      const bool owner = nrb == 2 ? (grp & 1) == 0 : grp == 0;
-      for (int part = 1; part < (nrb == 2 ? 2 : 4); ++part) {
-        const bool sender = nrb == 2 ? (grp & 1) == part : grp == part;
-        // with two row blocks the two blocks go one after the other (the buffer holds 128 rows)
-        for (int blk = 0; blk < nrb; ++blk) {
-          if (sender && rb == blk) xch[lrow] = make_float2(m, z);
-          epi_barrier();
-          if (owner && rb == blk) {
-            const float2 o = xch[lrow];
-            const float mn = fmaxf(m, o.x);
-            if (mn != -INFINITY) {
-              z = z * tc::ex2((m - mn) * a.scale_log2) + o.y * tc::ex2((o.x - mn) * a.scale_log2);
-              m = mn;
-            }
-          }
-          epi_barrier();
-        }
-      }
       // minus the log2-sum-exp of each row, shared with the token-owning
       // threads of pass B (-inf past the row group: those columns add nothing)
-      if (owner || (nrb == 1 && grp == 1)) {
-        const int r = (owner ? rb : 1) * 128 + lrow;
-        float lse = (owner && r < w.rows) ? m * a.scale_log2 + log2f(z) : INFINITY;
-        if (a.extra_lse != nullptr && owner && r < w.rows) {
+      {
+        const int row = (do_rows ? rb : 1) * 128 + lrow;
+        float lse = (do_rows && row < w.rows) ? m * a.scale_log2 + log2f(z) : INFINITY;
+        if (a.extra_lse != nullptr && do_rows && row < w.rows) {
           // full-context softmax: the keys outside the visual span join the denominator
-          const int j = w.row0 + r, hq = w.g * a.kv.G + j / w.nq, qi = j % w.nq;
+          const int j = w.row0 + row, hq = w.g * a.kv.G + j / w.nq, qi = j % w.nq;
           const float e = a.extra_lse[(int64_t(w.l) * a.kv.Hq + hq) * a.q_tot + w.q0 + qi];
           lse = log2_add(lse, e * kLog2e);
         }
-        s.lse[r] = -lse;
+        s.lse[row] = -lse;
       }
       epi_barrier();
-      // pass B share: 16-column chunks [c16_0, c16_1) of the group's rows
-      const int nc16 = (w.rows + 15) / 16;
-      const int c16_0 = (nc16 * grp) / 4, c16_1 = (nc16 * (grp + 1)) / 4;
-      float* pa_out = a.pa + ((lg * a.rg_max + w.rg) * 4 + grp) * n_tot + w.t0;
-      float* pa2_out = a.pa2 ? a.pa2 + ((lg * a.rg_max + w.rg) * 4 + grp) * n_tot + w.t0 : nullptr;
+      // pass B share: 32-row chunks [cb0, cb1)
+      const int nchunk = (w.rows + 31) / 32;
+      const int hc = (nchunk + 1) / 2;
+      const int cb0 = h * hc, cb1 = min(nchunk, cb0 + hc);
+      float* pa_out = a.pa + ((lg * a.rg_max + w.rg) * 2 + h) * n_tot + w.t0;
+      float* pa2_out = a.pa2 ? a.pa2 + ((lg * a.rg_max + w.rg) * 2 + h) * n_tot + w.t0 : nullptr;
       for (int i = w.tiles; i < 2 * w.tiles; ++i) {  // pass B
         const int slot = tseq & 1;
         const int tok = tile_of(w, i) * kTile + lrow;
@@ -639,40 +561,41 @@ __global__ void __launch_bounds__(kThreads, 1)
           continue;
         }
         tc::tc_fence_after();
-        // this thread's columns in loads of 32 (and one of 16); the slot is
-        // free again after the last load
-        const uint32_t col0 = uint32_t(slot) * kSlotCols;
-        const int cend = c16_1 * 16;
+        // this thread's columns [32 cb0, 32 cb1) in loads of 64 (and one of 32);
+        // the slot is free again after the last load
+        const uint32_t col0 = uint32_t(slot) * kSlotCols + cb0 * 32;
+        const int ncol = (cb1 - cb0) * 32;
+        const float* lse = s.lse + cb0 * 32;
         float acc = 0.f, acc2 = 0.f;
-        int c = c16_0 * 16;
-        for (; c + 32 <= cend; c += 32) {
-          float v[32];
-          tc::tmem_ld32(tmem + lane_base + col0 + c, v);
-          if (c + 32 == cend) {
+        int c = 0;
+        for (; c + 64 <= ncol; c += 64) {
+          float v[64];
+          tc::tmem_ld64(tmem + lane_base + col0 + c, v);
+          if (c + 64 == ncol) {
             tc::tc_fence_before();
             tc::mbar_arrive(&s.tempty[slot]);
           }
           if (pa2_out) {
             float q2;
-            acc += col_sum_sq<32>(v, s.lse + c, a.scale_log2, q2);
+            acc += col_sum_sq<64>(v, lse + c, a.scale_log2, q2);
             acc2 += q2;
           } else {
-            acc += col_sum<32>(v, s.lse + c, a.scale_log2);
+            acc += col_sum<64>(v, lse + c, a.scale_log2);
           }
         }
-        if (c < cend) {  // one 16-column chunk left
-          float v[16];
-          tc::tmem_ld16(tmem + lane_base + col0 + c, v);
+        if (c < ncol) {
+          float v[32];
+          tc::tmem_ld32(tmem + lane_base + col0 + c, v);
           tc::tc_fence_before();
           tc::mbar_arrive(&s.tempty[slot]);
           if (pa2_out) {
             float q2;
-            acc += col_sum_sq<16>(v, s.lse + c, a.scale_log2, q2);
+            acc += col_sum_sq<32>(v, lse + c, a.scale_log2, q2);
             acc2 += q2;
           } else {
-            acc += col_sum<16>(v, s.lse + c, a.scale_log2);
+            acc += col_sum<32>(v, lse + c, a.scale_log2);
           }
-        } else if (c16_0 == c16_1) {  // no columns for this group
+        } else if (ncol == 0) {
           tc::tc_fence_before();
           tc::mbar_arrive(&s.tempty[slot]);
         }
