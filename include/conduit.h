@@ -273,6 +273,39 @@ conduit_status conduit_select_topk(const conduit_batch* batch, const float* s, c
                                    void* stream);
 
 /*
+ * Scoring and the global selection in one call (Sec. 3.3-3.5, Eqs. 6-11;
+ * Algorithm 1 from the scoring loops to the top-k): the results of
+ * conduit_score_ex(kv, batch, q, layers, n_layers, opts, s, attn_sum, g, ...)
+ * followed by conduit_select_topk(batch, s, g, lambda, idx_off, idx_off_dev,
+ * idx, mask, s_hat, coeff, ...), bit for bit, with fewer launches: when every
+ * request holds at most 8192 tokens and the batch at most 32 tokens per SM of
+ * the device (4 864 on a 152-SM GPU), the per-token reductions (s_t, A_t),
+ * the image means g_j, c_j, s_hat and the top-k run as one launch after the
+ * scoring kernel (the last block to finish a request's tokens selects that
+ * request); other batches take the separate launches of the two calls.
+ * Arguments, layouts and ownership are those of the two calls (opts may be
+ * NULL: the defaults; attn_sum may be NULL).
+ *  workspace  device, 256-byte aligned,
+ *             conduit_score_select_topk_workspace_size bytes
+ * Errors: the union of the two calls' (INVALID_ARG, UNSUPPORTED, WORKSPACE,
+ * CUDA); nothing is enqueued when the arguments are rejected. status: the
+ * bits either call sets (NONFINITE; TIMEOUT from the scoring kernel).
+ */
+conduit_status conduit_score_select_topk_workspace_size(const conduit_kv* kv,
+                                                        const conduit_batch* batch,
+                                                        int32_t n_layers,
+                                                        const conduit_score_opts* opts,
+                                                        size_t* bytes);
+conduit_status conduit_score_select_topk(const conduit_kv* kv, const conduit_batch* batch,
+                                         const void* q, const int32_t* layers, int32_t n_layers,
+                                         const conduit_score_opts* opts, float lambda,
+                                         const int32_t* idx_off, const int32_t* idx_off_dev,
+                                         float* s, float* attn_sum, float* g, int32_t* idx,
+                                         uint8_t* mask, float* s_hat, float* coeff,
+                                         void* workspace, size_t workspace_bytes, int32_t* status,
+                                         void* stream);
+
+/*
  * Explicit per-image quotas instead of the global ranking (App. D.3: the
  * "explicit" variant of the cross-image diagnostic, compared there with the
  * deployed global rule). Per request, with c_j of conduit_select_topk:

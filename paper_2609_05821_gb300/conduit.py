@@ -88,6 +88,9 @@ def _load():
         "conduit_value_norms_update": (st, [P, P, P, P, P, P, P]),
         "conduit_score_with_norms_workspace_size": (st, [P, P, I32, ctypes.POINTER(SZ)]),
         "conduit_score_with_norms": (st, [P, P, P, P, I32, P, P, P, P, P, SZ, P, P]),
+        "conduit_score_select_topk_workspace_size": (st, [P, P, I32, P, ctypes.POINTER(SZ)]),
+        "conduit_score_select_topk": (st, [P, P, P, P, I32, P, ctypes.c_float, P, P, P, P, P, P, P, P,
+                                           P, P, SZ, P, P]),
         "conduit_select_workspace_size": (st, [P, ctypes.POINTER(SZ)]),
         "conduit_select_topk": (st, [P, P, P, ctypes.c_float, P, P, P, P, P, P, P, SZ, P, P]),
         "conduit_select_topk_noalloc": (st, [P, P, P, ctypes.c_float, P, P, P, P, P, P, P, P]),
@@ -286,6 +289,40 @@ def conduit_score_ex(kv: KvCache, batch: Batch, q: torch.Tensor, layers=None, st
                                  _ptr(s), _ptr(attn_sum), _ptr(g), _ptr(ws), ws.numel(),
                                  _ptr(status), _stream_ptr(stream)))
     return s, attn_sum, g
+
+
+def conduit_score_select_topk_workspace_size(kv: KvCache, batch: Batch, n_layers: int = 0,
+                                             opts: Optional[ConduitScoreOpts] = None) -> int:
+    n = ctypes.c_size_t(0)
+    _check(_lib.conduit_score_select_topk_workspace_size(kv.ref(), batch.ref(), int(n_layers),
+                                                         None if opts is None else ctypes.byref(opts),
+                                                         ctypes.byref(n)))
+    return int(n.value)
+
+
+def conduit_score_select_topk(kv: KvCache, batch: Batch, q: torch.Tensor, lam: float,
+                              idx_off: torch.Tensor, idx_off_dev: torch.Tensor, layers=None,
+                              statistic="mean", value_norm="v", vnorm=None, extra_lse=None, s=None,
+                              attn_sum=None, g=None, idx=None, mask=None, s_hat=None, coeff=None,
+                              workspace=None, status=None, stream=None):
+    """Scoring and global top-k in one call (Eqs. 6-11): conduit_score_ex then
+    conduit_select_topk, bitwise, in fewer launches.
+    Returns (s, attn_sum, g, idx, mask, s_hat, coeff)."""
+    dev = kv.k.device
+    larr, nl = _layer_array(layers)
+    opts = score_opts(statistic, value_norm, vnorm, extra_lse)
+    s = torch.empty(batch.n_tot, dtype=torch.float32, device=dev) if s is None else s
+    attn_sum = torch.empty(batch.n_tot, dtype=torch.float32, device=dev) if attn_sum is None else attn_sum
+    g = torch.empty(batch.num_images, dtype=torch.float32, device=dev) if g is None else g
+    n_sel = int(idx_off[-1])
+    idx = torch.empty(max(n_sel, 1), dtype=torch.int32, device=dev) if idx is None else idx
+    ws = _workspace(conduit_score_select_topk_workspace_size(kv, batch, nl, opts), dev, workspace)
+    _check(_lib.conduit_score_select_topk(kv.ref(), batch.ref(), _ptr(q), larr, nl, ctypes.byref(opts),
+                                          float(lam), _ptr(idx_off), _ptr(idx_off_dev), _ptr(s),
+                                          _ptr(attn_sum), _ptr(g), _ptr(idx), _ptr(mask), _ptr(s_hat),
+                                          _ptr(coeff), _ptr(ws), ws.numel(), _ptr(status),
+                                          _stream_ptr(stream)))
+    return s, attn_sum, g, idx[:n_sel], mask, s_hat, coeff
 
 
 def conduit_staleness_iso_workspace_size(kv: KvCache, batch: Batch, M: int) -> int:

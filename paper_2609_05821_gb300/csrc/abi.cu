@@ -258,13 +258,46 @@ conduit_status check_norm_cache(const conduit_kv* kv, const float* vnorm) {
 }
 
 // Every scoring entry point: conduit_score_ex with the options read into `mode`.
+// The selection that conduit_score_select_topk appends to a scoring call.
+struct SelectTail {
+  float lambda;
+  const int32_t* idx_off;      // host prefix sums of the budgets
+  const int32_t* idx_off_dev;  // the same on the device
+  int32_t* idx;
+  uint8_t* mask;
+  float* s_hat;
+  float* coeff;
+};
+
+// Workspace of conduit_score_select_topk: the scoring call's, then one
+// arrival counter per request (fused tail) and the selection's keys (the
+// separate launches, for requests of more than 8192 tokens).
+struct FusedLayout {
+  ScoreLayout score;
+  size_t arrivals, keys, total;
+};
+
+FusedLayout fused_layout(const conduit_kv* kv, const conduit_batch* b, int n_layers, const ScoreMode& mode) {
+  FusedLayout f;
+  f.score = score_layout(kv, b, n_layers, mode);
+  f.arrivals = f.score.total;
+  f.keys = f.arrivals + align_up(size_t(b->num_requests) * sizeof(int32_t));
+  f.total = f.keys + align_up(size_t(b->tok_off[b->num_requests]) * sizeof(uint32_t));
+  return f;
+}
+
 conduit_status score_impl(const conduit_kv* kv, const conduit_batch* batch, const void* q,
                           const int32_t* layers, int32_t n_layers, const ScoreMode& mode, float* s,
                           float* attn_sum, float* g, void* workspace, size_t workspace_bytes,
-                          int32_t* status, void* stream) {
+                          int32_t* status, void* stream, const SelectTail* tail = nullptr) {
   conduit_status st;
   if ((st = check_batch(batch)) || (st = check_kv(kv, batch))) return st;
   if (!q || !s || !g) return fail(CONDUIT_ERR_INVALID_ARG, "q, s and g are required");
+  if (tail) {
+    if (!(tail->lambda >= 0.f && tail->lambda <= 1.f))
+      return fail(CONDUIT_ERR_INVALID_ARG, "lambda must lie in [0, 1]");
+    if ((st = check_selection(batch, tail->idx_off, tail->idx_off_dev, true, tail->idx))) return st;
+  }
   if (!aligned16(q)) return fail(CONDUIT_ERR_INVALID_ARG, "q must be 16-byte aligned");
   for (int r = 0; r < batch->num_requests; ++r)
     if (batch->q_off[r + 1] == batch->q_off[r])
@@ -273,8 +306,9 @@ conduit_status score_impl(const conduit_kv* kv, const conduit_batch* batch, cons
   if ((st = make_layers(kv, layers, n_layers, &ll))) return st;
   const bool normed = mode.vmode != 0;
   if (mode.vmode == 1 && (st = check_norm_cache(kv, mode.vnorm))) return st;
-  const ScoreLayout lay = score_layout(kv, batch, ll.n, mode);
-  if ((st = check_workspace(workspace, workspace_bytes, lay.total))) return st;
+  const FusedLayout flay = fused_layout(kv, batch, ll.n, mode);
+  const ScoreLayout& lay = flay.score;
+  if ((st = check_workspace(workspace, workspace_bytes, tail ? flay.total : lay.total))) return st;
 
   const KvDev kd = make_kv(kv, batch);
   const BatchDev bd = make_batch(batch);
@@ -292,6 +326,10 @@ conduit_status score_impl(const conduit_kv* kv, const conduit_batch* batch, cons
   float* attn = attn_sum ? attn_sum : reinterpret_cast<float*>(ws + lay.attn);
   cudaStream_t cs = static_cast<cudaStream_t>(stream);
   cudaError_t err;
+  const bool fused = tail && finalize_select_supported(max_tok, kd.n_tot);
+  int32_t* arrivals = reinterpret_cast<int32_t*>(ws + flay.arrivals);
+  if (fused && (err = cudaMemsetAsync(arrivals, 0, size_t(R) * sizeof(int32_t), cs)))
+    return cuda_fail(err, "score_select");
   if (lay.tc) {  // the tensor-core kernel also streams V for the value norms (unless normed)
     err = launch_score_tc(kd, bd, batch->q_off, q, batch->q_off[R], ll, lay.rg_max, pa, ss, pa2,
                           mode.extra_lse, status, cs);
@@ -302,9 +340,21 @@ conduit_status score_impl(const conduit_kv* kv, const conduit_batch* batch, cons
                             mode.extra_lse, cs);
   }
   if (err) return cuda_fail(err, "score");
+  if (fused) {
+    if ((err = launch_finalize_select(pa, pa2, ss, mode.vnorm, mode.vmode, ll, bd, ll.n, kd.Hkv, kd.Hq,
+                                      lay.rg_max, lay.group_rows, lay.parts, kd.n_tot, max_tok, s, attn, g,
+                                      tail->lambda, tail->idx_off_dev, tail->idx, tail->mask, tail->s_hat,
+                                      tail->coeff, arrivals, status, cs)))
+      return cuda_fail(err, "finalize_select");
+    return CONDUIT_OK;
+  }
   if ((err = launch_finalize(pa, pa2, ss, mode.vnorm, mode.vmode, ll, bd, ll.n, kd.Hkv, kd.Hq,
                              lay.rg_max, lay.group_rows, lay.parts, kd.n_tot, s, attn, g, status, cs)))
     return cuda_fail(err, "finalize");
+  if (tail &&
+      (err = launch_select(bd, max_tok, s, g, tail->lambda, tail->idx_off_dev, tail->idx, tail->mask,
+                           tail->s_hat, tail->coeff, reinterpret_cast<uint32_t*>(ws + flay.keys), status, cs)))
+    return cuda_fail(err, "select");
   return CONDUIT_OK;
 }
 
@@ -369,6 +419,37 @@ conduit_status conduit_score_ex(const conduit_kv* kv, const conduit_batch* batch
   if ((st = read_opts(opts, &mode))) return st;
   return score_impl(kv, batch, q, layers, n_layers, mode, s, attn_sum, g, workspace,
                     workspace_bytes, status, stream);
+}
+
+conduit_status conduit_score_select_topk_workspace_size(const conduit_kv* kv,
+                                                        const conduit_batch* batch,
+                                                        int32_t n_layers,
+                                                        const conduit_score_opts* opts,
+                                                        size_t* bytes) {
+  conduit_status st;
+  if (!bytes) return fail(CONDUIT_ERR_INVALID_ARG, "bytes is NULL");
+  if ((st = check_batch(batch)) || (st = check_kv(kv, batch))) return st;
+  ScoreMode mode;
+  if ((st = read_opts(opts, &mode))) return st;
+  const int nl = n_layers > 0 ? n_layers : kv->num_layers;
+  *bytes = fused_layout(kv, batch, nl, mode).total;
+  return CONDUIT_OK;
+}
+
+conduit_status conduit_score_select_topk(const conduit_kv* kv, const conduit_batch* batch,
+                                         const void* q, const int32_t* layers, int32_t n_layers,
+                                         const conduit_score_opts* opts, float lambda,
+                                         const int32_t* idx_off, const int32_t* idx_off_dev,
+                                         float* s, float* attn_sum, float* g, int32_t* idx,
+                                         uint8_t* mask, float* s_hat, float* coeff,
+                                         void* workspace, size_t workspace_bytes, int32_t* status,
+                                         void* stream) {
+  conduit_status st;
+  ScoreMode mode;
+  if ((st = read_opts(opts, &mode))) return st;
+  const SelectTail tail{lambda, idx_off, idx_off_dev, idx, mask, s_hat, coeff};
+  return score_impl(kv, batch, q, layers, n_layers, mode, s, attn_sum, g, workspace, workspace_bytes,
+                    status, stream, &tail);
 }
 
 conduit_status conduit_value_norms(const conduit_kv* kv, const conduit_batch* batch, float* vnorm,

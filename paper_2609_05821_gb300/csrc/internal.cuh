@@ -183,6 +183,19 @@ cudaError_t launch_select(const BatchDev& b, int max_tokens, const float* s, con
                           float lambda, const int32_t* idx_off_dev, int32_t* idx, uint8_t* mask,
                           float* s_hat, float* coeff, uint32_t* keys, int32_t* status,
                           cudaStream_t stream, bool cluster_ok = true);
+// The scoring tail and the global selection in one launch
+// (conduit_score_select_topk): launch_finalize's reductions followed by
+// launch_select's top-k, for batches whose largest request has at most
+// 8 x 1024 tokens and whose 32-token blocks fit one wave of the current
+// device's SMs (finalize_select_supported). arrivals: one int per request,
+// zero when the kernel starts.
+bool finalize_select_supported(int max_tokens, int64_t n_tot);
+cudaError_t launch_finalize_select(const float* pa, const float* pa2, const float* ss, const float* vnorm,
+                                   int vmode, const LayerList& layers, const BatchDev& b, int n_layers,
+                                   int Hkv, int Hq, int rg_max, int group_rows, int parts, int64_t n_tot,
+                                   int max_tokens, float* s, float* attn_sum, float* g, float lambda,
+                                   const int32_t* idx_off_dev, int32_t* idx, uint8_t* mask, float* s_hat,
+                                   float* coeff, int32_t* arrivals, int32_t* status, cudaStream_t stream);
 // Explicit per-image quotas (App. D.3): quota_kernel per request, then one
 // selection CTA per image. scratch holds quota_scratch_bytes(K) bytes.
 size_t quota_scratch_bytes(int total_images);

@@ -17,6 +17,7 @@
 #include <mutex>
 
 #include "internal.cuh"
+#include "token_reduce.cuh"
 
 namespace conduit {
 namespace {
@@ -29,7 +30,7 @@ constexpr int kQuotaThreads = 256;
 //   g_bar = (((g_0 + g_1) + g_2) + ...) / K,  c_j = (1 - lambda) + lambda (g_j / g_bar).
 __device__ __forceinline__ float image_mean_f32(const float* g, int K) {
   float sum = 0.f;
-  for (int j = 0; j < K; ++j) sum = __fadd_rn(sum, g[j]);
+  for (int j = 0; j < K; ++j) sum = __fadd_rn(sum, __ldcg(g + j));
   return __fdiv_rn(sum, float(K));
 }
 __device__ __forceinline__ float image_coefficient(float gj, float gbar, float lambda, int K) {
@@ -65,22 +66,24 @@ __device__ __forceinline__ int block_exclusive_scan(int v, int* warp_s, int* tot
   return before;
 }
 
-// Segment selection. kQuota = false: one CTA per request, keys s_hat = s c_pi(t),
-// budget k_r (Eqs. 10-11). kQuota = true: one CTA per image j, keys s_t,
-// budget quota[j], output at the request's slice + qoff[j] (App. D.3).
+// Segment selection by one CTA of kSelThreads threads. kQuota = false:
+// segment = request `seg`, keys s_hat = s c_pi(t), budget k_r (Eqs. 10-11).
+// kQuota = true: segment = image `seg`, keys s_t, budget quota[j], output at
+// the request's slice + qoff[j] (App. D.3). s and g are read through L2, so
+// the fused scoring tail can select a request whose scores other blocks of
+// the same launch wrote.
 template <int kRegKeys, bool kQuota>  // keys a thread keeps in registers (0: keys in the workspace)
-__global__ void __launch_bounds__(kSelThreads) select_kernel(BatchDev b, const float* s,
-                                                             const float* g, float lambda,
-                                                             const int32_t* idx_off, int32_t* idx,
-                                                             uint8_t* mask, float* s_hat,
-                                                             float* coeff, uint32_t* keys,
-                                                             int32_t* status,
-                                                             const float* seg_coeff,
-                                                             const int32_t* seg_quota,
-                                                             const int32_t* seg_qoff) {
+__device__ __forceinline__ void select_segment(int seg, const BatchDev& b, const float* s,
+                                               const float* g, float lambda, const int32_t* idx_off,
+                                               int32_t* idx, uint8_t* mask, float* s_hat,
+                                               float* coeff, uint32_t* keys, int32_t* status,
+                                               const float* seg_coeff, const int32_t* seg_quota,
+                                               const int32_t* seg_qoff, const float* mean_attn = nullptr,
+                                               float* mean_g = nullptr, int mean_layers = 0) {
   __shared__ float c_s[kMaxImagesPerRequest];
   __shared__ int img_s[kMaxImagesPerRequest + 1];
   __shared__ unsigned hist[256];
+  __shared__ float mean_s[kMeanThreads / 32];
   __shared__ int warp_s[32];
   __shared__ uint32_t prefix_s;
   __shared__ int remaining_s;
@@ -89,8 +92,8 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(BatchDev b, const f
   int t0, N, k, K, base_t;
   int32_t* out;
   float c_seg = 1.f;
-  if (kQuota) {  // segment = image blockIdx.x
-    const int j = blockIdx.x;
+  if (kQuota) {  // segment = image seg
+    const int j = seg;
     const int r = request_of(b.req_img_off, b.R, j);
     t0 = b.img_off[j];
     N = b.img_off[j + 1] - t0;
@@ -99,36 +102,66 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(BatchDev b, const f
     base_t = t0 - b.tok_off[r];  // request-local index of the image's first token
     out = idx + idx_off[r] + seg_qoff[j];
     c_seg = seg_coeff[j];
-  } else {       // segment = request blockIdx.x
-    const int r = blockIdx.x;
+  } else {       // segment = request seg
+    const int r = seg;
     t0 = b.tok_off[r];
     N = b.tok_off[r + 1] - t0;
-    const int j0 = b.req_img_off[r];
-    K = b.req_img_off[r + 1] - j0;
+    K = b.req_img_off[r + 1] - b.req_img_off[r];
     k = idx_off[r + 1] - idx_off[r];
     base_t = 0;
     out = idx + idx_off[r];
-    // c_j (Eq. 9): g_bar in a fixed order by one thread.
-    for (int j = threadIdx.x; j <= K; j += blockDim.x) img_s[j] = b.img_off[j0 + j] - t0;
-    if (threadIdx.x == 0) gbar_s = image_mean_f32(g + j0, K);
-    __syncthreads();
-    const float gbar = gbar_s;
-    for (int j = threadIdx.x; j < K; j += blockDim.x) {
-      const float c = image_coefficient(g[j0 + j], gbar, lambda, K);
-      c_s[j] = c;
-      if (coeff) coeff[j0 + j] = c;
-    }
-    __syncthreads();
   }
 
   // s_hat (Eq. 10) and its sortable key (s itself in quota mode, where c_j is
   // constant over the segment and decides only the quota). Each thread owns the contiguous
   // tokens [lo, hi); up to kRegKeys of them stay in registers for the radix
   // passes (requests of up to 1024 x kRegKeys tokens), otherwise the keys go
-  // through the workspace.
+  // through the workspace. The scores held in registers are loaded before
+  // c_j is formed, so the two loads overlap.
   const int per = (N + kSelThreads - 1) / kSelThreads;
   const int lo = min(N, int(threadIdx.x) * per), hi = min(N, lo + per);
   const bool in_regs = kRegKeys > 0 && per <= kRegKeys;
+  float sv[kRegKeys > 0 ? kRegKeys : 1];
+  if (in_regs) {
+#pragma unroll
+    for (int j = 0; j < kRegKeys; ++j) sv[j] = lo + j < hi ? __ldcg(s + t0 + lo + j) : 0.f;
+  }
+  if (!kQuota && K == 1) {  // one image: c = 1 exactly (Sec. 3.5), the span is the request
+    // With mean_attn, g of the image (Eq. 8) is formed here too, in the order
+    // of image_mean_group, its loads in flight with the scores' above.
+    float macc = 0.f;
+    if (mean_attn && threadIdx.x < kMeanThreads) {
+      for (int t = int(threadIdx.x); t < N; t += kMeanThreads) macc += __ldcg(mean_attn + t0 + t);
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) macc += __shfl_xor_sync(0xffffffffu, macc, o);
+      if ((threadIdx.x & 31) == 0) mean_s[threadIdx.x >> 5] = macc;
+    }
+    if (threadIdx.x == 0) {
+      img_s[0] = 0;
+      img_s[1] = N;
+      c_s[0] = 1.f;
+      if (coeff) coeff[b.req_img_off[seg]] = 1.f;
+    }
+    __syncthreads();
+    if (mean_attn && threadIdx.x == 0) {
+      float tot = 0.f;
+      for (int w = 0; w < kMeanThreads / 32; ++w) tot += mean_s[w];
+      *mean_g = tot / (float(mean_layers) * float(N));
+    }
+  } else if (!kQuota) {
+    // c_j (Eq. 9): g_bar in a fixed order by one thread
+    const int j0 = b.req_img_off[seg];
+    for (int j = threadIdx.x; j <= K; j += blockDim.x) img_s[j] = b.img_off[j0 + j] - t0;
+    if (threadIdx.x == 0) gbar_s = image_mean_f32(g + j0, K);
+    __syncthreads();
+    const float gbar = gbar_s;
+    for (int j = threadIdx.x; j < K; j += blockDim.x) {
+      const float c = image_coefficient(__ldcg(g + j0 + j), gbar, lambda, K);
+      c_s[j] = c;
+      if (coeff) coeff[j0 + j] = c;
+    }
+    __syncthreads();
+  }
   uint32_t kr[kRegKeys > 0 ? kRegKeys : 1];
   bool bad = false;
   {
@@ -141,16 +174,16 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(BatchDev b, const f
       }
       img = a0;
     }
-    auto key_of = [&](int t) -> uint32_t {
+    auto key_of = [&](int t, float st) -> uint32_t {  // st = s[t0 + t]
       float key;
       if (kQuota) {
-        key = s[t0 + t];
+        key = st;
         const float sh = key * c_seg;
         if (!isfinite(sh) || sh < 0.f || !isfinite(key) || key < 0.f) bad = true;
         if (s_hat) s_hat[t0 + t] = sh == 0.f ? 0.f : sh;
       } else {
         while (img + 1 < K && img_s[img + 1] <= t) ++img;
-        key = s[t0 + t] * c_s[img];
+        key = st * c_s[img];
         if (!isfinite(key) || key < 0.f) bad = true;
         if (s_hat) s_hat[t0 + t] = key == 0.f ? 0.f : key;
       }
@@ -159,9 +192,9 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(BatchDev b, const f
     };
     if (in_regs) {
 #pragma unroll
-      for (int j = 0; j < kRegKeys; ++j) kr[j] = (lo + j < hi) ? key_of(lo + j) : 0u;
+      for (int j = 0; j < kRegKeys; ++j) kr[j] = (lo + j < hi) ? key_of(lo + j, sv[j]) : 0u;
     } else {
-      for (int t = lo; t < hi; ++t) keys[t0 + t] = key_of(t);
+      for (int t = lo; t < hi; ++t) keys[t0 + t] = key_of(t, __ldcg(s + t0 + t));
     }
   }
   if (bad) flag_status(status, CONDUIT_FLAG_NONFINITE);
@@ -263,6 +296,81 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(BatchDev b, const f
       if (lo + j < hi) emit(lo + j, kr[j]);
   } else {
     for (int t = lo; t < hi; ++t) emit(t, keys[t0 + t]);
+  }
+}
+
+template <int kRegKeys, bool kQuota>
+__global__ void __launch_bounds__(kSelThreads) select_kernel(BatchDev b, const float* s,
+                                                             const float* g, float lambda,
+                                                             const int32_t* idx_off, int32_t* idx,
+                                                             uint8_t* mask, float* s_hat,
+                                                             float* coeff, uint32_t* keys,
+                                                             int32_t* status,
+                                                             const float* seg_coeff,
+                                                             const int32_t* seg_quota,
+                                                             const int32_t* seg_qoff) {
+  select_segment<kRegKeys, kQuota>(int(blockIdx.x), b, s, g, lambda, idx_off, idx, mask, s_hat, coeff, keys,
+                                   status, seg_coeff, seg_quota, seg_qoff);
+}
+
+// ------------------------------------------- scoring tail + selection, fused
+// conduit_score_select_topk's one launch after the scoring kernel, for
+// batches whose requests each fit one CTA's registers (at most 8 x 1024
+// tokens): block i first reduces tokens [32 i, 32 i + 32) over the layers
+// exactly as finalize_tokens_kernel does (s_t, A_t); then it counts itself in
+// on each request its tokens belong to (one arrival counter per request,
+// zeroed before the scoring kernel), and the block that arrives last for a
+// request takes that request's image means g_j (Eq. 8, each image by a group
+// of 256 threads in image_means_kernel's order), then c_j, s_hat and the
+// top-k exactly as select_kernel does. The selection of early requests runs
+// while later requests are still being reduced, and the results equal those
+// of the three separate launches bit for bit.
+template <int kRegKeys>
+__global__ void __launch_bounds__(kSelThreads) finalize_select_kernel(
+    TokenReduceArgs f, const __grid_constant__ LayerList layers, BatchDev b, float lambda,
+    const int32_t* idx_off, int32_t* idx, uint8_t* mask, float* s_hat, float* coeff, float* g,
+    int32_t* arrivals) {
+  __shared__ float part_s[kLayerSlots][33];
+  __shared__ float part_a[kLayerSlots][33];
+  __shared__ float mean_s[kSelThreads / kMeanThreads][kMeanThreads / 32];
+  __shared__ int done_s[kTokBlock + 1];  // requests this block completes, then their count
+  const int64_t tok0 = int64_t(blockIdx.x) * kTokBlock;
+  token_reduce_block(f, layers, b, tok0, part_s, part_a);
+  __syncthreads();  // this block's s and A are written
+  if (threadIdx.x == 0) {
+    // Each arrival releases this block's s and A (written before the barrier
+    // above) at device scope; the last arrival also acquires every other
+    // block's, and the barrier below passes them on to the block's threads.
+    const int64_t tok1 = min(tok0 + kTokBlock, f.n_tot);
+    int nd = 0;
+    for (int r = request_of(b.tok_off, b.R, tok0); r < b.R && b.tok_off[r] < tok1; ++r) {
+      const int blocks = (b.tok_off[r + 1] - 1) / kTokBlock - b.tok_off[r] / kTokBlock + 1;
+      int old;
+      asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], 1;" : "=r"(old) : "l"(arrivals + r) : "memory");
+      if (old == blocks - 1) done_s[nd++] = r;
+    }
+    done_s[kTokBlock] = nd;
+  }
+  __syncthreads();
+  const int nd = done_s[kTokBlock];
+  const int grp = threadIdx.x / kMeanThreads, gt = threadIdx.x % kMeanThreads;
+  for (int i = 0; i < nd; ++i) {
+    const int r = done_s[i];
+    const int j0 = b.req_img_off[r], j1 = b.req_img_off[r + 1];
+    if (j1 - j0 == 1) {  // one image: c = 1, so g is formed inside the selection, alongside its loads
+      select_segment<kRegKeys, false>(r, b, f.s, g, lambda, idx_off, idx, mask, s_hat, coeff, nullptr,
+                                      f.status, nullptr, nullptr, nullptr, f.attn_sum, &g[j0], f.n_layers);
+    } else {
+      // group grp takes images j0 + grp, j0 + grp + 4, ...; its 256 threads
+      // walk the same images, so its named barrier (id grp + 1) always completes
+      for (int j = j0 + grp; j < j1; j += kSelThreads / kMeanThreads)
+        image_mean_group(f.attn_sum, b.img_off[j], b.img_off[j + 1], f.n_layers, gt, mean_s[grp], &g[j],
+                         [grp] { asm volatile("bar.sync %0, %1;" ::"r"(grp + 1), "n"(kMeanThreads) : "memory"); });
+      __syncthreads();  // g_j of the request are written
+      select_segment<kRegKeys, false>(r, b, f.s, g, lambda, idx_off, idx, mask, s_hat, coeff, nullptr,
+                                      f.status, nullptr, nullptr, nullptr);
+    }
+    __syncthreads();  // the next request reuses the shared arrays
   }
 }
 
@@ -639,6 +747,40 @@ cudaError_t launch_select(const BatchDev& b, int max_tokens, const float* s, con
   else
     select_kernel<0, false><<<b.R, kSelThreads, 0, stream>>>(
         b, s, g, lambda, idx_off_dev, idx, mask, s_hat, coeff, keys, status, nullptr, nullptr, nullptr);
+  count_launches(1);
+  return cudaGetLastError();
+}
+
+// The fused tail pays one fence and one atomic per token block before the
+// block may retire; with more token blocks than SMs those waits queue up
+// wave after wave (batched serving: 4 096 blocks, 27 waves, 0.32 ms against
+// 0.28 ms for the three separate launches), so it is taken only when every
+// token block runs in the first wave.
+bool finalize_select_supported(int max_tokens, int64_t n_tot) {
+  if (max_tokens > 8 * kSelThreads) return false;
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return false;
+  return (n_tot + kTokBlock - 1) / kTokBlock <= sms;
+}
+
+cudaError_t launch_finalize_select(const float* pa, const float* pa2, const float* ss, const float* vnorm,
+                                   int vmode, const LayerList& layers, const BatchDev& b, int n_layers,
+                                   int Hkv, int Hq, int rg_max, int group_rows, int parts, int64_t n_tot,
+                                   int max_tokens, float* s, float* attn_sum, float* g, float lambda,
+                                   const int32_t* idx_off_dev, int32_t* idx, uint8_t* mask, float* s_hat,
+                                   float* coeff, int32_t* arrivals, int32_t* status, cudaStream_t stream) {
+  if (max_tokens > 8 * kSelThreads) return cudaErrorInvalidValue;
+  const TokenReduceArgs f{pa, pa2, ss, vnorm, vmode, n_layers, Hkv, Hq, rg_max, group_rows, parts,
+                          n_tot, s, attn_sum, status};
+  const unsigned blocks = unsigned((n_tot + kTokBlock - 1) / kTokBlock);
+  if (max_tokens <= kSelThreads)
+    finalize_select_kernel<1><<<blocks, kSelThreads, 0, stream>>>(f, layers, b, lambda, idx_off_dev, idx, mask,
+                                                                   s_hat, coeff, g, arrivals);
+  else
+    finalize_select_kernel<8><<<blocks, kSelThreads, 0, stream>>>(f, layers, b, lambda, idx_off_dev, idx, mask,
+                                                                   s_hat, coeff, g, arrivals);
   count_launches(1);
   return cudaGetLastError();
 }

@@ -3,6 +3,8 @@
 ``RefreshPipeline.step()`` enqueues, on one CUDA stream and through the C ABI:
   1. conduit_score        scoring pass over the reused visual cache (Eqs. 6-8)
   2. conduit_select_topk  amplification + one global top-k per request (Eqs. 9-11)
+     (steps 1 and 2 as one call, conduit_score_select_topk, which runs the
+     scoring tail and the selection as one launch)
   3. conduit_kv_exchange  stale K/V rows of the selected tokens out, fresh rows in
                           (conduit_kv_gather + conduit_kv_scatter in one launch)
   4. conduit_refresh_attn causal attention of the refreshed rows over the patched cache
@@ -69,10 +71,13 @@ class RefreshPipeline:
         self.vnorm = C.conduit_value_norms(self.kv, self.batch) if value_norm == "side_cache" else None
         self.plain = statistic == "mean" and value_norm == "v" and extra_lse is None
         opts = C.score_opts(statistic, value_norm, self.vnorm, extra_lse)
-        self.ws_score = torch.empty(max(C.conduit_score_ex_workspace_size(self.kv, self.batch, nl, opts), 1),
-                                    dtype=torch.uint8, device=dev)
         if selection not in ("global", "quota"):
             raise ValueError("selection must be 'global' or 'quota'")
+        # the fused call's workspace starts with the scoring call's, so one
+        # buffer serves conduit_score(_ex) and conduit_score_select_topk
+        ws_bytes = (C.conduit_score_select_topk_workspace_size if selection == "global"
+                    else C.conduit_score_ex_workspace_size)(self.kv, self.batch, nl, opts)
+        self.ws_score = torch.empty(max(ws_bytes, 1), dtype=torch.uint8, device=dev)
         self.selection = selection
         self.quota = torch.empty(K, dtype=torch.int32, device=dev) if selection == "quota" else None
         sel_ws = (C.conduit_select_quota_workspace_size if selection == "quota"
@@ -126,8 +131,16 @@ class RefreshPipeline:
                                self.q_rows, self.out, self.ws_ref, self.status, stream)
 
     def score_select(self, stream=None):
-        self.score(stream)
-        self.select(stream)
+        """Steps 1 and 2. With the global rule, one call (conduit_score_select_topk):
+        the same results as score() then select(), in fewer launches."""
+        if self.selection == "quota":
+            self.score(stream)
+            self.select(stream)
+            return
+        C.conduit_score_select_topk(self.kv, self.batch, self.q, self.lam, self.idx_off, self.idx_off_dev,
+                                    self.layers, self.statistic, self.value_norm, self.vnorm, self.extra_lse,
+                                    self.s, self.attn_sum, self.g, self.idx, self.mask, self.s_hat,
+                                    self.coeff, self.ws_score, self.status, stream)
 
     def refresh(self, stream=None):
         self.exchange(stream)
@@ -149,16 +162,16 @@ class RefreshPipeline:
     def step(self, stream=None):
         """One pass of the whole hot path (launches only; asynchronous)."""
         if self.graph is not None:
-            self._score_select_step()
-            self._refresh_step()
+            self.graph[2].replay()
             return
         self.score_select(stream)
         self.refresh(stream)
 
     def capture(self):
-        """Capture the step as two CUDA graphs (scoring and selection; exchange
-        and refresh), so that step_from_host can start the first while the
-        second's inputs are still arriving; later step() calls replay them."""
+        """Capture the step as CUDA graphs: scoring and selection, exchange and
+        refresh (step_from_host starts the first while the second's inputs are
+        still arriving), and the whole step in one graph, which later step()
+        calls replay (one graph launch per step)."""
         s = torch.cuda.Stream(device=self.device)
         s.wait_stream(torch.cuda.current_stream())
         with torch.cuda.stream(s):
@@ -166,12 +179,15 @@ class RefreshPipeline:
             self.refresh(s)
         torch.cuda.current_stream().wait_stream(s)
         torch.cuda.synchronize()
-        g1, g2 = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+        g1, g2, g3 = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
         with torch.cuda.graph(g1):
             self.score_select()
         with torch.cuda.graph(g2):
             self.refresh()
-        self.graph = (g1, g2)
+        with torch.cuda.graph(g3):
+            self.score_select()
+            self.refresh()
+        self.graph = (g1, g2, g3)
 
     # ------------------------------------------------------------- end to end
     def host_buffers(self) -> dict:

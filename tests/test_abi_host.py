@@ -38,7 +38,8 @@ def test_header_declares_the_boundary():
                  "conduit_score_with_norms", "conduit_score_with_norms_workspace_size",
                  "conduit_score_ex", "conduit_score_ex_workspace_size",
                  "conduit_select_quota", "conduit_select_quota_workspace_size",
-                 "conduit_staleness_iso", "conduit_staleness_iso_workspace_size"):
+                 "conduit_staleness_iso", "conduit_staleness_iso_workspace_size",
+                 "conduit_score_select_topk", "conduit_score_select_topk_workspace_size"):
         assert want in names
 
 
@@ -152,6 +153,33 @@ def test_select_rejects_bad_budgets_and_lambda(C):
     ws = torch.zeros(8, dtype=torch.uint8)
     _expect(C, C.ERR_WORKSPACE, C.conduit_select_topk, b, s, g, 1.0, off, off_d, None, None, None,
             None, ws)
+
+
+def test_score_select_rejects_bad_arguments(C):
+    """conduit_score_select_topk checks both calls' arguments before it enqueues anything."""
+    kv, b = _kv(C), _batch(C)
+    q = torch.zeros((2, 4, 8, 64), dtype=torch.bfloat16)
+    off, off_d = C.idx_offsets([10, 65], "cpu")          # 65 > 64 tokens of request 1
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_score_select_topk, kv, b, q, 1.0, off, off_d, match="budget")
+    off, off_d = C.idx_offsets([10, 5], "cpu")
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_score_select_topk, kv, b, q, 1.5, off, off_d, match="lambda")
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_score_select_topk, kv, b, None, 1.0, off, off_d)
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_score_select_topk, kv, b, q, 1.0, off, off_d, [1, 0],
+            match="increasing")
+    opts = C.score_opts()
+    opts.statistic = 7
+    n = ctypes.c_size_t(0)
+    assert C._lib.conduit_score_select_topk_workspace_size(kv.ref(), b.ref(), 0, ctypes.byref(opts),
+                                                           ctypes.byref(n)) == C.ERR_INVALID_ARG
+    bad = _batch(C, qo=(0, 0, 8))
+    _expect(C, C.ERR_INVALID_ARG, C.conduit_score_select_topk, kv, bad, q, 1.0, off, off_d,
+            match="scoring span")
+    # the workspace is the scoring call's plus a counter per request and the selection's keys
+    need = C.conduit_score_select_topk_workspace_size(kv, b)
+    assert need >= C.conduit_score_workspace_size(kv, b) + 256 + C.conduit_select_workspace_size(b)
+    ws = torch.zeros(need - 256, dtype=torch.uint8)
+    _expect(C, C.ERR_WORKSPACE, C.conduit_score_select_topk, kv, b, q, 1.0, off, off_d, None, "mean", "v",
+            None, None, None, None, None, None, None, None, None, ws)
 
 
 def test_quota_select_rejects_bad_arguments(C):
