@@ -4,9 +4,9 @@
 //
 // Work item: one query tile of 128 rows of one (layer, KV head, request),
 // floor(128/G) consecutive selected rows times the G query heads that share
-// the KV head. Keys stream in tiles of 128 (a tcgen05.mma costs about the same
-// issue time for N = 64 and N = 128, so wide tiles halve the instruction
-// count). The kernel is persistent: one CTA per SM takes items from an atomic
+// the KV head. Keys stream in tiles of 128 (the MMA thread, which shares its
+// sub-partition with two softmax warps, is paced per instruction, so wide
+// tiles halve its work). The kernel is persistent: one CTA per SM takes items from an atomic
 // counter, and the query tile of the next item loads into a second buffer
 // while the current item computes. Roles (352 threads):
 //   warp 0     TMA loads: the query tile of each item (a 3-D box of 64 dims x
