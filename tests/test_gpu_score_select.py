@@ -201,3 +201,19 @@ def test_ragged_case_against_the_oracle(C):
         # the selection is exact on the kernel's own keys (integer work)
         assert idx[off[r]:off[r + 1]].tolist() == O.topk_select(s_hat[t0:t1].astype(np.float64),
                                                                 budgets[r]).tolist()
+
+
+def test_non_finite_scores_flag_both_paths_alike(C):
+    """A NaN query makes its request's scores NaN: the fused call flags
+    CONDUIT_FLAG_NONFINITE as the separate calls do and returns the same bits."""
+    kv, batch, inputs = _ragged(C, [[200, 56], [1], [90]], [6, 2, 5], L=2)
+    q = inputs["q"].clone()
+    q[1, 3, 0, 5] = float("nan")                      # layer 1, head 3, request 0's first query
+    one, two = _both(C, kv, batch, q, 1.0, _budgets(batch, 0.2))
+    names = ("s", "attn_sum", "g", "idx", "mask", "s_hat", "coeff", "status")
+    for name, x, y in zip(names, one, two):
+        bits = lambda t: t.view(torch.int32) if t.dtype == torch.float32 else t
+        assert x.shape == y.shape and torch.equal(bits(x), bits(y)), name
+    assert int(one[-1].item()) & C.FLAG_NONFINITE and int(one[-1].item()) == int(two[-1].item())
+    tok = batch.tok_off.tolist()
+    assert torch.isnan(one[0][tok[0]:tok[1]]).all() and torch.isfinite(one[0][tok[1]:]).all()
