@@ -242,7 +242,8 @@ def _src_hash(src: str) -> str:
 def _traffic(call: str, workload: str, src: str):
     """DRAM bytes per launch from a committed ncu summary, if the kernel source is unchanged.
 
-    profiles/traffic.txt lines: <call> <workload> <bytes per launch> <sha256[:12] of the source>.
+    profiles/traffic.txt lines: <call> <workload> <bytes per launch> <sha256[:12] of the source>;
+    the workload is the config name, with @<ratio> when the run overrides the ratio.
     """
     p = os.path.join(ROOT, "profiles", "traffic.txt")
     if not os.path.exists(p):
@@ -416,7 +417,9 @@ def run_conduit(args):
         achieved, peak, unit = model[dom]["flops"] / sec / 1e12, ALU_FP32_TFLOPS, "TFLOP/s"
         peak_note = "fp32 FMA: 152 SMs x 128 lanes x 2 FLOP x 2.07 GHz"
     # committed ncu traffic covers the default scoring pass only
-    traffic = _traffic(dom, args.config, src) if pipe.plain and pipe.selection == "global" else None
+    # the workload key carries a ratio override (long document at r = 0.05 / 0.10 / 0.20)
+    wkey = args.config + (f"@{args.ratio:g}" if args.ratio is not None else "")
+    traffic = _traffic(dom, wkey, src) if pipe.plain and pipe.selection == "global" else None
     roofline = {"bound": bound, "achieved": round(achieved, 3), "peak": round(peak, 1), "unit": unit,
                 "frac": round(achieved / peak, 4), "traffic": traffic, "kernel": dom,
                 "kernels": kernels, "peak_source": peak_note,
