@@ -49,3 +49,23 @@ def test_reference_arm_line_on_the_cpu(capsys):
     assert line["config"] == bench.run_config(args, 256, 25, 1)
     assert 0 < line["ms_per_step"] <= line["extrapolated_full_step_ms"] * 1.5
     assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["value"] > 0
+
+
+def test_traffic_lines_match_the_committed_kernels():
+    """Every DRAM-traffic line under profiles/ names the source it was captured
+    from; the bench reports it only while that source is unchanged, so the
+    default (batched) line's dominant kernel must have a current capture."""
+    import os
+    src = {"score": "score_tc.cu", "refresh": "refresh_tc.cu"}
+    seen = set()
+    for line in open(os.path.join(bench.ROOT, "profiles", "traffic.txt")):
+        if line.startswith("#") or not line.strip():
+            continue
+        call, workload, nbytes, digest = line.split()[:4]
+        assert float(nbytes) > 0
+        got = bench._traffic(call, workload, src[call])
+        assert got == (float(nbytes) if digest == bench._src_hash(src[call]) else None)
+        if got is not None:
+            seen.add((call, workload))
+    assert ("refresh", "batched") in seen
+    assert bench._traffic("refresh", "batched@0.3", "refresh_tc.cu") is None   # no capture at that ratio
