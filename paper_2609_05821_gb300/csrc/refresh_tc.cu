@@ -74,6 +74,7 @@ struct RefArgs {
   const int32_t* idx_off;
   const __nv_bfloat16* q_rows;
   __nv_bfloat16* out;
+  int32_t out32;           // out is 32-byte aligned: rows are written in 32-byte stores
   int32_t n_sel;
   int32_t rows_per_tile;   // selected rows per query tile, floor(128 / G)
   int32_t n_blocks;        // query tiles per (layer, KV head)
@@ -581,20 +582,30 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc::tc_fence_after();
         const float inv = total > 0.f ? 1.f / total : 0.f;
         __nv_bfloat16* dst = a.out + ((int64_t(it.l) * a.n_sel + i_row) * Hq + h_row) * kD;
-        for (int c = hh * 64; c < hh * 64 + 64; c += 32) {
-          float o[32];
-          tc::tmem_ld32(tl + kOCol + c, o);
-          if (row_ok && p_row >= 0) {
+        // This thread's 64 columns of O in one load, then its half row as
+        // bf16. Each lane writes its own row, so a warp's store covers 32
+        // rows: 32-byte stores (whole sectors) when the buffer allows them.
+        float o[64];
+        tc::tmem_ld64(tl + kOCol + hh * 64, o);
+        if (row_ok && p_row >= 0) {
+          uint32_t w[32];
 #pragma unroll
-            for (int u4 = 0; u4 < 4; ++u4) {
-              uint32_t w4[4];
+          for (int k2 = 0; k2 < 32; ++k2) {
+            __nv_bfloat162 pr = __floats2bfloat162_rn(o[2 * k2] * inv, o[2 * k2 + 1] * inv);
+            w[k2] = *reinterpret_cast<uint32_t*>(&pr);
+          }
+          __nv_bfloat16* drow = dst + hh * 64;
+          if (a.out32) {
 #pragma unroll
-              for (int k2 = 0; k2 < 4; ++k2) {
-                __nv_bfloat162 pr = __floats2bfloat162_rn(o[u4 * 8 + 2 * k2] * inv, o[u4 * 8 + 2 * k2 + 1] * inv);
-                w4[k2] = *reinterpret_cast<uint32_t*>(&pr);
-              }
-              *reinterpret_cast<uint4*>(dst + c + u4 * 8) = make_uint4(w4[0], w4[1], w4[2], w4[3]);
-            }
+            for (int u8 = 0; u8 < 4; ++u8)
+              asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(drow + u8 * 16),
+                           "r"(w[8 * u8]), "r"(w[8 * u8 + 1]), "r"(w[8 * u8 + 2]), "r"(w[8 * u8 + 3]),
+                           "r"(w[8 * u8 + 4]), "r"(w[8 * u8 + 5]), "r"(w[8 * u8 + 6]), "r"(w[8 * u8 + 7])
+                           : "memory");
+          } else {
+#pragma unroll
+            for (int u4 = 0; u4 < 8; ++u4)
+              *reinterpret_cast<uint4*>(drow + u4 * 8) = make_uint4(w[4 * u4], w[4 * u4 + 1], w[4 * u4 + 2], w[4 * u4 + 3]);
           }
         }
       }
@@ -690,6 +701,7 @@ cudaError_t launch_refresh_tc(const KvDev& kv, const BatchDev& b, const int32_t*
   a.idx_off = idx_off_dev;
   a.q_rows = static_cast<const __nv_bfloat16*>(q_rows);
   a.out = static_cast<__nv_bfloat16*>(out);
+  a.out32 = (reinterpret_cast<uintptr_t>(out) & 31) == 0;
   a.n_sel = n_sel;
   a.rows_per_tile = kRows / kv.G;
   int blocks = 0;
