@@ -156,8 +156,12 @@ def barrier(world: int):
 
 
 # ------------------------------------------------------------ work models
-def work_model(pipe) -> dict:
-    """Algorithmic bytes / FLOPs of one step, per C-ABI call."""
+def work_model(pipe, idx_sets=None) -> dict:
+    """Algorithmic bytes / FLOPs of one step, per C-ABI call. The refresh
+    figures depend on the selected positions, which change from step to step
+    (each step's exchange rewrites the cache the next step scores): with
+    `idx_sets` (the selections of the timed calls) they are the mean over
+    those selections, else those of the selection now in `pipe.idx`."""
     kv, b = pipe.kv, pipe.batch
     esz = pipe.kv.k.element_size()
     L = kv.num_layers if pipe.layers is None else len(pipe.layers)
@@ -177,14 +181,19 @@ def work_model(pipe) -> dict:
     if pipe.selection == "quota":  # coefficients, quotas and offsets through the workspace
         sel_bytes += 2 * 12 * K
     copy_bytes = 2 * 2 * Lall * k_sel * Hkv * d * esz
-    idx = pipe.idx[:k_sel].cpu().tolist()
+    if not idx_sets:
+        idx_sets = [pipe.idx[:k_sel].cpu().tolist()]
     off = pipe.idx_off.tolist()
-    ref_flops, ref_bytes = 0, 2 * Lall * k_sel * Hq * d * esz  # the query rows in, the output out
-    for r in range(R):
-        ps = idx[off[r]:off[r + 1]]
-        ref_flops += sum(4 * Hq * d * (p + 1) for p in ps) * Lall
-        if ps:
-            ref_bytes += 2 * Lall * Hkv * (max(ps) + 1) * d * esz
+    ref_flops, ref_bytes = 0, 0
+    for idx in idx_sets:
+        for r in range(R):
+            ps = idx[off[r]:off[r + 1]]
+            ref_flops += sum(4 * Hq * d * (p + 1) for p in ps) * Lall
+            if ps:
+                ref_bytes += 2 * Lall * Hkv * (max(ps) + 1) * d * esz
+    ref_flops /= len(idx_sets)
+    ref_bytes /= len(idx_sets)
+    ref_bytes += 2 * Lall * k_sel * Hq * d * esz  # the query rows in, the output out
     out = {
         "score": {"bytes": score_bytes, "flops": score_flops},
         "select": {"bytes": sel_bytes, "flops": 0},
@@ -353,6 +362,7 @@ def run_conduit(args):
     seq.append(("refresh", pipe.refresh_attn))
     calls = {name: [] for name, _ in seq}
     stream = torch.cuda.current_stream()
+    idx_sets = []  # each timed refresh call's selection, read back after its events
     for _ in range(args.steps):
         flush()
         ev = [torch.cuda.Event(enable_timing=True) for _ in range(len(seq) + 1)]
@@ -363,6 +373,7 @@ def run_conduit(args):
         ev[-1].synchronize()
         for i, (name, _) in enumerate(seq):
             calls[name].append(ev[i].elapsed_time(ev[i + 1]))
+        idx_sets.append(pipe.idx[:pipe.n_sel].cpu().tolist())
     # the step runs scoring and selection as one call (conduit_score_select_topk)
     # under the global rule: timed the same way, on its own
     fused_ms = None
@@ -400,7 +411,7 @@ def run_conduit(args):
     status = C.conduit_read_status(pipe.status)
 
     # roofline of the dominant call
-    model = work_model(pipe)
+    model = work_model(pipe, idx_sets)
     dom = max(call_ms, key=call_ms.get)
     kernels, bound, src = call_kernels(pipe)[dom]
     if bound in ("hbm", "tensor"):

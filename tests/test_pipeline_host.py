@@ -80,3 +80,12 @@ def test_bench_work_model_matches_closed_forms(P):
     alone = P.from_inputs(_own(x), budgets=[k], value_norm="none")
     alone.idx[:k] = torch.tensor(sel, dtype=torch.int32)
     assert m["score"]["bytes"] - bench.work_model(alone)["score"]["bytes"] == L * Hkv * N * d * b
+    # over several timed calls (the cache, and so the selection, changes from
+    # step to step) the refresh work is the mean over their selections
+    sel2 = [0, 2, 4, 6, 8]
+    m2 = bench.work_model(pipe, [sel, sel2])
+    f1 = L * sum(4 * Hq * d * (p + 1) for p in sel)
+    f2 = L * sum(4 * Hq * d * (p + 1) for p in sel2)
+    assert m2["refresh"]["flops"] == (f1 + f2) / 2
+    assert m2["refresh"]["bytes"] == 2 * L * k * Hq * d * b + L * Hkv * (max(sel) + max(sel2) + 2) * d * b
+    assert m2["score"] == m["score"] and m2["exchange"] == m["exchange"]
