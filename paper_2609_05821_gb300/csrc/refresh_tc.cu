@@ -4,11 +4,12 @@
 //
 // Work item: one query tile of 128 rows of one (layer, KV head, request),
 // floor(128/G) consecutive selected rows times the G query heads that share
-// the KV head. Keys stream in tiles of 128 (the MMA thread, which shares its
-// sub-partition with two softmax warps, is paced per instruction, so wide
-// tiles halve its work). The kernel is persistent: one CTA per SM takes items from an atomic
-// counter, and the query tile of the next item loads into a second buffer
-// while the current item computes. Roles (352 threads):
+// the KV head. Keys stream in tiles of 128 (an MMA-issuing thread, which
+// shares its sub-partition with two softmax warps, is paced per instruction,
+// so wide tiles halve its work). The kernel is persistent: one CTA per SM
+// takes items from an atomic counter, and the query tile of the next item
+// loads into a second buffer while the current item computes. Roles (384
+// threads):
 //   warp 0     TMA loads: the query tile of each item (a 3-D box of 64 dims x
 //              G heads x floor(128/G) rows lands in the tile's row order) into
 //              one of two buffers, then its K tiles (two stages); the lanes
@@ -16,8 +17,11 @@
 //              paged)
 //   warp 10    the same for the V tiles (two stages), so that a V stage
 //              waiting for its P.V never holds back K and the next query tile
-//   warp 1     one thread issues tcgen05 MMAs: S(t) = Q K(t)^T into one of two
-//              TMEM buffers, O += P(t) V(t) with P read from TMEM
+//   warp 1     one thread issues S(t) = Q K(t)^T into TMEM buffer t % 3
+//   warp 11    one thread issues O += P(t) V(t) with P read from TMEM; two
+//              issuing threads, because one thread issuing both (with a wait
+//              for each P.V before the S that reuses its buffer) took longer
+//              per key tile than the softmax
 //   warps 2-9  softmax, two warps per TMEM lane quarter: each thread owns one
 //              row and one half (64 keys) of every key tile. Per tile it reads
 //              its half of S(t), applies the causal mask j <= p_i, exchanges
@@ -27,11 +31,13 @@
 //              warp-collective), writes its half of P as bf16 pairs over the
 //              upper half of S(t), and at the item's end writes its half of
 //              O / rowsum
-// TMEM: S buffers at columns [0, 128) and [128, 256) (P in the upper 64 of
-// each), O at [256, 384). S(t+1) is computed while the softmax works on
-// S(t); S(t+2) reuses the buffer of P(t), so it is issued once P(t) V(t) has
-// completed; the next item's first S tiles are computed while the softmax
-// writes the previous item's O. Rows are sorted by position, so an item needs
+// TMEM: three S buffers at columns [0, 384) (P in the upper 64 of each), O at
+// [384, 512). S(t) reuses the buffer of P(t-3), so it is issued once
+// P(t-3) V(t-3) has completed (per-buffer completion barriers): the S thread
+// runs up to two tiles ahead of the softmax, which finds S(t+1) ready when it
+// finishes P(t) and probes for it without suspending; the next item's first
+// S tiles are computed while the softmax writes the previous item's O. Rows
+// are sorted by position, so an item needs
 // keys up to its last row's position only. Every barrier phase follows from
 // per-CTA sequence numbers (items n, key tiles T) that all roles advance
 // alike. Every wait is bounded by one second; a role that gives up raises an
@@ -50,7 +56,8 @@ constexpr int kKT = 128;                         // keys per tile
 constexpr int kRows = 128;                       // rows per query tile
 constexpr int kSoftThreads = 256;
 constexpr int kVWarp = 10;                       // after the loader, MMA and eight softmax warps
-constexpr int kThreads = 64 + kSoftThreads + 32;
+constexpr int kPvWarp = 11;                      // the thread issuing O += P V
+constexpr int kThreads = 64 + kSoftThreads + 64;
 constexpr int kKStages = 2;
 constexpr int kVStages = 2;
 constexpr int kQBufs = 2;
@@ -61,10 +68,11 @@ constexpr uint32_t kTileBytes = 2 * kTileHalf;   // 32 KB
 constexpr int kRecInts = 9;                      // decoded item record (see Smem::rec)
 constexpr uint32_t kSmem = 1024 + kQBufs * kQBytes + (kKStages + kVStages) * kTileBytes + 256 +
                            2 * 2 * 128 * 4 + 2 * 128 * 4 + kQBufs * (kRecInts + kRows) * 4;
-constexpr uint32_t kTmemCols = 512;              // 384 used; allocations are powers of two
+constexpr uint32_t kTmemCols = 512;              // three S / P buffers and O
 constexpr uint32_t kSCols = 128;                 // one S buffer
+constexpr int kSBufs = 3;                        // S runs up to two key tiles ahead of the softmax
 constexpr uint32_t kPCol = 64;                   // P (bf16 pairs) over the upper half of S
-constexpr uint32_t kOCol = 256;                  // O
+constexpr uint32_t kOCol = kSBufs * kSCols;      // O
 constexpr float kRescaleLog2 = 8.f;
 
 struct RefArgs {
@@ -135,11 +143,11 @@ struct Smem {
   uint8_t* v;        // [kVStages][2 halves][128 keys][128 B]
   uint64_t *kfull, *kempty;   // [kKStages]
   uint64_t *vfull, *vempty;   // [kVStages]
-  uint64_t *sfull, *pfull;    // [2] per S buffer
-  uint64_t *pvdone;           // once per key tile
+  uint64_t *sfull, *pfull;    // [kSBufs] per S buffer
+  uint64_t *pvdone;           // [kSBufs] per S buffer: the P.V that read its P has completed
   uint64_t *qfull, *qempty;   // [kQBufs] query tile (and item index) of one item
   uint64_t *ofull, *oempty;   // once per item: O complete / O read out
-  uint64_t *mdone;
+  uint64_t *mdone;            // [2] per MMA thread: all its MMAs completed
   uint32_t* tmem_slot;
   volatile int* abort;
   uint32_t* counters;  // [0] K loads, [1] V loads, [2] K consumed, [3] V consumed
@@ -165,14 +173,14 @@ __device__ __forceinline__ Smem carve(uint8_t* raw) {
   s.vfull = s.kempty + kKStages;
   s.vempty = s.vfull + kVStages;
   s.sfull = s.vempty + kVStages;
-  s.pfull = s.sfull + 2;
-  s.pvdone = s.pfull + 2;
-  s.qfull = s.pvdone + 1;
+  s.pfull = s.sfull + kSBufs;
+  s.pvdone = s.pfull + kSBufs;
+  s.qfull = s.pvdone + kSBufs;
   s.qempty = s.qfull + kQBufs;
   s.ofull = s.qempty + kQBufs;
   s.oempty = s.ofull + 1;
   s.mdone = s.oempty + 1;
-  s.tmem_slot = reinterpret_cast<uint32_t*>(s.mdone + 1);
+  s.tmem_slot = reinterpret_cast<uint32_t*>(s.mdone + 2);
   s.abort = reinterpret_cast<volatile int*>(s.tmem_slot + 1);
   s.counters = reinterpret_cast<uint32_t*>(s.tmem_slot + 2);
   s.xmax = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bar) + 256);
@@ -180,6 +188,20 @@ __device__ __forceinline__ Smem carve(uint8_t* raw) {
   s.rec = reinterpret_cast<volatile int*>(s.xsum + 2 * 128);
   s.pos = s.rec + kQBufs * kRecInts;
   return s;
+}
+
+// Non-blocking test of the phase with the given parity (no suspension): for
+// the softmax's wait on S, which the S thread has usually completed already.
+// Waits that are often not yet complete (the MMA threads') use wait_or_abort
+// alone: a probe in front of them cost more than it saved.
+__device__ __forceinline__ bool mbar_probe(uint64_t* bar, uint32_t parity) {
+  uint32_t done;
+  asm volatile(
+      "{\n.reg .pred p;\nmbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\nselp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(done)
+      : "r"(tc::smem_u32(bar)), "r"(parity)
+      : "memory");
+  return done != 0;
 }
 
 __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int* abort) {
@@ -257,20 +279,22 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::mbar_init(&s.vfull[i], 1);
       tc::mbar_init(&s.vempty[i], 1);
     }
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < kSBufs; ++i) {
       tc::mbar_init(&s.sfull[i], 1);
       // per buffer, so the softmax can never be two phases ahead of the MMA's
-      // wait: P(t+2) needs S(t+2), issued only after the wait for P(t)
+      // wait: P(t+3) needs S(t+3), issued only after P(t) V(t) has completed
       tc::mbar_init(&s.pfull[i], kSoftThreads);
+      tc::mbar_init(&s.pvdone[i], 1);
     }
     for (int i = 0; i < kQBufs; ++i) {
       tc::mbar_init(&s.qfull[i], 1);   // the loader's expect-tx (or plain arrive at the end)
-      tc::mbar_init(&s.qempty[i], 3);  // the MMA thread's commit + the softmax and V warps' reads of the item
+      // the S thread's commit + the P.V thread's, softmax's and V warp's reads of the item
+      tc::mbar_init(&s.qempty[i], 4);
     }
-    tc::mbar_init(s.pvdone, 1);
     tc::mbar_init(s.ofull, 1);
     tc::mbar_init(s.oempty, kSoftThreads);
-    tc::mbar_init(s.mdone, 1);
+    tc::mbar_init(&s.mdone[0], 1);
+    tc::mbar_init(&s.mdone[1], 1);
     *s.abort = 0;
     for (int i = 0; i < 4; ++i) s.counters[i] = 0;
     tc::fence_barrier_init();
@@ -379,28 +403,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     if (lane == 0) s.counters[1] = nv;
   } else if (warp == 1 && lane == 0) {
-    // ------------------------------------------------------------------ MMA
-    uint32_t ck = 0, cv = 0, T = 0;
-    bool ok = true, any_pv = false;
+    // ---------------------------------------------------------- MMA: S = Q K^T
+    // S(t) goes to buffer t % kSBufs once P(t-3) V(t-3), which read that
+    // buffer's P, has completed (possibly of an earlier item); so this thread
+    // runs up to two tiles ahead of the P.V thread
+    uint32_t ck = 0, T = 0;
+    bool ok = true;
     const uint32_t idesc_s = tc::idesc_bf16(kRows, kKT);
-    const uint32_t idesc_o = tc::idesc_bf16(kRows, kD, /*b_mn_major=*/true);
-    // S(T) = Q K(T)^T into S buffer T & 1
-    auto issue_s = [&](uint32_t q_addr, uint32_t Ts) -> bool {
-      const int sk = Ts % kKStages;
-      if (!wait_or_abort(&s.kfull[sk], (Ts / kKStages) & 1, s.abort)) return false;
-      ++ck;
-      tc::tc_fence_after();
-      const uint32_t k_addr = tc::smem_u32(s.k + sk * kTileBytes);
-#pragma unroll
-      for (int kk = 0; kk < 8; ++kk) {
-        const uint32_t off = (kk & 3) * 32;
-        tc::mma_bf16(tmem + (Ts & 1) * kSCols, tc::desc_sw128(q_addr + (kk >> 2) * kQHalf + off),
-                     tc::desc_sw128(k_addr + (kk >> 2) * kTileHalf + off), idesc_s, kk > 0);
-      }
-      tc::mma_commit(&s.sfull[Ts & 1]);
-      tc::mma_commit(&s.kempty[sk]);
-      return true;
-    };
     for (uint32_t n = 0; ok; ++n) {
       const int qs = n & 1;
       if (!wait_or_abort(&s.qfull[qs], (n >> 1) & 1, s.abort)) { ok = false; break; }
@@ -408,46 +417,71 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int nt = s.rec[qs * kRecInts + 6];
       const uint32_t q_addr = tc::smem_u32(s.q + qs * kQBytes);
       tc::tc_fence_after();
-      // the S buffers are free once the previous item's last P.V has completed
-      // (the latest pvdone commit, so its parity cannot alias)
-      if (any_pv && nt > 0 && !wait_or_abort(s.pvdone, (T - 1) & 1, s.abort)) { ok = false; break; }
-      if (nt > 0 && !issue_s(q_addr, T)) { ok = false; break; }
-      if (nt > 1 && !issue_s(q_addr, T + 1)) { ok = false; break; }
-      if (nt <= 2) tc::mma_commit(&s.qempty[qs]);  // every S of this item is issued
+      for (int t = 0; t < nt; ++t) {
+        const uint32_t Ts = T + t;
+        const int b = Ts % kSBufs, sk = Ts % kKStages;
+        if (Ts >= uint32_t(kSBufs) && !wait_or_abort(&s.pvdone[b], ((Ts / kSBufs) - 1) & 1, s.abort)) {
+          ok = false;
+          break;
+        }
+        if (!wait_or_abort(&s.kfull[sk], (Ts / kKStages) & 1, s.abort)) { ok = false; break; }
+        ++ck;
+        tc::tc_fence_after();
+        const uint32_t k_addr = tc::smem_u32(s.k + sk * kTileBytes);
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk) {
+          const uint32_t off = (kk & 3) * 32;
+          tc::mma_bf16(tmem + b * kSCols, tc::desc_sw128(q_addr + (kk >> 2) * kQHalf + off),
+                       tc::desc_sw128(k_addr + (kk >> 2) * kTileHalf + off), idesc_s, kk > 0);
+        }
+        tc::mma_commit(&s.sfull[b]);
+        tc::mma_commit(&s.kempty[sk]);
+      }
+      if (!ok) break;
+      tc::mma_commit(&s.qempty[qs]);  // every S of this item is issued
+      T += nt;
+    }
+    if (!ok) raise_abort(a, s, tc::kSiteMma);
+    s.counters[2] = ck;
+    tc::mma_commit(&s.mdone[0]);  // every MMA issued above has completed once this arrives
+    tc::mbar_wait(&s.mdone[0], 0);
+  } else if (warp == kPvWarp && lane == 0) {
+    // -------------------------------------------------------- MMA: O += P V
+    uint32_t cv = 0, T = 0;
+    bool ok = true;
+    const uint32_t idesc_o = tc::idesc_bf16(kRows, kD, /*b_mn_major=*/true);
+    for (uint32_t n = 0; ok; ++n) {
+      const int qs = n & 1;
+      if (!wait_or_abort(&s.qfull[qs], (n >> 1) & 1, s.abort)) { ok = false; break; }
+      const int u = s.rec[qs * kRecInts], nt = s.rec[qs * kRecInts + 6];
+      tc::mbar_arrive(&s.qempty[qs]);  // this thread is done with the record
+      if (u < 0) break;
       for (int t = 0; t < nt; ++t) {
         const uint32_t Tc = T + t;
-        const int sv = Tc % kVStages;
+        const int b = Tc % kSBufs, sv = Tc % kVStages;
         if (!wait_or_abort(&s.vfull[sv], (Tc / kVStages) & 1, s.abort)) { ok = false; break; }
         ++cv;
-        if (!wait_or_abort(&s.pfull[Tc & 1], (Tc >> 1) & 1, s.abort)) { ok = false; break; }
+        if (!wait_or_abort(&s.pfull[b], (Tc / kSBufs) & 1, s.abort)) { ok = false; break; }
         // O of the previous item must have been read out before P(0) V(0) overwrites it
         if (t == 0 && n > 0 && !wait_or_abort(s.oempty, (n - 1) & 1, s.abort)) { ok = false; break; }
         tc::tc_fence_after();
         const uint32_t v_addr = tc::smem_u32(s.v + sv * kTileBytes);
-        const uint32_t pb = tmem + (Tc & 1) * kSCols + kPCol;
+        const uint32_t pb = tmem + b * kSCols + kPCol;
 #pragma unroll
         for (int kk = 0; kk < kKT / 16; ++kk)  // O += P(t) V(t)
           tc::mma_bf16_ts(tmem + kOCol, pb + kk * 8, tc::desc_sw128_mn(v_addr + kk * 2048, kTileHalf),
                           idesc_o, t > 0 || kk > 0);
-        tc::mma_commit(s.pvdone);
+        tc::mma_commit(&s.pvdone[b]);
         tc::mma_commit(&s.vempty[sv]);
-        any_pv = true;
-        if (t + 2 < nt) {
-          // S(t+2) overwrites P(t): wait until P(t) V(t) has completed
-          if (!wait_or_abort(s.pvdone, Tc & 1, s.abort)) { ok = false; break; }
-          if (!issue_s(q_addr, Tc + 2)) { ok = false; break; }
-          if (t + 3 == nt) tc::mma_commit(&s.qempty[qs]);  // that was the item's last S
-        }
       }
       if (!ok) break;
       T += nt;
       tc::mma_commit(s.ofull);  // O of this item is complete once this arrives
     }
     if (!ok) raise_abort(a, s, tc::kSiteMma);
-    s.counters[2] = ck;
     s.counters[3] = cv;
-    tc::mma_commit(s.mdone);  // every MMA issued above has completed once this arrives
-    tc::mbar_wait(s.mdone, 0);
+    tc::mma_commit(&s.mdone[1]);
+    tc::mbar_wait(&s.mdone[1], 0);
   } else if (warp >= 2 && warp < kVWarp) {
     // -------------------------------------------------------------- softmax
     const int et = tid - 64;                             // 0..255
@@ -487,9 +521,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       float m_ref = -INFINITY, lsum = 0.f;  // running max (scaled, log2 units, same in both halves) and half-row sum
       for (int t = 0; t < nt; ++t) {
         const uint32_t Tc = T + t;
-        const uint32_t sb = tl + (Tc & 1) * kSCols;
+        const uint32_t sbuf = Tc % kSBufs;
+        const uint32_t sb = tl + sbuf * kSCols;
         // the tcgen05.ld below is warp-collective: the whole warp goes on or stops
-        const bool gs = __all_sync(0xffffffffu, ok && wait_or_abort(&s.sfull[Tc & 1], (Tc >> 1) & 1, s.abort));
+        const bool gs = __all_sync(0xffffffffu, ok && (mbar_probe(&s.sfull[sbuf], (Tc / kSBufs) & 1) ||
+                                                       wait_or_abort(&s.sfull[sbuf], (Tc / kSBufs) & 1, s.abort)));
         if (!gs) {
           if (ok) raise_abort(a, s, tc::kSiteMma);
           ok = false;
@@ -546,10 +582,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         lsum += (ls[0] + ls[1]) + (ls[2] + ls[3]);
         if (__any_sync(0xffffffffu, need) && t > 0) {
           // P(t-1) V(t-1) must have completed before this warp rescales its half
-          // of O. S(t) was issued after P(t-2) V(t-2) completed, so pvdone is at
-          // most one phase behind here and its parity cannot alias; P(t) V(t)
-          // waits for this warp's pfull arrival below.
-          if (!__all_sync(0xffffffffu, wait_or_abort(s.pvdone, (Tc - 1) & 1, s.abort))) {
+          // of O. That buffer's next P.V needs a P this softmax has not written
+          // yet, so the barrier's parity cannot alias; P(t) V(t) waits for this
+          // warp's pfull arrival below.
+          if (!__all_sync(0xffffffffu,
+                          wait_or_abort(&s.pvdone[(Tc - 1) % kSBufs], ((Tc - 1) / kSBufs) & 1, s.abort))) {
             raise_abort(a, s, tc::kSiteMma);
             ok = false;
             continue;
@@ -564,7 +601,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
         tc::tc_fence_before();
-        tc::mbar_arrive(&s.pfull[Tc & 1]);
+        tc::mbar_arrive(&s.pfull[sbuf]);
       }
       T += nt;
       // row sum = the two halves' sums (same running max in both)
