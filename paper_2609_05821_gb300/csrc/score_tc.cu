@@ -164,6 +164,19 @@ __device__ __forceinline__ Smem carve(uint8_t* raw) {
 }
 
 // Bounded wait that also gives up when another role has aborted.
+// Non-blocking test of the phase with the given parity (no suspension): for
+// the epilogue's waits on an accumulator slot, which the MMA thread has
+// usually filled already.
+__device__ __forceinline__ bool mbar_probe(uint64_t* bar, uint32_t parity) {
+  uint32_t done;
+  asm volatile(
+      "{\n.reg .pred p;\nmbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\nselp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(done)
+      : "r"(tc::smem_u32(bar)), "r"(parity)
+      : "memory");
+  return done != 0;
+}
+
 __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int* abort) {
   if (tc::mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = tc::globaltimer_ns();
@@ -489,7 +502,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int i = 0; i < w.tiles; ++i) {            // pass A
         const int slot = tseq & 1;
         // tcgen05.ld is warp-collective: the whole warp goes on or stops
-        const bool got = __all_sync(0xffffffffu, ok && wait_or_abort(&s.tfull[slot], (tseq >> 1) & 1, s.abort));
+        const bool got = __all_sync(0xffffffffu, ok && (mbar_probe(&s.tfull[slot], (tseq >> 1) & 1) ||
+                                                        wait_or_abort(&s.tfull[slot], (tseq >> 1) & 1, s.abort)));
         ++tseq;
         if (!got) {
           if (ok && !*s.abort) raise_abort(a, s, tc::kSiteMma);
@@ -553,7 +567,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int slot = tseq & 1;
         const int tok = tile_of(w, i) * kTile + lrow;
         // tcgen05.ld is warp-collective: the whole warp goes on or stops
-        const bool got = __all_sync(0xffffffffu, ok && wait_or_abort(&s.tfull[slot], (tseq >> 1) & 1, s.abort));
+        const bool got = __all_sync(0xffffffffu, ok && (mbar_probe(&s.tfull[slot], (tseq >> 1) & 1) ||
+                                                        wait_or_abort(&s.tfull[slot], (tseq >> 1) & 1, s.abort)));
         ++tseq;
         if (!got) {
           if (ok && !*s.abort) raise_abort(a, s, tc::kSiteMma);
