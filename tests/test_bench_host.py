@@ -53,8 +53,8 @@ def test_reference_arm_line_on_the_cpu(capsys):
 
 def test_traffic_lines_match_the_committed_kernels():
     """Every DRAM-traffic line under profiles/ names the source it was captured
-    from; the bench reports it only while that source is unchanged, so the
-    default (batched) line's dominant kernel must have a current capture."""
+    from; the bench reports it only while that source is unchanged, so every
+    line must have been captured from the current kernel sources."""
     import os
     src = {"score": "score_tc.cu", "refresh": "refresh_tc.cu"}
     seen = set()
@@ -67,5 +67,9 @@ def test_traffic_lines_match_the_committed_kernels():
         assert got == (float(nbytes) if digest == bench._src_hash(src[call]) else None)
         if got is not None:
             seen.add((call, workload))
-    assert ("refresh", "batched") in seen
+    # the four workloads' refresh lines and the scoring lines of the large ones
+    # were all captured from the current sources
+    for key in [("refresh", w) for w in ("batched", "multi", "single", "longdoc@0.1")] + \
+               [("score", w) for w in ("batched", "multi", "longdoc@0.1")]:
+        assert key in seen, key
     assert bench._traffic("refresh", "batched@0.3", "refresh_tc.cu") is None   # no capture at that ratio
